@@ -1,0 +1,458 @@
+"""Pins of the CPU oracle to facts outside the oracle itself (no GPU).
+
+Each test checks the oracle against something the paper or the mathematics
+fixes: published tables (Max 1960, splitmix64), closed forms (d = 3 uniform
+marginal, 1-bit centroid), independent numerical integration, Monte Carlo over
+random unit vectors, byte counts printed in the paper (Sec. II-B, Table I),
+invariants of the filtered search (Sec. III-B) and brute force on tiny inputs.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy import integrate, special, stats
+
+import oracle as O
+from paper_2607_16973_gb300 import synth
+from conftest import GOLDEN
+
+
+# ---------------------------------------------------------------- fixtures ---
+def _read_max_table():
+    rows = {}
+    with open(os.path.join(GOLDEN, "max1960_gaussian.txt")) as f:
+        for line in f:
+            if line.startswith("#") or not line.strip():
+                continue
+            parts = line.split()
+            L, kind, vals = int(parts[0]), parts[1], [float(v) for v in parts[2:]]
+            rows.setdefault(L, {})[kind] = vals
+    return rows
+
+
+def _coord_density(d):
+    """Textbook density of one coordinate of a uniform random unit vector in
+    R^d, written here independently of the oracle."""
+    logc = math.lgamma(d / 2) - math.lgamma((d - 1) / 2) - 0.5 * math.log(math.pi)
+    return lambda x: math.exp(logc + (d - 3) / 2 * math.log1p(-x * x)) if abs(x) < 1 else 0.0
+
+
+def _random_unit_rows(n, d, seed):
+    g = np.random.default_rng(seed).standard_normal((n, d))
+    return g / np.linalg.norm(g, axis=1, keepdims=True)
+
+
+# ---------------------------------------------------------------- codebook ---
+@pytest.mark.parametrize("L", [2, 4, 8, 16])
+def test_gaussian_codebook_matches_max_1960(L):
+    """Sec. II-B step 3 with the N(0, 1/d) marginal at d = 1 is Max's table."""
+    tab = _read_max_table()[L]
+    cb = O.codebook(1, int(math.log2(L)), "gauss")
+    half = cb.centroids[L // 2:]
+    assert np.allclose(half, tab["y"], atol=6e-4, rtol=0)
+    assert np.allclose(cb.boundaries[L // 2 - 1:], tab["x"], atol=6e-4, rtol=0)
+    assert cb.distortion == pytest.approx(tab["D"][0], rel=1e-3)
+
+
+def test_gaussian_codebook_scales_with_sqrt_d():
+    unit = O.codebook(1, 4, "gauss")
+    cb = O.codebook(1536, 4, "gauss")
+    assert np.allclose(cb.centroids * math.sqrt(1536), unit.centroids, rtol=1e-11, atol=1e-12)
+    assert cb.distortion * 1536 == pytest.approx(unit.distortion, rel=1e-10)
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 4])
+def test_beta_d3_is_uniform_quantiser(bits):
+    """At d = 3 the coordinate marginal is uniform on [-1, 1] (Archimedes), so
+    Lloyd-Max is the uniform quantiser: c_i = (2i+1)/L - 1, D = (2/L)^2 / 12."""
+    L = 1 << bits
+    cb = O.codebook(3, bits, "beta")
+    i = np.arange(L)
+    assert np.allclose(cb.centroids, (2 * i + 1) / L - 1, atol=1e-13)
+    assert np.allclose(cb.boundaries, 2 * (i[:-1] + 1) / L - 1, atol=1e-13)
+    assert cb.distortion == pytest.approx((2 / L) ** 2 / 12, rel=1e-10)
+
+
+@pytest.mark.parametrize("d", [4, 10, 100, 1536])
+def test_beta_one_bit_centroid_by_quadrature(d):
+    """1-bit Lloyd-Max of a symmetric density: t = 0, c = E[x | x > 0]."""
+    f = _coord_density(d)
+    hi = min(1.0, 12 / math.sqrt(d))
+    mass = integrate.quad(f, 0, hi, epsabs=0, epsrel=1e-13, limit=200)[0]
+    mom = integrate.quad(lambda x: x * f(x), 0, hi, epsabs=0, epsrel=1e-13, limit=200)[0]
+    cb = O.codebook(d, 1, "beta")
+    assert cb.boundaries[0] == 0.0
+    assert cb.centroids[1] == pytest.approx(mom / mass, rel=1e-10)
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_beta_centroids_are_conditional_means(bits):
+    """Lloyd-Max fixed point: each centroid is the mean of its cell, checked by
+    adaptive quadrature of the density (independent of the closed forms)."""
+    d = 1536
+    f = _coord_density(d)
+    cb = O.codebook(d, bits, "beta")
+    edges = np.concatenate([[-12 / math.sqrt(d)], cb.boundaries, [12 / math.sqrt(d)]])
+    for i, c in enumerate(cb.centroids):
+        a, b = edges[i], edges[i + 1]
+        m0 = integrate.quad(f, a, b, epsabs=0, epsrel=1e-12, limit=200)[0]
+        m1 = integrate.quad(lambda x: x * f(x), a, b, epsabs=0, epsrel=1e-12, limit=200)[0]
+        assert c == pytest.approx(m1 / m0, rel=1e-9, abs=1e-14)
+    total = integrate.quad(f, -1, 1, epsabs=0, epsrel=1e-12, points=[0.0], limit=400)[0]
+    assert total == pytest.approx(1.0, abs=1e-10)
+
+
+def test_beta_marginal_is_coordinate_of_random_unit_vector():
+    """Monte Carlo: one coordinate of uniform unit vectors in R^64 follows the
+    marginal the oracle integrates (KS bound at 99.9%)."""
+    d = 64
+    x = np.sort(_random_unit_rows(100_000, d, 1)[:, 0])
+    edges = np.concatenate([[-1.0], x])
+    cdf = np.cumsum(O.cell_moments(edges, d, "beta")[0])
+    emp_hi = np.arange(1, len(x) + 1) / len(x)
+    ks = max(np.max(np.abs(emp_hi - cdf)), np.max(np.abs(emp_hi - 1 / len(x) - cdf)))
+    assert ks < 1.95 / math.sqrt(len(x))
+
+
+@pytest.mark.parametrize("bits", [2, 4])
+def test_distortion_matches_monte_carlo(bits):
+    """Per-coordinate MSE of nearest-centroid quantisation of random unit
+    vectors equals the integrated distortion D."""
+    d = 1536
+    cb = O.codebook(d, bits, "beta")
+    y = _random_unit_rows(1500, d, 2).ravel()
+    near = cb.centroids[np.argmin(np.abs(y[:, None] - cb.centroids[None, :]), axis=1)]
+    mse = np.mean((y - near) ** 2)
+    assert mse == pytest.approx(cb.distortion, rel=0.01)
+
+
+def test_beta_tends_to_gaussian():
+    """The Beta marginal converges to N(0, 1/d) (Sec. II-B step 2)."""
+    errs = []
+    for d in (1536, 100_000):
+        b = O.codebook(d, 4, "beta").centroids * math.sqrt(d)
+        g = O.codebook(d, 4, "gauss").centroids * math.sqrt(d)
+        errs.append(np.max(np.abs(b - g)))
+    assert 0 < errs[0] < 5e-3
+    assert errs[1] < errs[0] / 30
+
+
+@pytest.mark.parametrize("marginal", ["beta", "gauss"])
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_codebook_structure(marginal, bits):
+    cb = O.codebook(1536, bits, marginal)
+    c, t = cb.centroids, cb.boundaries
+    assert np.all(np.diff(c) > 0)
+    assert np.array_equal(c, -c[::-1])
+    assert np.array_equal(t, (c[:-1] + c[1:]) / 2)
+    assert t[len(t) // 2] == 0.0
+    # Sec. V-A / VI: the codebook takes no corpus data: repeated calls agree bit for bit
+    cb2 = O.codebook(1536, bits, marginal)
+    assert np.array_equal(cb.centroids, cb2.centroids)
+
+
+def test_golden_codebooks_are_oracle_output():
+    with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+        g = json.load(f)
+    for e in g["entries"]:
+        if e["bits"] > 4:
+            c = np.asarray(e["centroids"])
+            assert np.all(np.diff(c) > 0) and np.allclose(c, -c[::-1], atol=0)
+            continue
+        cb = O.codebook(e["d"], e["bits"], e["marginal"])
+        assert np.allclose(cb.centroids, e["centroids"], rtol=1e-12, atol=0)
+        assert np.allclose(cb.boundaries, e["boundaries"], rtol=1e-12, atol=1e-300)
+
+
+def test_golden_8bit_distortion_matches_monte_carlo():
+    with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+        g = json.load(f)
+    e = [e for e in g["entries"] if e["bits"] == 8 and e["marginal"] == "beta"][0]
+    c = np.asarray(e["centroids"])
+    t = np.asarray(e["boundaries"])
+    y = _random_unit_rows(600, 1536, 3).ravel()
+    near = c[np.searchsorted(t, y)]
+    assert np.mean((y - near) ** 2) == pytest.approx(e["distortion"], rel=0.02)
+
+
+# ---------------------------------------------------------------- rotation ---
+def test_splitmix64_published_sequence():
+    with open(os.path.join(GOLDEN, "splitmix64.txt")) as f:
+        lines = [l.split() for l in f if l.strip() and not l.startswith("#")]
+    seed = int(lines[0][1])
+    want = [int(l[0]) for l in lines[1:]]
+    got = O.splitmix64(seed, np.arange(len(want)))
+    assert [int(v) for v in got] == want
+
+
+def test_gaussian_matrix_is_standard_normal():
+    g = O.gaussian_matrix(256, 11).ravel()
+    assert abs(g.mean()) < 5 / math.sqrt(g.size)
+    assert g.var() == pytest.approx(1.0, abs=0.02)
+    assert stats.kstest(g, "norm").pvalue > 1e-3
+
+
+@pytest.mark.parametrize("d", [32, 96, 1536])
+def test_rotation_orthogonal_and_qr_of_its_gaussian(d):
+    R = O.rotation(d, 1536)
+    assert np.max(np.abs(R @ R.T - np.eye(d))) < 1e-12
+    U = R.T @ O.gaussian_matrix(d, 1536)     # G = R U, U upper triangular, diag > 0
+    assert np.max(np.abs(np.tril(U, -1))) < 1e-9 * np.max(np.abs(U))
+    assert np.all(np.diag(U) > 0)
+    R32 = R.astype(np.float32).astype(np.float64)
+    assert np.max(np.abs(R32 @ R32.T - np.eye(d))) < 1e-6
+    x = synth.gaussian_rows(50, d, 3).astype(np.float64)
+    assert np.max(np.abs(np.linalg.norm(x @ R32.T, axis=1) - np.linalg.norm(x, axis=1))
+                  / np.linalg.norm(x, axis=1)) < 1e-6
+
+
+def test_rotation_seeded():
+    assert np.array_equal(O.rotation(64, 5), O.rotation(64, 5))
+    assert not np.allclose(O.rotation(64, 5), O.rotation(64, 6))
+
+
+def test_rotated_coordinates_follow_marginal():
+    """After the rotation each coordinate of a fixed unit vector is distributed
+    as the marginal: check E[y^2] = 1/d and the fourth moment 3/(d(d+2))."""
+    d = 96
+    x = np.zeros(d)
+    x[0] = 1.0
+    ys = np.array([O.rotation(d, s) @ x for s in range(300)]).ravel()
+    assert np.mean(ys ** 2) == pytest.approx(1 / d, rel=0.05)
+    assert np.mean(ys ** 4) == pytest.approx(3 / (d * (d + 2)), rel=0.12)
+
+
+# ---------------------------------------------------------------- packing ----
+def test_pack_layout_by_hand():
+    assert O.pack(np.array([[1, 2, 3, 4]]), 4).tolist() == [[0x21, 0x43]]
+    assert O.pack(np.array([[1, 2, 3, 0]]), 2).tolist() == [[1 | 2 << 2 | 3 << 4]]
+    assert O.pack(np.array([[1, 2, 3, 4, 5, 6, 7, 0]]), 3).tolist() == [[0xD1, 0x58, 0x1F]]
+    assert O.pack(np.array([[7, 255, 0, 128]]), 8).tolist() == [[7, 255, 0, 128]]
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 4, 5, 8])
+def test_pack_round_trip(bits):
+    rng = np.random.default_rng(bits)
+    codes = rng.integers(0, 1 << bits, size=(7, 64))
+    packed = O.pack(codes, bits)
+    assert packed.shape == (7, 64 * bits // 8)
+    assert np.array_equal(O.unpack(packed, 64, bits), codes)
+
+
+def test_sizes_printed_in_paper():
+    with open(os.path.join(GOLDEN, "paper_sizes.txt")) as f:
+        rows = [l.split() for l in f if l.strip() and not l.startswith("#")]
+    for r in rows:
+        if r[0] == "vector":
+            assert O.row_bytes(int(r[1]), int(r[2])) == int(r[3])
+        elif r[0] == "vector_fp32":
+            assert int(r[1]) * int(r[2]) // 8 == int(r[3])
+        else:
+            n, bits, mb = int(r[1]), int(r[2]), float(r[3])
+            total = n * O.row_bytes(1536, bits) / 1e6
+            assert total == pytest.approx(mb, abs=0.5 + 1e-9)
+
+
+# ---------------------------------------------------------------- encode -----
+@pytest.fixture(scope="module")
+def small_index():
+    d, n, bits = 256, 3000, 4
+    X = synth.mixture_corpus(n, d, 32, seed=9)
+    R = O.rotation(d, 1536).astype(np.float32)
+    cb = O.codebook(d, bits)
+    return X, R, cb, d, bits
+
+
+def test_code_is_count_of_boundaries_below(small_index):
+    X, R, cb, d, bits = small_index
+    enc = O.encode(X[:200], R, cb.centroids32, cb.boundaries32, bits)
+    y32 = enc.y.astype(np.float32)
+    literal = (y32[:, :, None] > cb.boundaries32[None, None, :]).sum(-1)
+    assert np.array_equal(enc.codes, literal)
+    # ... which is the nearest centroid (boundaries are midpoints)
+    near = np.argmin(np.abs(enc.y[:, :, None] - cb.centroids[None, None, :]), axis=-1)
+    assert np.mean(near == enc.codes) > 0.9999
+
+
+@pytest.mark.parametrize("bits", [2, 4])
+def test_reconstruction_mse_equals_distortion(bits):
+    """Sec. II-B: per-vector reconstruction error of x/||x|| equals d * D."""
+    d = 1536
+    X = synth.mixture_corpus(2000, d, 64, seed=42)
+    R = O.rotation(d, 1536).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits, "none")
+    xhat = O.decode(enc.packed, np.ones(len(X), np.float32), R, cb.centroids32, d, bits)
+    err = np.sum((X / np.linalg.norm(X, axis=1, keepdims=True) - xhat) ** 2, axis=1)
+    assert np.mean(err) == pytest.approx(d * cb.distortion, rel=0.02)
+
+
+def test_zero_row_and_scales(small_index):
+    X, R, cb, d, bits = small_index
+    X = X[:50].copy()
+    X[3] = 0.0
+    X[7] *= 3.5
+    for mode in O.SCALE_MODES:
+        enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits, mode)
+        assert np.all(enc.codes[3] == (1 << bits) // 2 - 1) and enc.scale[3] == 0.0
+        c = cb.centroids32.astype(np.float64)[enc.codes]
+        n = np.linalg.norm(X.astype(np.float64), axis=1)
+        rows = np.arange(len(X)) != 3
+        if mode == "none":
+            assert np.allclose(enc.scale[rows], n[rows], rtol=1e-7)
+        elif mode == "norm":    # reconstruction keeps the length of x
+            assert np.allclose(enc.scale[rows] * np.linalg.norm(c[rows], axis=1), n[rows], rtol=1e-6)
+        else:                   # unbiased: the self inner product is exact
+            self_ip = enc.scale * np.sum((X.astype(np.float64) @ R.astype(np.float64).T) * c, axis=1)
+            assert np.allclose(self_ip[rows], n[rows] ** 2, rtol=1e-6)
+
+
+# ---------------------------------------------------------------- search -----
+def _brute_force_topk(Q, R, centroids, bits, packed, scale, d, k, allowed=None):
+    """Pure-Python loops straight from the definitions (Sec. II-B step 5)."""
+    out = []
+    for q in Q.astype(np.float64):
+        qr = [sum(float(R[i, j]) * q[j] for j in range(d)) for i in range(d)]
+        scored = []
+        for v in range(packed.shape[0]):
+            bitpos, s = 0, 0.0
+            for j in range(d):
+                code = 0
+                for t in range(bits):
+                    byte = packed[v, (bitpos + t) // 8]
+                    code |= ((int(byte) >> ((bitpos + t) % 8)) & 1) << t
+                bitpos += bits
+                s += qr[j] * float(centroids[code])
+            if allowed is None or allowed[v]:
+                scored.append((-np.float32(s * float(scale[v])), v))
+        scored.sort()
+        out.append([v for _, v in scored[:k]])
+    return out
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+def test_search_brute_force_tiny(bits):
+    d, n, k = 32, 60, 7
+    X = synth.mixture_corpus(n, d, 4, seed=5)
+    R = O.rotation(d, 77).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    Q = synth.perturb(X[[1, 20, 33]], seed=3)
+    res = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
+    want = _brute_force_topk(Q, R, cb.centroids32, bits, enc.packed, enc.scale, d, k)
+    assert res.ids.tolist() == want
+
+
+def test_quantised_scores_error_matches_distortion():
+    """<q, x_hat> - <q, x> has variance ~ D |q|^2: ties the search score to the
+    codebook's distortion (wrong rotation orientation would break it)."""
+    d = 1536
+    X = synth.mixture_corpus(1500, d, 64, seed=42)
+    R = O.rotation(d, 1536).astype(np.float32)
+    for bits in (4, 8):
+        if bits == 8:
+            with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+                e = [e for e in json.load(f)["entries"] if e["bits"] == 8 and e["marginal"] == "beta"][0]
+            c32 = np.asarray(e["centroids"], np.float32)
+            t32 = np.asarray(e["boundaries"], np.float32)
+            D = e["distortion"]
+        else:
+            cb = O.codebook(d, bits)
+            c32, t32, D = cb.centroids32, cb.boundaries32, cb.distortion
+        enc = O.encode(X, R, c32, t32, bits, "none")
+        Q = synth.perturb(X[:20], seed=4)
+        S = O.quantized_scores(Q, R, c32, bits, enc.packed, enc.scale, d)
+        E = Q.astype(np.float64) @ X.astype(np.float64).T
+        assert np.mean((S - E) ** 2) == pytest.approx(D, rel=0.15)
+
+
+def test_search_recall_high_at_8_bits():
+    d, n = 1536, 3000
+    X = synth.mixture_corpus(n, d, 64, seed=42)
+    R = O.rotation(d, 1536).astype(np.float32)
+    with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+        e = [e for e in json.load(f)["entries"] if e["bits"] == 8 and e["marginal"] == "beta"][0]
+    c32, t32 = np.asarray(e["centroids"], np.float32), np.asarray(e["boundaries"], np.float32)
+    enc = O.encode(X, R, c32, t32, 8)
+    src = synth.query_sources(n, 30)
+    Q = synth.perturb(X[src], sigma=0.1, per_coordinate=False)
+    res = O.search(Q, R, c32, 8, enc.packed, enc.scale, 10, d)
+    ex, _ = O.exact_knn(X, Q, 10)
+    assert O.recall_at_k(res.ids, ex) > 0.95
+    assert np.all(res.ids[:, 0] == ex[:, 0]) or O.recall_at_k(res.ids[:, :1], ex[:, :1]) > 0.9
+
+
+@pytest.fixture(scope="module")
+def tenant_index():
+    d, n, bits, T = 64, 800, 4, 10
+    X = synth.mixture_corpus(n, d, 8, seed=12)
+    R = O.rotation(d, 3).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    tid, values = synth.zipf_tenants(n, T)
+    src = synth.query_sources(n, 12)
+    Q = synth.perturb(X[src])
+    return X, R, cb, enc, tid, values, src, Q, d, bits
+
+
+def test_filter_all_tenants_equals_unfiltered(tenant_index):
+    X, R, cb, enc, tid, values, src, Q, d, bits = tenant_index
+    off = np.arange(len(Q) + 1) * len(values)
+    ids = np.tile(values, len(Q))
+    a = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d, tid, off, ids)
+    b = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d)
+    assert np.array_equal(a.ids, b.ids) and np.array_equal(a.scores, b.scores)
+
+
+def test_filter_one_tenant_equals_subset_search(tenant_index):
+    """Sec. III-B: filtering inside the scan returns what searching only the
+    allowed vectors returns (no over-fetch loss)."""
+    X, R, cb, enc, tid, values, src, Q, d, bits = tenant_index
+    off, ids = synth.allowlists(src, tid, values, frac_multi=0.0)
+    filt = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d, tid, off, ids)
+    for q in range(len(Q)):
+        keep = np.nonzero(tid == ids[off[q]])[0]
+        sub = O.search(Q[q:q + 1], R, cb.centroids32, bits, enc.packed[keep], enc.scale[keep], 10, d)
+        got = sub.ids[0]
+        remapped = np.where(got >= 0, keep[np.maximum(got, 0)], -1)
+        assert np.array_equal(remapped, filt.ids[q])
+
+
+def test_filter_underfull_and_empty(tenant_index):
+    X, R, cb, enc, tid, values, src, Q, d, bits = tenant_index
+    smallest = values[-1]
+    cnt = int(np.sum(tid == smallest))
+    off = np.array([0, 1, 1], dtype=np.int64)
+    ids = np.array([smallest], dtype=np.uint32)
+    res = O.search(Q[:2], R, cb.centroids32, bits, enc.packed, enc.scale, cnt + 5, d, tid, off, ids)
+    assert np.all(res.ids[0, :cnt] >= 0) and np.all(res.ids[0, cnt:] == -1)
+    assert np.all(np.isneginf(res.scores[0, cnt:]))
+    assert np.all(res.ids[1] == -1)
+
+
+def test_ties_break_by_id():
+    d, bits = 32, 2
+    X = synth.mixture_corpus(10, d, 2, seed=1)
+    X = np.concatenate([X, X[[3, 3, 5]]])
+    R = O.rotation(d, 2).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    res = O.search(X[[3]], R, cb.centroids32, bits, enc.packed, enc.scale, 4, d)
+    top = res.ids[0].tolist()
+    assert top[:3] == [3, 10, 11]
+
+
+def test_exact_knn_and_recall_definitions():
+    X = synth.mixture_corpus(40, 32, 3, seed=8)
+    Q = synth.perturb(X[:4], seed=1)
+    ids, sc = O.exact_knn(X, Q, 5)
+    for q in range(4):
+        s = [float(np.dot(Q[q].astype(np.float64), X[v].astype(np.float64))) for v in range(40)]
+        want = sorted(range(40), key=lambda v: (-s[v], v))[:5]
+        assert ids[q].tolist() == want
+    assert O.recall_at_k(ids, ids) == 1.0
+    wrong = ids.copy()
+    wrong[:, -1] = -1
+    assert O.recall_at_k(wrong, ids) == pytest.approx(4 / 5)
