@@ -1,0 +1,457 @@
+#!/usr/bin/env python
+"""Benchmark of the TurboQuant search path on GB300 (one JSON line on stdout).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config scale|c2|tiny] [--batches 1,1024] [--k 5]
+
+Workload (default "scale"): N = 999,000 synthetic L2-normalised d = 1536
+vectors (1,024-cluster Gaussian mixture, seed 42), rotated by a seeded Haar R
+and encoded to 4-bit codes (767.2 MB packed) on the GPU; 10,000
+perturbed-corpus queries; top-5 by inner product.  A step is one search of a
+batch of B queries through tq_search: query rotation, the scan with fused
+top-k, and the merge (Sec. II-B step 5).  Inputs are resident in HBM when the
+timed region starts; the 767 MB corpus is larger than the 129 MB L2, so every
+step streams it from HBM.  The headline `value` is queries/s at the first batch
+size; every batch size measured is reported under "batches".
+
+--impl reference times the CPU oracle (float64 numpy) on the host cores on a
+bounded sample of the same workload.  Under torchrun every rank runs an
+independent replica (the search path needs no collective), the timed region is
+bracketed by barriers and the slowest rank's time is used.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+CONFIGS = {
+    # name: corpus size, dim, bits, clusters, query pool, k, batch sizes
+    "scale": dict(n=999_000, d=1536, bits=4, clusters=1024, pool=10_000, k=5, batches=[1, 1024]),
+    "c2": dict(n=100_000, d=1536, bits=4, clusters=256, pool=1_000, k=10, batches=[1, 256]),
+    "tiny": dict(n=10_000, d=1536, bits=4, clusters=64, pool=100, k=10, batches=[1, 100]),
+}
+
+METRIC = "queries/sec at 999Kx1536 4-bit top-5 (batch 1 / 1024); % of HBM / TC roofline"
+
+
+# ------------------------------------------------------------------ helpers --
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p["bf16_tflops_sustained"]), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def source_hash(*files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel_file: str, profile_md: str):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current kernel source (the summary records the source hash)."""
+    path = os.path.join(ROOT, "profiles", profile_md)
+    if not os.path.exists(path):
+        return None
+    want = source_hash(kernel_file)
+    got_hash, traffic = None, None
+    with open(path) as f:
+        for line in f:
+            if line.startswith("source_sha256_16:"):
+                got_hash = line.split(":", 1)[1].strip()
+            if line.startswith("dram_bytes_per_launch:"):
+                traffic = float(line.split(":", 1)[1].strip())
+    return traffic if got_hash == want else None
+
+
+class ClockSampler:
+    """Samples SM clock and clock-event reasons during the timed region, via
+    NVML (read-only queries), else `nvidia-smi -lms`."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+               0x2: "applications_clocks_setting"}
+
+    def __init__(self, pci_bus_id: str | None, index: int):
+        self.samples, self.reasons, self.max_mhz = [], set(), None
+        self._stop = threading.Event()
+        self._nvml = None
+        self._dev = ctypes.c_void_p()
+        self._index = index
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit")
+            ok = -1
+            if pci_bus_id:
+                ok = nv.nvmlDeviceGetHandleByPciBusId_v2(pci_bus_id.encode(), ctypes.byref(self._dev))
+            if ok != 0:
+                ok = nv.nvmlDeviceGetHandleByIndex_v2(index, ctypes.byref(self._dev))
+            if ok != 0:
+                raise OSError("nvml handle")
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(self._dev, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = mx.value
+            self._nvml = nv
+        except OSError:
+            self._nvml = None
+
+    def _loop_nvml(self):
+        nv = self._nvml
+        mhz = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        getr = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(self._dev, 1, ctypes.byref(mhz)) == 0:
+                self.samples.append(mhz.value)
+            if getr(self._dev, ctypes.byref(rs)) == 0:
+                for bit, name in self.REASONS.items():
+                    if rs.value & bit:
+                        self.reasons.add(name)
+            time.sleep(0.002)
+
+    def _loop_smi(self):
+        cmd = ["nvidia-smi", "-i", str(self._index), "--query-gpu=clocks.sm,clocks.max.sm,"
+               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+               "--format=csv,noheader,nounits", "-lms", "200"]
+        try:
+            self._proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, text=True)
+        except OSError:
+            return
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self._proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            try:
+                self.samples.append(int(parts[0]))
+                self.max_mhz = int(parts[1])
+                for nm, v in zip(names, parts[2:]):
+                    if v.lower().startswith("active"):
+                        self.reasons.add(nm)
+            except (ValueError, IndexError):
+                pass
+            if self._stop.is_set():
+                break
+
+    def __enter__(self):
+        self._t = threading.Thread(target=self._loop_nvml if self._nvml else self._loop_smi, daemon=True)
+        self._t.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        if getattr(self, "_proc", None) is not None:
+            self._proc.terminate()
+        self._t.join(timeout=2)
+
+    def summary(self):
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                "samples": len(self.samples), "source": "nvml" if self._nvml else "nvidia-smi"}
+
+
+# --------------------------------------------------------------- workloads --
+def make_corpus(cfg, workers):
+    from paper_2607_16973_gb300 import synth
+    t0 = time.time()
+    X = synth.mixture_corpus(cfg["n"], cfg["d"], cfg["clusters"], workers=workers)
+    src = synth.query_sources(cfg["n"], cfg["pool"])
+    Q = synth.perturb(X[src])
+    log(f"[bench] generated corpus {X.shape} + {len(Q)} queries in {time.time() - t0:.1f}s")
+    return X, Q
+
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    return os.cpu_count() or 1
+
+
+def oracle_qps_sample(cfg, sample_rows: int, n_queries: int, seconds_cap: float = 30.0):
+    """Times the oracle's search of single queries over a bounded sample of
+    the corpus rows (encoded by the oracle itself) and scales to the full
+    corpus.  Returns (qps_full, info)."""
+    import oracle as O
+    from paper_2607_16973_gb300 import synth
+    d, bits, k = cfg["d"], cfg["bits"], cfg["k"]
+    X = synth.mixture_rows(0, sample_rows, d, cfg["clusters"], workers=8)
+    R = O.rotation(d, synth.SEED_ROTATION).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    Q = synth.perturb(X[synth.query_sources(sample_rows, n_queries)])
+    times = []
+    t_start = time.time()
+    for q in range(n_queries):
+        t0 = time.perf_counter()
+        O.search(Q[q:q + 1], R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
+        times.append(time.perf_counter() - t0)
+        if time.time() - t_start > seconds_cap:
+            break
+    per_q_sample = statistics.median(times)
+    per_q_full = per_q_sample * cfg["n"] / sample_rows
+    return 1.0 / per_q_full, {
+        "sample": f"oracle search (float64 numpy) of {len(times)} single queries over the first "
+                  f"{sample_rows} of {cfg['n']} corpus rows, median time scaled by {cfg['n']}/{sample_rows}",
+        "per_query_s_sample": per_q_sample}
+
+
+# -------------------------------------------------------------- reference --
+def run_reference(args, cfg, rank, world):
+    if world > 1 and rank != 0:
+        return
+    import oracle as O
+    from paper_2607_16973_gb300 import synth
+    d, bits, k = cfg["d"], cfg["bits"], cfg["k"]
+    sample_rows = min(cfg["n"], args.ref_sample)
+    X = synth.mixture_rows(0, sample_rows, d, cfg["clusters"], workers=8)
+    R = O.rotation(d, synth.SEED_ROTATION).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    Q = synth.perturb(X[synth.query_sources(sample_rows, max(args.steps + args.warmup, 1))])
+    B = 1
+    for i in range(args.warmup):
+        O.search(Q[i:i + 1], R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        j = args.warmup + i
+        O.search(Q[j:j + 1], R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
+    el = time.perf_counter() - t0
+    scale_up = cfg["n"] / sample_rows
+    per_step_full = el / max(args.steps, 1) * scale_up
+    qps = B / per_step_full
+    cores = cpu_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": qps, "unit": "queries/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_full * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": f"{args.config}: N={cfg['n']} d={d} {bits}-bit top-{k}, batch 1",
+                   "n": cfg["n"], "d": d, "bits": bits, "k": k, "batch": 1},
+        "cpu_baseline": {"value": qps, "unit": "queries/s", "cores": cores, "kind": "oracle",
+                         "sample": f"each step: oracle search of 1 query over the first {sample_rows} "
+                                   f"rows, time scaled by {cfg['n']}/{sample_rows}"},
+        "e2e": {"value": qps, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------- ours ----
+def run_ours(args, cfg, rank, world):
+    import torch
+    import paper_2607_16973_gb300 as tq
+    from paper_2607_16973_gb300 import synth
+    from paper_2607_16973_gb300.build import build
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+    build()
+    tq.load()
+    d, bits, k, n = cfg["d"], cfg["bits"], cfg["k"], cfg["n"]
+    batches = [int(b) for b in args.batches.split(",")] if args.batches else cfg["batches"]
+    if args.k:
+        k = args.k
+    stream = torch.cuda.Stream(device=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    # ---- index build: codebook + rotation on the host, encode on the GPU
+    X, Qpool = make_corpus(cfg, workers=min(16, os.cpu_count() or 4))
+    cen, bnd, _ = tq.codebook(d, bits)
+    R = tq.rotation(d, synth.SEED_ROTATION)
+    with torch.cuda.stream(stream):
+        Xd = torch.from_numpy(X).to(dev, non_blocking=False)
+        Rd = torch.from_numpy(R).to(dev)
+        cd = torch.from_numpy(cen).to(dev)
+        bd = torch.from_numpy(bnd).to(dev)
+        codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
+        scale = torch.empty(n, dtype=torch.float32, device=dev)
+        Qd = torch.from_numpy(Qpool).to(dev)
+    del X
+    barrier()
+    enc_ms = []
+    for i in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream)
+        e1.record(stream)
+        e1.synchronize()
+        enc_ms.append(e0.elapsed_time(e1))
+    enc_ms = min(enc_ms[1:])
+    del Xd
+    torch.cuda.empty_cache()
+    log(f"[bench] encode {n} vectors: {enc_ms:.1f} ms ({n / enc_ms * 1e3:.3g} vec/s)")
+
+    pk = peaks()
+    pci = None
+    try:
+        pr = torch.cuda.get_device_properties(dev)
+        pci = f"{pr.pci_domain_id:08X}:{pr.pci_bus_id:02X}:{pr.pci_device_id:02X}.0"
+    except Exception:
+        pci = None
+    results = {}
+    for B in batches:
+        nbatches = max(1, len(Qpool) // B)
+        ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
+        ids = torch.empty((B, k), dtype=torch.int64, device=dev)
+        scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+
+        def step(i):
+            j = (i % nbatches) * B
+            tq.search(Qd[j:j + B], Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids,
+                      out_scores=scs, stream=stream)
+
+        for i in range(args.warmup):
+            step(i)
+        # scan-kernel events recorded inside the timed loop
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        with ClockSampler(pci, local) as clk:
+            t0.record(stream)
+            for i in range(args.steps):
+                tq.profile_events(*evs[i])
+                step(args.warmup + i)
+            t1.record(stream)
+            t1.synchronize()
+        tq.profile_events(None, None)
+        barrier()
+        ms = t0.elapsed_time(t1)
+        if world > 1:
+            tt = torch.tensor([ms], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            ms = float(tt.item())
+        scan_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
+        qps = B * args.steps * world / (ms / 1e3)
+        # roofline of the scan kernel: the corpus (codes + scales) read once per launch
+        alg_bytes = n * (d * bits // 8 + 4)
+        achieved = alg_bytes / (scan_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
+                "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu",
+                                            f"scan_lut_{n // 1000}k_b{B}.md"),
+                "kernel": "k_scan_lut", "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
+                "frac_of_8tbs_nominal": achieved / 8000.0}
+        # e2e through the public API with host buffers
+        qh = torch.empty((B, d), dtype=torch.float32).pin_memory()
+        qh.copy_(torch.from_numpy(Qpool[:B]))
+        qdev = torch.empty((B, d), dtype=torch.float32, device=dev)
+        ih = torch.empty((B, k), dtype=torch.int64).pin_memory()
+        sh = torch.empty((B, k), dtype=torch.float32).pin_memory()
+        with torch.cuda.stream(stream):
+            for _ in range(max(1, args.warmup)):
+                tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
+                                    out_ids=ids, out_scores=scs, stream=stream)
+            barrier()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(args.steps):
+                tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
+                                    out_ids=ids, out_scores=scs, stream=stream)
+            b.record(stream)
+            b.synchronize()
+        e2e_ms = a.elapsed_time(b)
+        results[B] = {
+            "value": qps, "ms_per_step": ms / args.steps, "roofline": roof, "clocks": clk.summary(),
+            "e2e": {"value": B * args.steps * world / (e2e_ms / 1e3), "unit": "queries/s",
+                    "h2d_bytes_per_step": B * d * 4, "d2h_bytes_per_step": B * k * 12},
+        }
+        log(f"[bench] B={B}: {qps:.4g} q/s, {ms / args.steps:.3f} ms/step, scan {scan_ms:.3f} ms "
+            f"= {achieved:.0f} GB/s ({100 * achieved / pk['hbm_gbs']:.1f}% of {pk['source']} HBM)")
+        del ws
+
+    head = batches[0]
+    r = results[head]
+    line = {
+        "metric": METRIC, "value": r["value"], "unit": "queries/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded Gaussian-mixture corpus, perturbed-corpus queries)",
+        "config": {"workload": f"{args.config}: N={n} d={d} {bits}-bit top-{k}, batch {head}, "
+                               f"codes {n * d * bits // 8 / 1e6:.1f} MB resident in HBM",
+                   "n": n, "d": d, "bits": bits, "k": k, "batch": head,
+                   "l2": "inputs larger than L2 (corpus streamed from HBM every step)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
+        "gpu_launches": 3 * args.steps,
+        "batches": {str(b): {"value": v["value"], "ms_per_step": v["ms_per_step"],
+                             "roofline": v["roofline"], "e2e": v["e2e"]} for b, v in results.items()},
+        "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
+                   "tflops": 2.0 * n * d * d / (enc_ms / 1e3) / 1e12},
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        qps_cpu, info = oracle_qps_sample(cfg, sample_rows=min(n, args.ref_sample), n_queries=5)
+        line["cpu_baseline"] = {"value": qps_cpu, "unit": "queries/s", "cores": cpu_threads(),
+                                "kind": "oracle", "sample": info["sample"]}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", choices=sorted(CONFIGS), default="scale")
+    ap.add_argument("--batches", default=None, help="comma-separated batch sizes (first = headline)")
+    ap.add_argument("--k", type=int, default=None)
+    ap.add_argument("--ref-sample", type=int, default=100_000, help="corpus rows the oracle scans")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    cfg = CONFIGS[args.config]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, cfg, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        dist.init_process_group("nccl")
+    run_ours(args, cfg, rank, world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,208 @@
+/*
+ * tq.h - C ABI of the GB300 TurboQuant search library (libtq.so).
+ *
+ * The library implements the data-parallel hot path of TurboQuant as studied
+ * in "TurboVec: A Case Study in Cost-Efficient Private Retrieval for
+ * Enterprise RAG via Codebook-Oblivious Quantization" (arXiv 2607.16973):
+ *
+ *   Sec. II-B, steps 1-5: normalise (keep the norm), rotate by a fixed random
+ *     orthogonal R, quantise every coordinate with a Lloyd-Max codebook derived
+ *     from the analytic coordinate marginal (no corpus data), bit-pack, and
+ *     score with a per-vector length-renormalisation scalar;
+ *   Sec. III-A/III-B: flat (brute-force) top-k inner-product search with an
+ *     allowlist of tenants passed to the scan; blocks with no allowed vector
+ *     are skipped before scoring, disallowed vectors in scored blocks never
+ *     enter the top-k;
+ *   Sec. III-C: the add() / search() / search(allowlist) operations.
+ *
+ * Conventions shared by every call:
+ *  - Sizes are element counts.  d must be a multiple of 32 with 32 <= d <= 8192;
+ *    bits is 2, 3, 4 or 8.
+ *  - "host" pointers are ordinary CPU memory; "device" pointers are CUDA device
+ *    memory of the current device, owned by the caller, which must keep them
+ *    alive until the work queued on `stream` has finished.  Device pointers
+ *    must be 16-byte aligned.
+ *  - Device calls are asynchronous and stream-ordered on `stream` (a
+ *    cudaStream_t passed as void*; NULL is the legacy default stream).  They
+ *    validate every argument before queueing any work.
+ *  - Errors: every call returns a tq_status.  TQ_EINVAL for invalid arguments
+ *    (nothing is queued), TQ_ECUDA when the CUDA runtime reports an error,
+ *    TQ_ENOMEM when a library-owned allocation fails, TQ_EUNSUPPORTED for a
+ *    valid request this build cannot serve.  tq_last_error() returns a
+ *    thread-local message for the last non-OK status of the calling thread.
+ *    No call aborts, prints or lets a C++ exception escape.
+ *  - Packed codes: row i holds d*bits/8 bytes, a little-endian bit stream in
+ *    which coordinate j occupies bits [bits*j, bits*j + bits).  At d = 1536,
+ *    bits = 4 that is 768 bytes per vector (Sec. II-B step 4).
+ */
+#ifndef TQ_H
+#define TQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum tq_status {
+  TQ_OK = 0,
+  TQ_EINVAL = 1,
+  TQ_ENOMEM = 2,
+  TQ_ECUDA = 3,
+  TQ_ETIMEOUT = 4,
+  TQ_EUNSUPPORTED = 5
+} tq_status;
+
+/* Coordinate marginal the codebook is fitted to (Sec. II-A: "Beta/Gaussian
+ * marginals after random rotation"; Sec. II-B step 3). */
+enum { TQ_MARGINAL_BETA = 0, TQ_MARGINAL_GAUSS = 1 };
+
+/* Per-vector scoring scalar (Sec. II-B step 5, "length-renormalized scoring"):
+ *  NORM      scale = ||x|| / ||c[code]||   (reconstruction keeps the length of x)
+ *  NONE      scale = ||x||                 (no renormalisation)
+ *  UNBIASED  scale = ||x|| / <y, c[code]>  (self inner product is exact)
+ * A zero row gets scale 0 in every mode. */
+enum { TQ_SCALE_NORM = 0, TQ_SCALE_NONE = 1, TQ_SCALE_UNBIASED = 2 };
+
+/* Search kernels: AUTO picks by batch size; LUT forces the per-query lookup
+ * scan, MMA forces the tensor-core decode-GEMM scan (used by tests). */
+enum { TQ_PATH_AUTO = 0, TQ_PATH_LUT = 1, TQ_PATH_MMA = 2 };
+
+typedef struct tq_filter tq_filter; /* opaque, library-owned */
+
+/* Thread-local, NUL-terminated message describing the calling thread's last
+ * non-OK status; "" if none.  The pointer stays valid until the next call. */
+const char* tq_last_error(void);
+
+/* ABI version of this header (major * 100 + minor). */
+int tq_version(void);
+
+/*
+ * tq_codebook - Lloyd-Max scalar quantiser of the rotated-coordinate marginal
+ * (Sec. II-B step 3; Sec. II-A: derived analytically, no corpus-dependent
+ * training).  Host-only, deterministic, takes no data.
+ *   d          dimension (>= 8); selects the marginal f_d(x) proportional to
+ *              (1 - x^2)^((d-3)/2) on [-1, 1] (BETA) or N(0, 1/d) (GAUSS)
+ *   bits       1..8; L = 2^bits levels
+ *   marginal   TQ_MARGINAL_BETA or TQ_MARGINAL_GAUSS
+ *   centroids  host out [L], ascending, symmetric (c_i = -c_{L-1-i})
+ *   boundaries host out [L-1], t_i = (c_i + c_{i+1}) / 2; coordinate y maps to
+ *              code #{i : t_i < y}
+ *   distortion host out, per-coordinate mean squared error (nullable)
+ * Returns TQ_EINVAL on bad d/bits/marginal or a NULL required pointer.
+ */
+tq_status tq_codebook(int d, int bits, int marginal, float* centroids,
+                      float* boundaries, double* distortion);
+
+/*
+ * tq_rotation - the "fixed random orthogonal matrix R" of Sec. II-B step 2.
+ * Host-only.  R = Q diag(sign(diag(U))) where G = Q U is the QR factorisation
+ * of a d x d standard Gaussian matrix filled row-major from splitmix64(seed)
+ * through Box-Muller (pair p: a = out(2p), b = out(2p+1),
+ * u1 = ((a>>11)+1) 2^-53, u2 = (b>>11) 2^-53, g = sqrt(-2 ln u1) (cos, sin)(2 pi u2)).
+ *   d     dimension (>= 2, <= 8192)
+ *   seed  generator seed
+ *   R     host out [d*d] float32, row-major; the rotation is y = R x
+ * Computed in float64 and rounded once.
+ */
+tq_status tq_rotation(int d, uint64_t seed, float* R);
+
+/*
+ * tq_encode - add(): encode n rows (Sec. II-B steps 1-5).
+ * For each row x: n = ||x||; y = R x / n (y = 0 if n = 0); code_j =
+ * #{i : boundaries[i] < y_j}; pack; scale per scale_mode.
+ *   X           device [n*d] float32, row-major
+ *   n           rows (>= 0; 0 is a no-op)
+ *   R           device [d*d] float32 row-major (tq_rotation's layout)
+ *   centroids   device [2^bits] float32, ascending
+ *   boundaries  device [2^bits - 1] float32, ascending
+ *   bits        2, 3, 4 or 8
+ *   scale_mode  TQ_SCALE_*
+ *   codes       device out [n * d*bits/8] uint8
+ *   scale       device out [n] float32
+ * y is computed in float32 (FFMA); a coordinate within ~1e-6 of a boundary may
+ * land in either neighbouring cell.
+ */
+tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
+                    const float* centroids, const float* boundaries, int bits,
+                    int scale_mode, uint8_t* codes, float* scale, void* stream);
+
+/*
+ * tq_filter_build - per-corpus tenant filter for search(allowlist=...)
+ * (Sec. III-B: filtering at vector-block granularity).
+ *   tenant_ids  device [n] uint32: the tenant of each vector
+ *   n           vectors (>= 1)
+ *   block       vectors per filter block: 32 or 64 (the paper uses 32)
+ *   out         host out: a new library-owned handle; free with
+ *               tq_filter_destroy
+ * The handle holds the sorted distinct tenant ids (T of them), each vector's
+ * dense tenant index and a T-bit tenant bitmap per block, all in device
+ * memory.  Synchronises `stream` (the distinct ids are counted on the host).
+ */
+tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int block,
+                          tq_filter** out, void* stream);
+
+/* Frees a handle from tq_filter_build (NULL is a no-op).  The caller ensures
+ * no queued search still uses it. */
+tq_status tq_filter_destroy(tq_filter* filter);
+
+/* Reports a handle's vector count, block size and distinct tenant count
+ * (each out pointer nullable). */
+tq_status tq_filter_info(const tq_filter* filter, int64_t* n, int* block,
+                         int64_t* n_tenants);
+
+/*
+ * tq_search_workspace - bytes of device scratch tq_search needs for these
+ * sizes on the current device (query rotation, allow bitmaps, per-CTA top-k
+ * candidates).  filter may be NULL (unfiltered).
+ */
+tq_status tq_search_workspace(int64_t nq, int64_t n, int d, int bits, int k,
+                              const tq_filter* filter, size_t* bytes);
+
+/*
+ * tq_search - search() / search(allowlist=...): top-k inner product of each
+ * query against the encoded corpus (Sec. II-B step 5, Sec. III-B).
+ * score(q, i) = scale[i] * sum_j (R q)_j * centroids[code_ij]; the k best
+ * allowed vectors per query by (score descending, id ascending).
+ *   Q              device [nq*d] float32 queries (not quantised)
+ *   nq             queries (>= 0; 0 is a no-op)
+ *   R, centroids   as for tq_encode
+ *   codes          device [n * d*bits/8] packed codes (tq_encode output)
+ *   scale          device [n] float32, or NULL for scale 1
+ *   n              corpus vectors (>= 1)
+ *   filter         NULL (every vector allowed) or a handle built for these
+ *                  n vectors
+ *   allow_off      device [nq+1] int64 CSR offsets into allow_tenants
+ *                  (required iff filter != NULL; allow_off[0] = 0, non-decreasing)
+ *   allow_tenants  device uint32 tenant ids allowed per query; ids absent from
+ *                  the corpus are ignored; an empty list allows nothing
+ *   k              1..256
+ *   out_ids        device out [nq*k] int64, -1 where fewer than k vectors are allowed
+ *   out_scores     device out [nq*k] float32, -INFINITY where out_ids is -1
+ *   workspace      device scratch of ws_bytes >= tq_search_workspace(...)
+ * Scores are float32 sums (LUT path) or fp16 products with float32
+ * accumulation (MMA path).
+ */
+tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
+                    const float* centroids, int bits, const uint8_t* codes,
+                    const float* scale, int64_t n, const tq_filter* filter,
+                    const int64_t* allow_off, const uint32_t* allow_tenants,
+                    int k, int64_t* out_ids, float* out_scores, void* workspace,
+                    size_t ws_bytes, void* stream);
+
+/* Selects the search kernels for later tq_search calls of the calling thread
+ * (TQ_PATH_*).  AUTO is the default. */
+tq_status tq_set_search_path(int path);
+
+/* Records two caller-created CUDA events (cudaEvent_t passed as void*) on the
+ * search stream immediately before and after the scan kernel of the calling
+ * thread's later tq_search calls, for per-kernel timing.  NULL, NULL turns it
+ * off. */
+tq_status tq_profile_events(void* scan_start, void* scan_stop);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TQ_H */

@@ -1,5 +1,180 @@
 """GB300-native TurboQuant search path (rotate, quantise, pack; filtered top-k scan).
 
-The compute runs in the CUDA library `libtq.so` built from `csrc/`; this package
-is a thin binding over its C ABI (see include/tq.h).
+Every computation runs in the CUDA library libtq.so built from csrc/ (C ABI in
+include/tq.h).  This module only marshals torch tensors and numpy arrays into
+that ABI: torch provides device memory and streams.  There is no CPU fallback:
+if libtq.so is missing, every call raises.
 """
+from __future__ import annotations
+
+import ctypes as C
+
+import numpy as np
+
+from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
+
+__all__ = ["codebook", "rotation", "encode", "Filter", "search", "search_workspace",
+           "search_from_host", "set_search_path", "profile_events", "row_bytes", "load",
+           "TQError"]
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _stream_handle(stream) -> int:
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _dev_ptr(t, name: str, dtype=None, contiguous: bool = True) -> int:
+    if t is None:
+        return 0
+    if not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype not in (dtype if isinstance(dtype, tuple) else (dtype,)):
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if contiguous and not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return int(t.data_ptr())
+
+
+def row_bytes(d: int, bits: int) -> int:
+    """Bytes of one packed vector: d*bits/8 (768 at d=1536, 4 bits)."""
+    return d * bits // 8
+
+
+def codebook(d: int, bits: int, marginal: str = "beta"):
+    """tq_codebook: Lloyd-Max centroids [2^bits], boundaries [2^bits - 1]
+    (float32 numpy) and the per-coordinate distortion."""
+    lib = load()
+    L = 1 << bits
+    c = np.zeros(L, np.float32)
+    t = np.zeros(max(L - 1, 1), np.float32)
+    D = C.c_double()
+    check(lib.tq_codebook(d, bits, MARGINALS[marginal], c.ctypes.data, t.ctypes.data, C.byref(D)))
+    return c, t[: L - 1], D.value
+
+
+def rotation(d: int, seed: int) -> np.ndarray:
+    """tq_rotation: float32 [d, d] row-major R (y = R x)."""
+    R = np.empty((d, d), np.float32)
+    check(load().tq_rotation(d, seed, R.ctypes.data))
+    return R
+
+
+def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
+           codes=None, scale=None, stream=None):
+    """tq_encode on CUDA tensors: returns (codes uint8 [n, d*bits/8], scale f32 [n])."""
+    torch = _torch()
+    n, d = X.shape
+    if codes is None:
+        codes = torch.empty((n, row_bytes(d, bits)), dtype=torch.uint8, device=X.device)
+    if scale is None:
+        scale = torch.empty(n, dtype=torch.float32, device=X.device)
+    f32 = torch.float32
+    check(load().tq_encode(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32),
+                           _dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32),
+                           bits, SCALE_MODES[scale_mode], _dev_ptr(codes, "codes", torch.uint8),
+                           _dev_ptr(scale, "scale", f32), _stream_handle(stream)))
+    return codes, scale
+
+
+class Filter:
+    """tq_filter handle: per-block tenant bitmaps of a corpus (Sec. III-B)."""
+
+    def __init__(self, tenant_ids, block: int = 64, stream=None):
+        torch = _torch()
+        self._h = C.c_void_p()
+        ptr = _dev_ptr(tenant_ids, "tenant_ids", (torch.int32, getattr(torch, "uint32", torch.int32)))
+        check(load().tq_filter_build(ptr, tenant_ids.numel(), block, C.byref(self._h),
+                                     _stream_handle(stream)))
+
+    @property
+    def handle(self) -> int:
+        return self._h.value or 0
+
+    def info(self):
+        n, b, t = C.c_int64(), C.c_int(), C.c_int64()
+        check(load().tq_filter_info(self._h, C.byref(n), C.byref(b), C.byref(t)))
+        return {"n": n.value, "block": b.value, "n_tenants": t.value}
+
+    def close(self) -> None:
+        if self._h and self._h.value:
+            load().tq_filter_destroy(self._h)
+            self._h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def search_workspace(nq: int, n: int, d: int, bits: int, k: int, filter: Filter | None = None) -> int:
+    out = C.c_size_t()
+    check(load().tq_search_workspace(nq, n, d, bits, k, filter.handle if filter else None, C.byref(out)))
+    return out.value
+
+
+def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | None = None,
+           allow_off=None, allow_tenants=None, workspace=None, out_ids=None, out_scores=None,
+           stream=None):
+    """tq_search on CUDA tensors: returns (ids int64 [nq, k], scores f32 [nq, k])."""
+    torch = _torch()
+    nq, d = Q.shape
+    n = codes.shape[0]
+    dev = Q.device
+    if out_ids is None:
+        out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    if out_scores is None:
+        out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    need = search_workspace(nq, n, d, bits, k, filter)
+    if workspace is None:
+        workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
+    f32 = torch.float32
+    u32 = (torch.int32, getattr(torch, "uint32", torch.int32))
+    check(load().tq_search(
+        _dev_ptr(Q, "Q", f32), nq, d, _dev_ptr(R, "R", f32), _dev_ptr(centroids, "centroids", f32), bits,
+        _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), n,
+        filter.handle if filter else None, _dev_ptr(allow_off, "allow_off", torch.int64),
+        _dev_ptr(allow_tenants, "allow_tenants", u32), k, _dev_ptr(out_ids, "out_ids", torch.int64),
+        _dev_ptr(out_scores, "out_scores", f32), _dev_ptr(workspace, "workspace", contiguous=True),
+        workspace.numel() * workspace.element_size(), _stream_handle(stream)))
+    return out_ids, out_scores
+
+
+def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, q_dev, ids_host,
+                     scores_host, filter: Filter | None = None, allow_off=None, allow_tenants=None,
+                     workspace=None, out_ids=None, out_scores=None, stream=None):
+    """search() for queries in (pinned) host memory: copies Q to q_dev, runs
+    tq_search and copies ids/scores back into the host tensors, all queued on
+    `stream`."""
+    q_dev.copy_(Q_host, non_blocking=True)
+    ids, scores = search(q_dev, R, centroids, bits, codes, scale, k, filter, allow_off, allow_tenants,
+                         workspace, out_ids, out_scores, stream)
+    ids_host.copy_(ids, non_blocking=True)
+    scores_host.copy_(scores, non_blocking=True)
+    return ids_host, scores_host
+
+
+def set_search_path(path: str) -> None:
+    """'auto' (default), 'lut' or 'mma' for later searches on this thread."""
+    check(load().tq_set_search_path(PATHS[path]))
+
+
+def profile_events(start=None, stop=None) -> None:
+    """Record two torch.cuda.Events around the scan kernel of later searches.
+    torch creates an event's CUDA handle on its first record(), so events that
+    have never been recorded are recorded once here first."""
+    handles = []
+    for ev in (start, stop):
+        if ev is None:
+            handles.append(None)
+            continue
+        if not int(ev.cuda_event):
+            ev.record()
+        handles.append(int(ev.cuda_event))
+    check(load().tq_profile_events(*handles))

@@ -1,0 +1,213 @@
+// C ABI entry points that queue device work: tq_encode, tq_filter_*,
+// tq_search_workspace, tq_search.  Every argument is validated before any
+// work is queued; CUDA errors come back as TQ_ECUDA with the runtime's text.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "tq_internal.h"
+#include "tq_kernels.h"
+
+struct tq_filter {
+  tq::FilterDev f;
+  int device = 0;
+};
+
+namespace tq {
+namespace {
+
+tq_status cuda_fail(const char* where, cudaError_t e) {
+  return fail(TQ_ECUDA, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+tq_status check_common(const char* fn, int d, int bits) {
+  if (d < 32 || d > kMaxD || d % 32 != 0)
+    return fail(TQ_EINVAL, "%s: d=%d must be a multiple of 32 in [32, %d]", fn, d, kMaxD);
+  if (!valid_bits(bits)) return fail(TQ_EINVAL, "%s: bits=%d must be 2, 3, 4 or 8", fn, bits);
+  return TQ_OK;
+}
+
+constexpr size_t kAlign = 256;
+inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+struct SearchPlan {
+  int grid_x = 1;
+  size_t off_rot = 0, off_allow = 0, off_cs = 0, off_ci = 0, total = 0;
+};
+
+SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
+  SearchPlan p;
+  p.grid_x = scan_lut_grid_x(nq, n, k, bits, d);
+  size_t off = 0;
+  p.off_rot = off;
+  off = align_up(off + (size_t)nq * d * sizeof(float));
+  p.off_allow = off;
+  if (filter) off = align_up(off + (size_t)nq * filter->f.words * sizeof(uint32_t));
+  p.off_cs = off;
+  off = align_up(off + (size_t)nq * p.grid_x * k * sizeof(float));
+  p.off_ci = off;
+  off = align_up(off + (size_t)nq * p.grid_x * k * sizeof(int32_t));
+  p.total = off;
+  return p;
+}
+
+}  // namespace
+}  // namespace tq
+
+using tq::fail;
+
+extern "C" tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
+                               const float* centroids, const float* boundaries, int bits,
+                               int scale_mode, uint8_t* codes, float* scale, void* stream) {
+  tq_status st = tq::check_common("tq_encode", d, bits);
+  if (st != TQ_OK) return st;
+  if (n < 0 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_encode: n=%lld outside [0, 2^31-1]", (long long)n);
+  if (scale_mode != TQ_SCALE_NORM && scale_mode != TQ_SCALE_NONE && scale_mode != TQ_SCALE_UNBIASED)
+    return fail(TQ_EINVAL, "tq_encode: unknown scale_mode %d", scale_mode);
+  if (n == 0) return tq::ok();
+  if (!X || !R || !centroids || !boundaries || !codes || !scale)
+    return fail(TQ_EINVAL, "tq_encode: NULL device pointer");
+  if (!tq::aligned16(X) || !tq::aligned16(R) || !tq::aligned16(codes))
+    return fail(TQ_EINVAL, "tq_encode: X, R and codes must be 16-byte aligned");
+  if (((uintptr_t)scale & 3u) || ((uintptr_t)centroids & 3u) || ((uintptr_t)boundaries & 3u))
+    return fail(TQ_EINVAL, "tq_encode: scale, centroids and boundaries must be 4-byte aligned");
+  cudaError_t e = tq::launch_encode(X, n, d, R, centroids, boundaries, bits, scale_mode, codes, scale,
+                                    (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_encode", e);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int block,
+                                     tq_filter** out, void* stream) {
+  if (!out) return fail(TQ_EINVAL, "tq_filter_build: NULL out");
+  *out = nullptr;
+  if (n < 1 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_filter_build: n=%lld outside [1, 2^31-1]", (long long)n);
+  if (block != 32 && block != 64) return fail(TQ_EINVAL, "tq_filter_build: block=%d must be 32 or 64", block);
+  if (!tenant_ids) return fail(TQ_EINVAL, "tq_filter_build: NULL tenant_ids");
+  cudaStream_t s = (cudaStream_t)stream;
+  tq_filter* h = nullptr;
+  try {
+    std::vector<uint32_t> ids((size_t)n);
+    cudaError_t e = cudaMemcpyAsync(ids.data(), tenant_ids, (size_t)n * sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return tq::cuda_fail("tq_filter_build: reading tenant ids", e);
+    std::sort(ids.begin(), ids.end());
+    ids.erase(std::unique(ids.begin(), ids.end()), ids.end());
+    h = new tq_filter();
+    cudaGetDevice(&h->device);
+    tq::FilterDev& f = h->f;
+    f.n = n;
+    f.block = block;
+    f.n_tenants = (int64_t)ids.size();
+    f.words = (int)((f.n_tenants + 31) / 32);
+    const int64_t nblocks = (n + block - 1) / block;
+    e = cudaMalloc(&f.tenants, ids.size() * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&f.dense, (size_t)n * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&f.block_bits, (size_t)nblocks * f.words * sizeof(uint32_t));
+    if (e != cudaSuccess) {
+      tq_filter_destroy(h);
+      cudaGetLastError();
+      return fail(TQ_ENOMEM, "tq_filter_build: device allocation failed: %s", cudaGetErrorString(e));
+    }
+    e = cudaMemcpyAsync(f.tenants, ids.data(), ids.size() * sizeof(uint32_t), cudaMemcpyHostToDevice, s);
+    if (e == cudaSuccess) e = tq::launch_filter_build(tenant_ids, f, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);  // `ids` is freed on return
+    if (e != cudaSuccess) {
+      tq_filter_destroy(h);
+      return tq::cuda_fail("tq_filter_build", e);
+    }
+    *out = h;
+    return tq::ok();
+  } catch (const std::bad_alloc&) {
+    if (h) tq_filter_destroy(h);
+    return fail(TQ_ENOMEM, "tq_filter_build: out of host memory");
+  }
+}
+
+extern "C" tq_status tq_filter_destroy(tq_filter* filter) {
+  if (!filter) return tq::ok();
+  cudaFree(filter->f.tenants);
+  cudaFree(filter->f.dense);
+  cudaFree(filter->f.block_bits);
+  delete filter;
+  return tq::ok();
+}
+
+extern "C" tq_status tq_filter_info(const tq_filter* filter, int64_t* n, int* block, int64_t* n_tenants) {
+  if (!filter) return fail(TQ_EINVAL, "tq_filter_info: NULL filter");
+  if (n) *n = filter->f.n;
+  if (block) *block = filter->f.block;
+  if (n_tenants) *n_tenants = filter->f.n_tenants;
+  return tq::ok();
+}
+
+namespace {
+tq_status check_search(int64_t nq, int64_t n, int d, int bits, int k) {
+  tq_status st = tq::check_common("tq_search", d, bits);
+  if (st != TQ_OK) return st;
+  if (nq < 0 || nq > (1 << 24)) return fail(TQ_EINVAL, "tq_search: nq=%lld outside [0, 2^24]", (long long)nq);
+  if (n < 1 || n > INT32_MAX - 1) return fail(TQ_EINVAL, "tq_search: n=%lld outside [1, 2^31-2]", (long long)n);
+  if (k < 1 || k > tq::kMaxK) return fail(TQ_EINVAL, "tq_search: k=%d outside [1, %d]", k, tq::kMaxK);
+  if (d > 2048) return fail(TQ_EUNSUPPORTED, "tq_search: d=%d > 2048 is not supported by this build", d);
+  return TQ_OK;
+}
+}  // namespace
+
+extern "C" tq_status tq_search_workspace(int64_t nq, int64_t n, int d, int bits, int k,
+                                         const tq_filter* filter, size_t* bytes) {
+  if (!bytes) return fail(TQ_EINVAL, "tq_search_workspace: NULL bytes");
+  tq_status st = check_search(nq, n, d, bits, k);
+  if (st != TQ_OK) return st;
+  *bytes = tq::plan_search(nq, n, d, bits, k, filter).total;
+  return tq::ok();
+}
+
+extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
+                               const float* centroids, int bits, const uint8_t* codes,
+                               const float* scale, int64_t n, const tq_filter* filter,
+                               const int64_t* allow_off, const uint32_t* allow_tenants, int k,
+                               int64_t* out_ids, float* out_scores, void* workspace,
+                               size_t ws_bytes, void* stream) {
+  tq_status st = check_search(nq, n, d, bits, k);
+  if (st != TQ_OK) return st;
+  if (nq == 0) return tq::ok();
+  if (!Q || !R || !centroids || !codes || !out_ids || !out_scores || !workspace)
+    return fail(TQ_EINVAL, "tq_search: NULL device pointer");
+  if (!tq::aligned16(Q) || !tq::aligned16(R) || !tq::aligned16(codes) || !tq::aligned16(workspace))
+    return fail(TQ_EINVAL, "tq_search: Q, R, codes and workspace must be 16-byte aligned");
+  if (((uintptr_t)centroids & 3u) || ((uintptr_t)scale & 3u) || ((uintptr_t)out_scores & 3u) ||
+      ((uintptr_t)out_ids & 7u))
+    return fail(TQ_EINVAL, "tq_search: misaligned centroids/scale/out pointers");
+  if (filter) {
+    if (filter->f.n != n)
+      return fail(TQ_EINVAL, "tq_search: filter built for n=%lld, search has n=%lld",
+                  (long long)filter->f.n, (long long)n);
+    if (!allow_off || !allow_tenants)
+      return fail(TQ_EINVAL, "tq_search: a filter needs allow_off and allow_tenants");
+    if (((uintptr_t)allow_off & 7u) || ((uintptr_t)allow_tenants & 3u))
+      return fail(TQ_EINVAL, "tq_search: misaligned allowlist pointers");
+  }
+  const int path = tq::search_path();
+  if (path == TQ_PATH_MMA) return fail(TQ_EUNSUPPORTED, "tq_search: the MMA path is not built yet");
+  const tq::SearchPlan p = tq::plan_search(nq, n, d, bits, k, filter);
+  if (ws_bytes < p.total)
+    return fail(TQ_EINVAL, "tq_search: workspace of %zu bytes, %zu needed", ws_bytes, p.total);
+  cudaStream_t s = (cudaStream_t)stream;
+  char* ws = static_cast<char*>(workspace);
+  float* qrot = reinterpret_cast<float*>(ws + p.off_rot);
+  uint32_t* allow = filter ? reinterpret_cast<uint32_t*>(ws + p.off_allow) : nullptr;
+  float* cs = reinterpret_cast<float*>(ws + p.off_cs);
+  int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
+  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, s);
+  if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
+  if (e == cudaSuccess)
+    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, filter ? &filter->f : nullptr, allow,
+                            k, p.grid_x, cs, ci, s, (cudaEvent_t)tq::profile_start(),
+                            (cudaEvent_t)tq::profile_stop());
+  if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_x * k, k, out_ids, out_scores, s);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
+  return tq::ok();
+}

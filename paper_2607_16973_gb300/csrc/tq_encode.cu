@@ -1,0 +1,326 @@
+// Encode (Sec. II-B steps 1-5) and query rotation (Sec. II-B step 2).
+//
+// The rotation y = R x is an FFMA SGEMM Y = X R^T (X row-major n x d, R
+// row-major d x d, both K-contiguous).  Each CTA owns a panel of 128 rows and
+// walks every 128-column tile of Y itself, so the per-row reductions the
+// scale needs (sum c^2, sum y c) are accumulated in shared memory in a fixed
+// order: results are deterministic and no scratch memory is used.  The
+// epilogue of every tile divides by the row norm, searches the boundaries,
+// and packs the codes straight to HBM (little-endian bit stream per row).
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "tq_internal.h"
+#include "tq_kernels.h"
+
+namespace tq {
+namespace {
+
+constexpr int BM = 128, BN = 128, BK = 8, PAD = 4, NT = 256;
+
+struct GemmSmem {
+  float A[2][BK][BM + PAD];
+  float B[2][BK][BN + PAD];
+};
+
+// Loads one BK-slice of an operand tile: 128 rows x 8 k as 256 float4.
+__device__ __forceinline__ float4 load_slice(const float* __restrict__ M, int64_t row0,
+                                             int64_t rows_valid, int d, int k0) {
+  const int t = threadIdx.x;
+  const int64_t r = row0 + (t >> 1);
+  if (r < rows_valid)
+    return __ldg(reinterpret_cast<const float4*>(M + r * d + k0 + (t & 1) * 4));
+  return make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+__device__ __forceinline__ void store_slice(float (*S)[BM + PAD], float4 v) {
+  const int t = threadIdx.x;
+  const int r = t >> 1, kq = (t & 1) * 4;
+  S[kq + 0][r] = v.x;
+  S[kq + 1][r] = v.y;
+  S[kq + 2][r] = v.z;
+  S[kq + 3][r] = v.w;
+}
+
+// acc = X[row0 .. row0+127, :] . R[col0 .. col0+127, :]^T over K = d.
+// Thread (tx = tid % 16, ty = tid / 16) owns rows ty*4 + {0..3} (+64) and
+// columns tx*4 + {0..3} (+64): acc[i][j], i < 4 -> first row block.
+__device__ __forceinline__ void gemm_tile(const float* __restrict__ X, int64_t row0, int64_t n_rows,
+                                          const float* __restrict__ R, int col0, int d,
+                                          GemmSmem& sm, float acc[8][8]) {
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  const int nk = d / BK;
+  float4 pa = load_slice(X, row0, n_rows, d, 0);
+  float4 pb = load_slice(R, col0, d, d, 0);
+  store_slice(sm.A[0], pa);
+  store_slice(sm.B[0], pb);
+  __syncthreads();
+  for (int kt = 0; kt < nk; ++kt) {
+    const int buf = kt & 1;
+    if (kt + 1 < nk) {
+      pa = load_slice(X, row0, n_rows, d, (kt + 1) * BK);
+      pb = load_slice(R, col0, d, d, (kt + 1) * BK);
+    }
+#pragma unroll
+    for (int k = 0; k < BK; ++k) {
+      const float4 a0 = *reinterpret_cast<const float4*>(&sm.A[buf][k][ty * 4]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&sm.A[buf][k][64 + ty * 4]);
+      const float4 b0 = *reinterpret_cast<const float4*>(&sm.B[buf][k][tx * 4]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&sm.B[buf][k][64 + tx * 4]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    if (kt + 1 < nk) {
+      store_slice(sm.A[buf ^ 1], pa);
+      store_slice(sm.B[buf ^ 1], pb);
+    }
+    __syncthreads();
+  }
+}
+
+__device__ __forceinline__ int tile_row(int i) { return (i < 4 ? 0 : 64) + (threadIdx.x >> 4) * 4 + (i & 3); }
+__device__ __forceinline__ int tile_col(int j) { return (j < 4 ? 0 : 64) + (threadIdx.x & 15) * 4 + (j & 3); }
+
+struct EncodeSmem {
+  GemmSmem g;
+  uint8_t ctile[BM][BN + 8];  // row stride 136 B keeps 8-byte reads aligned
+  float norm[BM], inv[BM], sum_c2[BM], sum_yc[BM];
+  float bnd[255], cen[256];
+};
+
+template <int BITS>
+__global__ void __launch_bounds__(NT, 2)
+k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict__ R,
+         const float* __restrict__ centroids, const float* __restrict__ boundaries, int scale_mode,
+         uint8_t* __restrict__ codes, float* __restrict__ scale) {
+  constexpr int L = 1 << BITS;
+  __shared__ EncodeSmem sm;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i = tid; i < L; i += NT) sm.cen[i] = centroids[i];
+  for (int i = tid; i < L - 1; i += NT) sm.bnd[i] = boundaries[i];
+  const int64_t row_bytes = (int64_t)d * BITS / 8;
+  const int64_t panels = (n + BM - 1) / BM;
+  const int ntiles = (d + BN - 1) / BN;
+
+  for (int64_t p = blockIdx.x; p < panels; p += gridDim.x) {
+    const int64_t row0 = p * BM;
+    // step 1: row norms (one warp per row, fixed summation order)
+    for (int r = warp; r < BM; r += NT / 32) {
+      float s = 0.f;
+      if (row0 + r < n) {
+        const float4* xr = reinterpret_cast<const float4*>(X + (row0 + r) * d);
+        for (int j = lane; j < d / 4; j += 32) {
+          const float4 v = __ldg(xr + j);
+          s = fmaf(v.x, v.x, s);
+          s = fmaf(v.y, v.y, s);
+          s = fmaf(v.z, v.z, s);
+          s = fmaf(v.w, v.w, s);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+      if (lane == 0) {
+        const float nr = sqrtf(s);
+        sm.norm[r] = nr;
+        sm.inv[r] = nr > 0.f ? 1.0f / nr : 0.f;
+        sm.sum_c2[r] = 0.f;
+        sm.sum_yc[r] = 0.f;
+      }
+    }
+    __syncthreads();
+    for (int nt = 0; nt < ntiles; ++nt) {
+      const int col0 = nt * BN;
+      float acc[8][8];
+      gemm_tile(X, row0, n, R, col0, d, sm.g, acc);
+      // step 2-3: y = acc / ||x||, code = #{t < y}
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = tile_row(i);
+        const float inv = sm.inv[r];
+        float pc2 = 0.f, pyc = 0.f;
+#pragma unroll
+        for (int jh = 0; jh < 2; ++jh) {
+          uint32_t packed4 = 0;
+#pragma unroll
+          for (int jj = 0; jj < 4; ++jj) {
+            const int j = jh * 4 + jj;
+            const float y = acc[i][j] * inv;
+            int code = 0;
+#pragma unroll
+            for (int step = L / 2; step >= 1; step >>= 1)
+              if (y > sm.bnd[code + step - 1]) code += step;
+            const float c = sm.cen[code];
+            if (col0 + tile_col(j) < d) {
+              pc2 = fmaf(c, c, pc2);
+              pyc = fmaf(y, c, pyc);
+            }
+            packed4 |= (uint32_t)code << (8 * jj);
+          }
+          *reinterpret_cast<uint32_t*>(&sm.ctile[r][tile_col(jh * 4)]) = packed4;
+        }
+#pragma unroll
+        for (int o = 1; o < 16; o <<= 1) {
+          pc2 += __shfl_xor_sync(0xffffffffu, pc2, o);
+          pyc += __shfl_xor_sync(0xffffffffu, pyc, o);
+        }
+        if ((tid & 15) == 0) {
+          sm.sum_c2[r] += pc2;
+          sm.sum_yc[r] += pyc;
+        }
+      }
+      __syncthreads();
+      // step 4: pack 8 codes per item straight to HBM
+      for (int item = tid; item < BM * (BN / 8); item += NT) {
+        const int r = item / (BN / 8), g = item % (BN / 8);
+        const int64_t row = row0 + r;
+        const int dim0 = col0 + g * 8;
+        if (row >= n || dim0 >= d) continue;
+        const uint2 cc = *reinterpret_cast<const uint2*>(&sm.ctile[r][g * 8]);
+        const uint64_t c8 = (uint64_t)cc.x | ((uint64_t)cc.y << 32);
+        uint64_t bitsv = 0;
+#pragma unroll
+        for (int t = 0; t < 8; ++t) bitsv |= ((c8 >> (8 * t)) & (uint64_t)(L - 1)) << (BITS * t);
+        uint8_t* dst = codes + row * row_bytes + (int64_t)dim0 * BITS / 8;
+        if constexpr (BITS == 8) {
+          *reinterpret_cast<uint64_t*>(dst) = bitsv;
+        } else if constexpr (BITS == 4) {
+          *reinterpret_cast<uint32_t*>(dst) = (uint32_t)bitsv;
+        } else if constexpr (BITS == 2) {
+          *reinterpret_cast<uint16_t*>(dst) = (uint16_t)bitsv;
+        } else {
+          dst[0] = (uint8_t)bitsv;
+          dst[1] = (uint8_t)(bitsv >> 8);
+          dst[2] = (uint8_t)(bitsv >> 16);
+        }
+      }
+      __syncthreads();
+    }
+    // step 5: per-vector scalar
+    for (int r = tid; r < BM; r += NT) {
+      const int64_t row = row0 + r;
+      if (row >= n) continue;
+      const float nr = sm.norm[r];
+      float s = 0.f;
+      if (nr > 0.f) {
+        if (scale_mode == TQ_SCALE_NONE) {
+          s = nr;
+        } else if (scale_mode == TQ_SCALE_NORM) {
+          const float cn = sqrtf(sm.sum_c2[r]);
+          s = cn > 0.f ? nr / cn : 0.f;
+        } else {
+          const float yc = sm.sum_yc[r];
+          s = yc != 0.f ? nr / yc : 0.f;
+        }
+      }
+      scale[row] = s;
+    }
+    __syncthreads();
+  }
+}
+
+// Q' = Q R^T, plain store epilogue (nq > 8).
+__global__ void __launch_bounds__(NT, 2)
+k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R,
+              float* __restrict__ out) {
+  __shared__ GemmSmem sm;
+  const int64_t row0 = (int64_t)blockIdx.x * BM;
+  const int col0 = blockIdx.y * BN;
+  float acc[8][8];
+  gemm_tile(Q, row0, nq, R, col0, d, sm, acc);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int64_t r = row0 + tile_row(i);
+    if (r >= nq) continue;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int c = col0 + tile_col(j);
+      if (c < d) out[r * d + c] = acc[i][j];
+    }
+  }
+}
+
+// Q' = Q R^T for nq <= 8: one warp per output coordinate, R read once.
+template <int NQ>
+__global__ void __launch_bounds__(256)
+k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, float* __restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (i >= d) return;
+  float acc[NQ];
+#pragma unroll
+  for (int q = 0; q < NQ; ++q) acc[q] = 0.f;
+  const float4* r4 = reinterpret_cast<const float4*>(R + (int64_t)i * d);
+  for (int j = lane; j < d / 4; j += 32) {
+    const float4 rv = __ldg(r4 + j);
+#pragma unroll
+    for (int q = 0; q < NQ; ++q) {
+      const float4 qv = __ldg(reinterpret_cast<const float4*>(Q + (int64_t)q * d) + j);
+      acc[q] = fmaf(rv.x, qv.x, acc[q]);
+      acc[q] = fmaf(rv.y, qv.y, acc[q]);
+      acc[q] = fmaf(rv.z, qv.z, acc[q]);
+      acc[q] = fmaf(rv.w, qv.w, acc[q]);
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < NQ; ++q) {
+    float s = acc[q];
+#pragma unroll
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    if (lane == 0) out[(int64_t)q * d + i] = s;
+  }
+}
+
+}  // namespace
+
+int device_sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
+  return sms > 0 ? sms : 1;
+}
+
+cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,
+                          const float* boundaries, int bits, int scale_mode, uint8_t* codes,
+                          float* scale, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  const int64_t panels = (n + BM - 1) / BM;
+  const int grid = (int)std::min<int64_t>(panels, (int64_t)device_sm_count() * 2);
+  switch (bits) {
+    case 2: k_encode<2><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
+    case 3: k_encode<3><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
+    case 4: k_encode<4><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
+    case 8: k_encode<8><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out,
+                          cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  if (nq <= 8) {
+    const int grid = (d + 7) / 8;
+    switch (nq) {
+#define TQ_GEMV_CASE(N) \
+  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, d, R, out); break;
+      TQ_GEMV_CASE(1) TQ_GEMV_CASE(2) TQ_GEMV_CASE(3) TQ_GEMV_CASE(4)
+      TQ_GEMV_CASE(5) TQ_GEMV_CASE(6) TQ_GEMV_CASE(7) TQ_GEMV_CASE(8)
+#undef TQ_GEMV_CASE
+    }
+    return cudaGetLastError();
+  }
+  dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN));
+  k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out);
+  return cudaGetLastError();
+}
+
+}  // namespace tq

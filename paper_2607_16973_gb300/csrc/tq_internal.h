@@ -1,0 +1,31 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cstdarg>
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/tq.h"
+
+namespace tq {
+
+// Records a thread-local error message and returns `st`.
+tq_status fail(tq_status st, const char* fmt, ...);
+// Clears the thread-local message and returns TQ_OK.
+tq_status ok();
+
+// Thread-local settings (tq_set_search_path / tq_profile_events).
+int search_path();
+void* profile_start();
+void* profile_stop();
+
+constexpr int kMaxK = 256;
+constexpr int kMaxKMma = 64;     // per-thread top-k lists of the tensor-core scan
+constexpr int kMmaMinBatch = 16; // AUTO uses the tensor-core scan from this batch size
+constexpr int kMaxD = 8192;
+
+inline bool valid_bits(int b) { return b == 2 || b == 3 || b == 4 || b == 8; }
+inline int64_t row_bytes(int d, int bits) { return (int64_t)d * bits / 8; }
+inline bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+}  // namespace tq

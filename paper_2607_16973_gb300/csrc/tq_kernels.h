@@ -1,0 +1,60 @@
+// Host-side launchers of the CUDA kernels (internal to libtq.so).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace tq {
+
+struct FilterDev {
+  int64_t n = 0;
+  int block = 64;
+  int64_t n_tenants = 0;  // T distinct tenant ids
+  int words = 0;          // ceil(T / 32)
+  uint32_t* tenants = nullptr;    // device [T] sorted distinct raw ids
+  uint32_t* dense = nullptr;      // device [n] dense tenant index per vector
+  uint32_t* block_bits = nullptr; // device [nblocks * words]
+};
+
+// Encode (Sec. II-B steps 1-5): fused rotation GEMM + quantise + pack + scale.
+cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,
+                          const float* boundaries, int bits, int scale_mode, uint8_t* codes,
+                          float* scale, cudaStream_t s);
+
+// q' = R q for nq queries: out [nq * d] float32.
+cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out,
+                          cudaStream_t s);
+
+// Per-query allow bitmaps over the dense tenant index: out [nq * words].
+cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
+                              const uint32_t* allow_tenants, int64_t nq, uint32_t* out,
+                              cudaStream_t s);
+
+// Filter build: dense index per vector and per-block tenant bitmaps.
+cudaError_t launch_filter_build(const uint32_t* tenant_ids, FilterDev& f, cudaStream_t s);
+
+// LUT scan: per-CTA top-k candidates [nq][grid_x][k] (score, id).
+int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d);
+cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
+                            const uint8_t* codes, const float* scale, int64_t n, const FilterDev* f,
+                            const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
+                            int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1);
+
+// Final merge of per-CTA candidates into sorted top-k.
+cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
+                         int k, int64_t* out_ids, float* out_scores, cudaStream_t s);
+
+// Tensor-core decode-GEMM scan (bits 2, 4, 8; k <= kMaxKMma; unfiltered).
+bool mma_supported(int bits, int d, int k);
+int scan_mma_grid_x(int64_t nq, int64_t n);
+size_t mma_qpack_bytes(int64_t nq, int d);
+cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
+                            const uint8_t* codes, const float* scale, int64_t n, int k, int grid_x,
+                            void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
+                            cudaEvent_t ev0, cudaEvent_t ev1);
+
+int device_sm_count();
+
+}  // namespace tq

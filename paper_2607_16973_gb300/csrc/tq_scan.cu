@@ -1,0 +1,391 @@
+// Search-side kernels: the lookup scan with fused top-k (Sec. II-B step 5,
+// Sec. III-B), per-query allow bitmaps, the filter build and the final merge.
+//
+// Lookup scan layout.  One warp scores one vector at a time.  The packed row
+// is cut into chunks of 16 codes (2*bits bytes); lane l owns chunks l, l+32,
+// l+64, ... of every row, so each load instruction of a warp reads a
+// contiguous run of the row and every lane always handles the same
+// coordinates.  Lane l keeps the rotated query's values for its coordinates
+// in registers and looks the centroid of each code up in a table replicated
+// across the 32 shared-memory banks (entry (code, lane) lives in bank lane), so
+// the lookups of a warp never conflict.  score = scale * sum_j q'_j c[code_j].
+//
+// Top-k: each warp keeps a sorted list of its k best (score desc, id asc) in
+// shared memory, entered only when a score beats the list's k-th entry; a
+// disallowed vector never enters (Sec. III-B: dropped at heap insert).  Blocks
+// of `block` vectors whose tenant bitmap shares no bit with the query's allow
+// bitmap are skipped before any code byte is read (Sec. III-B).
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cmath>
+#include <cstdint>
+
+#include "tq_internal.h"
+#include "tq_kernels.h"
+
+namespace tq {
+namespace {
+
+constexpr unsigned FULL = 0xffffffffu;
+constexpr int SCAN_NT = 256;
+constexpr int SCAN_WARPS = SCAN_NT / 32;
+constexpr int MERGE_P = 2048;
+
+__device__ __forceinline__ bool better(float s1, int i1, float s2, int i2) {
+  return s1 > s2 || (s1 == s2 && i1 < i2);
+}
+
+// Bitonic sort of P (a power of two) (score, id) pairs in shared memory, best
+// first.  All threads of the block take part.
+__device__ void block_sort(float* s, int* id, int P) {
+  for (int size = 2; size <= P; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int t = threadIdx.x; t < P / 2; t += blockDim.x) {
+        const int i = 2 * t - (t & (stride - 1));
+        const int j = i + stride;
+        const float si = s[i], sj = s[j];
+        const int ii = id[i], ij = id[j];
+        const bool best_first = (i & size) == 0;
+        const bool swap = best_first ? better(sj, ij, si, ii) : better(si, ii, sj, ij);
+        if (swap) {
+          s[i] = sj;
+          s[j] = si;
+          id[i] = ij;
+          id[j] = ii;
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// Inserts (s, id) into a warp's sorted list of `cnt` entries (capacity k).
+// The caller has checked that it beats the k-th entry (or cnt < k).
+__device__ __forceinline__ void warp_insert(float* ws, int* wi, int k, int cnt, float s, int id) {
+  const int lane = threadIdx.x & 31;
+  int pos = 0;
+  for (int base = 0; base < cnt; base += 32) {
+    const int i = base + lane;
+    const bool b = i < cnt && better(ws[i], wi[i], s, id);
+    pos += __popc(__ballot_sync(FULL, b));
+  }
+  const int last = min(cnt, k - 1);  // entries [pos, last) move down one slot
+  for (int base = ((max(last, 1) - 1) >> 5) << 5; base >= 0; base -= 32) {
+    if (base + 32 <= pos) break;
+    const int i = base + lane;
+    const bool mv = i >= pos && i < last;
+    float sv = 0.f;
+    int iv = 0;
+    if (mv) {
+      sv = ws[i];
+      iv = wi[i];
+    }
+    __syncwarp();
+    if (mv) {
+      ws[i + 1] = sv;
+      wi[i + 1] = iv;
+    }
+    __syncwarp();
+  }
+  if (lane == 0) {
+    ws[pos] = s;
+    wi[pos] = id;
+  }
+  __syncwarp();
+}
+
+// 16 codes of `BITS` bits starting at a chunk boundary.
+template <int BITS>
+struct Chunk;
+
+template <>
+struct Chunk<4> {
+  uint32_t w0, w1;
+  __device__ __forceinline__ void load(const uint8_t* p) {
+    const uint2 v = __ldcs(reinterpret_cast<const uint2*>(p));
+    w0 = v.x;
+    w1 = v.y;
+  }
+  __device__ __forceinline__ uint32_t code(int t) const { return ((t < 8 ? w0 : w1) >> (4 * (t & 7))) & 15u; }
+};
+
+template <>
+struct Chunk<2> {
+  uint32_t w;
+  __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const unsigned int*>(p)); }
+  __device__ __forceinline__ uint32_t code(int t) const { return (w >> (2 * t)) & 3u; }
+};
+
+template <>
+struct Chunk<8> {
+  uint4 w;
+  __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const uint4*>(p)); }
+  __device__ __forceinline__ uint32_t code(int t) const {
+    const uint32_t x = t < 4 ? w.x : t < 8 ? w.y : t < 12 ? w.z : w.w;
+    return (x >> (8 * (t & 3))) & 255u;
+  }
+};
+
+template <>
+struct Chunk<3> {
+  uint64_t v;  // 48 bits
+  __device__ __forceinline__ void load(const uint8_t* p) {
+    const unsigned short* h = reinterpret_cast<const unsigned short*>(p);
+    v = (uint64_t)__ldcs(h) | ((uint64_t)__ldcs(h + 1) << 16) | ((uint64_t)__ldcs(h + 2) << 32);
+  }
+  __device__ __forceinline__ uint32_t code(int t) const { return (uint32_t)(v >> (3 * t)) & 7u; }
+};
+
+template <int BITS, int S>
+__global__ void __launch_bounds__(SCAN_NT, 2)
+k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
+           const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+           const uint32_t* __restrict__ dense, const uint32_t* __restrict__ block_bits, int words,
+           int fblock, const uint32_t* __restrict__ allow_bits, int k, int P,
+           float* __restrict__ cand_s, int* __restrict__ cand_i) {
+  constexpr int L = 1 << BITS;
+  constexpr int CB = 2 * BITS;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* ctab = reinterpret_cast<float*>(smem_raw);  // [L][32], entry (c, lane) in bank lane
+  float* ls = ctab + L * 32;                          // [P] scores; warp w's list at [w*k, w*k+k)
+  int* li = reinterpret_cast<int*>(ls + P);           // [P] ids
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int q = blockIdx.y;
+  for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  for (int i = tid; i < P; i += SCAN_NT) {
+    ls[i] = -INFINITY;
+    li[i] = INT_MAX;
+  }
+  const int nchunks = d >> 4;
+  const float* qq = qrot + (size_t)q * d;
+  float qr[S][16];
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    const int chunk = lane + 32 * s;
+#pragma unroll
+    for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+  }
+  __syncthreads();
+
+  const int64_t row_bytes = (int64_t)d * BITS / 8;
+  const uint32_t* ab = allow_bits ? allow_bits + (size_t)q * words : nullptr;
+  float* wl_s = ls + warp * k;
+  int* wl_i = li + warp * k;
+  int cnt = 0;
+  float th_s = -INFINITY;
+  int th_i = INT_MAX;
+  const int nfb = (n + fblock - 1) / fblock;
+  for (int b = blockIdx.x; b < nfb; b += gridDim.x) {
+    if (ab) {
+      uint32_t any = 0;
+      for (int w = lane; w < words; w += 32) any |= __ldg(block_bits + (size_t)b * words + w) & __ldg(ab + w);
+      if (!__any_sync(FULL, any != 0u)) continue;  // no allowed vector in this block
+    }
+    const int v_end = min(n, (b + 1) * fblock);
+    for (int v = b * fblock + warp; v < v_end; v += SCAN_WARPS) {
+      const uint8_t* row = codes + (size_t)v * row_bytes;
+      float acc = 0.f;
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        const int chunk = lane + 32 * s;
+        if (chunk < nchunks) {
+          Chunk<BITS> c;
+          c.load(row + chunk * CB);
+#pragma unroll
+          for (int t = 0; t < 16; ++t) acc = fmaf(qr[s][t], ctab[(c.code(t) << 5) | lane], acc);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(FULL, acc, o);
+      const float score = scale ? acc * __ldg(scale + v) : acc;
+      bool allowed = true;
+      if (ab) {
+        const uint32_t t = __ldg(dense + v);
+        allowed = (__ldg(ab + (t >> 5)) >> (t & 31)) & 1u;
+      }
+      if (allowed && better(score, v, th_s, th_i)) {
+        warp_insert(wl_s, wl_i, k, cnt, score, v);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = wl_s[k - 1];
+          th_i = wl_i[k - 1];
+        }
+      }
+    }
+  }
+  __syncthreads();
+  block_sort(ls, li, P);
+  for (int i = tid; i < k; i += SCAN_NT) {
+    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
+    cand_s[o] = ls[i];
+    cand_i[o] = li[i];
+  }
+}
+
+// Merges per_query candidates of each query into its sorted top-k.
+__global__ void __launch_bounds__(256)
+k_merge(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int per_query, int k,
+        int P, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* s = reinterpret_cast<float*>(smem_raw);
+  int* id = reinterpret_cast<int*>(s + P);
+  const int q = blockIdx.x;
+  const float* cs = cand_s + (size_t)q * per_query;
+  const int* ci = cand_i + (size_t)q * per_query;
+  for (int i = threadIdx.x; i < k; i += blockDim.x) {
+    s[i] = -INFINITY;
+    id[i] = INT_MAX;
+  }
+  const int chunk = P - k;
+  for (int c0 = 0; c0 < per_query; c0 += chunk) {
+    for (int i = threadIdx.x; i < chunk; i += blockDim.x) {
+      const int j = c0 + i;
+      s[k + i] = j < per_query ? cs[j] : -INFINITY;
+      id[k + i] = j < per_query ? ci[j] : INT_MAX;
+    }
+    __syncthreads();
+    block_sort(s, id, P);
+  }
+  for (int i = threadIdx.x; i < k; i += blockDim.x) {
+    const bool pad = id[i] == INT_MAX;
+    out_ids[(size_t)q * k + i] = pad ? -1 : (int64_t)id[i];
+    out_scores[(size_t)q * k + i] = pad ? -INFINITY : s[i];
+  }
+}
+
+__device__ __forceinline__ int64_t find_tenant(const uint32_t* __restrict__ tenants, int64_t T, uint32_t x) {
+  int64_t lo = 0, hi = T;
+  while (lo < hi) {
+    const int64_t mid = (lo + hi) >> 1;
+    if (__ldg(tenants + mid) < x) lo = mid + 1; else hi = mid;
+  }
+  return (lo < T && __ldg(tenants + lo) == x) ? lo : -1;
+}
+
+__global__ void k_allow_bits(const uint32_t* __restrict__ tenants, int64_t T, int words,
+                             const int64_t* __restrict__ off, const uint32_t* __restrict__ ids,
+                             uint32_t* __restrict__ out) {
+  const int64_t q = blockIdx.x;
+  uint32_t* o = out + q * words;
+  for (int w = threadIdx.x; w < words; w += blockDim.x) o[w] = 0u;
+  __syncthreads();
+  const int64_t a = off[q], b = off[q + 1];
+  for (int64_t j = a + threadIdx.x; j < b; j += blockDim.x) {
+    const int64_t pos = find_tenant(tenants, T, ids[j]);
+    if (pos >= 0) atomicOr(o + (pos >> 5), 1u << (pos & 31));
+  }
+}
+
+__global__ void k_filter_build(const uint32_t* __restrict__ tenant_ids, int64_t n,
+                               const uint32_t* __restrict__ tenants, int64_t T, int words, int block,
+                               uint32_t* __restrict__ dense, uint32_t* __restrict__ block_bits) {
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n; v += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t pos = find_tenant(tenants, T, tenant_ids[v]);  // always found: tenants holds every id
+    const uint32_t p = (uint32_t)(pos < 0 ? 0 : pos);
+    dense[v] = p;
+    atomicOr(block_bits + (v / block) * words + (p >> 5), 1u << (p & 31));
+  }
+}
+
+int next_pow2(int x) {
+  int p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+template <int BITS, int S>
+cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
+                           const float* centroids, const uint8_t* codes, const float* scale, int n,
+                           const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
+                           const uint32_t* allow, int k, int P, float* cs, int* ci) {
+  cudaError_t e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_scan_lut<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
+                                                  words, fblock, allow, k, P, cs, ci);
+  return cudaGetLastError();
+}
+
+template <int BITS>
+cudaError_t scan_lut_bits(int S, dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
+                          const float* centroids, const uint8_t* codes, const float* scale, int n,
+                          const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
+                          const uint32_t* allow, int k, int P, float* cs, int* ci) {
+  switch (S) {
+    case 1: return scan_lut_typed<BITS, 1>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 2: return scan_lut_typed<BITS, 2>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 3: return scan_lut_typed<BITS, 3>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 4: return scan_lut_typed<BITS, 4>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d) {
+  (void)k;
+  (void)bits;
+  (void)d;
+  const int64_t target = (int64_t)device_sm_count() * 4;
+  int64_t gx = (target + nq - 1) / (nq > 0 ? nq : 1);
+  const int64_t blocks = (n + 31) / 32;
+  if (gx > blocks) gx = blocks;
+  if (gx < 1) gx = 1;
+  return (int)gx;
+}
+
+cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
+                            const uint8_t* codes, const float* scale, int64_t n, const FilterDev* f,
+                            const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
+                            int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1) {
+  if (nq == 0) return cudaSuccess;
+  const int S = (d + 511) / 512;
+  const int P = next_pow2(SCAN_WARPS * k);
+  const size_t smem = (size_t)(1 << bits) * 32 * sizeof(float) + (size_t)P * (sizeof(float) + sizeof(int));
+  const dim3 grid((unsigned)grid_x, (unsigned)nq);
+  const uint32_t* dense = f ? f->dense : nullptr;
+  const uint32_t* bb = f ? f->block_bits : nullptr;
+  const int words = f ? f->words : 0;
+  const int fblock = f ? f->block : 64;
+  cudaError_t e;
+  if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;
+  switch (bits) {
+    case 2: e = scan_lut_bits<2>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 3: e = scan_lut_bits<3>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 4: e = scan_lut_bits<4>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 8: e = scan_lut_bits<8>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    default: e = cudaErrorInvalidValue;
+  }
+  if (e != cudaSuccess) return e;
+  if (ev1 && (e = cudaEventRecord(ev1, s)) != cudaSuccess) return e;
+  return cudaSuccess;
+}
+
+cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
+                         int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  const int P = std::min(MERGE_P, next_pow2(std::max(per_query + k, 64)));
+  const size_t smem = (size_t)P * (sizeof(float) + sizeof(int));
+  k_merge<<<(unsigned)nq, 256, smem, s>>>(cand_s, cand_i, per_query, k, P, out_ids, out_scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
+                              const uint32_t* allow_tenants, int64_t nq, uint32_t* out,
+                              cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  k_allow_bits<<<(unsigned)nq, 128, 0, s>>>(f.tenants, f.n_tenants, f.words, allow_off, allow_tenants, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_filter_build(const uint32_t* tenant_ids, FilterDev& f, cudaStream_t s) {
+  const int64_t nblocks = (f.n + f.block - 1) / f.block;
+  cudaError_t e = cudaMemsetAsync(f.block_bits, 0, (size_t)nblocks * f.words * sizeof(uint32_t), s);
+  if (e != cudaSuccess) return e;
+  const int grid = (int)std::min<int64_t>((f.n + 255) / 256, (int64_t)device_sm_count() * 8);
+  k_filter_build<<<grid, 256, 0, s>>>(tenant_ids, f.n, f.tenants, f.n_tenants, f.words, f.block, f.dense,
+                                      f.block_bits);
+  return cudaGetLastError();
+}
+
+}  // namespace tq

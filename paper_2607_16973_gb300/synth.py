@@ -42,18 +42,20 @@ def mixture_centers(d: int, n_clusters: int, seed: int = SEED_DATA) -> np.ndarra
 
 def mixture_rows(start: int, stop: int, d: int, n_clusters: int,
                  seed: int = SEED_DATA, spread: float = 0.5,
-                 centers: np.ndarray | None = None) -> np.ndarray:
+                 centers: np.ndarray | None = None, workers: int = 1) -> np.ndarray:
     """Rows [start, stop) of the seeded mixture corpus, float32, unit L2 norm.
 
     Row r belongs to chunk r // CHUNK_ROWS; chunk c draws from the stream
-    seeded by (seed, c), so any range is reproducible on its own.
+    seeded by (seed, c), so any range is reproducible on its own (and the
+    result does not depend on `workers`).
     """
     if centers is None:
         centers = mixture_centers(d, n_clusters, seed)
     out = np.empty((max(stop - start, 0), d), dtype=np.float32)
     c0 = start // CHUNK_ROWS
     c1 = (stop + CHUNK_ROWS - 1) // CHUNK_ROWS
-    for c in range(c0, c1):
+
+    def one(c: int) -> None:
         # every chunk draws all CHUNK_ROWS rows so a row never depends on
         # which range asked for it
         rng = np.random.default_rng([seed, c, n_clusters, d])
@@ -65,14 +67,22 @@ def mixture_rows(start: int, stop: int, d: int, n_clusters: int,
         block = centers[z[a:b]] + spread * noise[a:b].astype(np.float64)
         block /= np.linalg.norm(block, axis=1, keepdims=True)
         out[lo - start: hi - start] = block.astype(np.float32)
+
+    if workers > 1 and c1 - c0 > 1:
+        from concurrent.futures import ThreadPoolExecutor
+        with ThreadPoolExecutor(max_workers=workers) as ex:
+            list(ex.map(one, range(c0, c1)))
+    else:
+        for c in range(c0, c1):
+            one(c)
     return out
 
 
 def mixture_corpus(n: int, d: int, n_clusters: int, seed: int = SEED_DATA,
-                   spread: float = 0.5) -> np.ndarray:
+                   spread: float = 0.5, workers: int = 1) -> np.ndarray:
     """The whole seeded mixture corpus, float32 [n, d], unit rows."""
     centers = mixture_centers(d, n_clusters, seed)
-    return mixture_rows(0, n, d, n_clusters, seed, spread, centers)
+    return mixture_rows(0, n, d, n_clusters, seed, spread, centers, workers)
 
 
 def query_sources(n: int, nq: int, seed: int = SEED_QUERIES) -> np.ndarray:

@@ -1,0 +1,267 @@
+"""Parity of the CUDA path with the oracle, element by element, on seeded
+inputs the oracle finishes in seconds (several tiles plus ragged tails), and
+the edge cases of the method.  Every call goes through the C ABI."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2607_16973_gb300 import synth
+from conftest import GOLDEN
+from parity import TOL_LUT, check_encode, check_topk, recall
+
+pytestmark = pytest.mark.gpu
+
+
+def _cb(d, bits, marginal="beta"):
+    if d == 1536:
+        with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+            e = [e for e in json.load(f)["entries"] if e["bits"] == bits and e["marginal"] == marginal][0]
+        return np.asarray(e["centroids"], np.float32), np.asarray(e["boundaries"], np.float32)
+    cb = O.codebook(d, bits, marginal)
+    return cb.centroids32, cb.boundaries32
+
+
+@pytest.fixture(scope="module")
+def torch_dev(cuda_lib):
+    import torch
+    return torch, torch.device("cuda:0")
+
+
+def _t(torch, dev, a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+
+# ------------------------------------------------------------------- encode --
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+@pytest.mark.parametrize("mode", ["norm", "none", "unbiased"])
+def test_encode_parity(cuda_lib, torch_dev, bits, mode):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, n = 1536, 2077                       # 16 panels of 128 rows + a ragged 29
+    X = synth.mixture_corpus(n, d, 64, seed=42)
+    X[5] = 0.0                              # zero row: codes L/2-1, scale 0
+    X[6] *= 3.0
+    R = O.rotation(d, 1536).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    enc = O.encode(X, R, c32, t32, bits, mode)
+    codes, scale = tq.encode(_t(torch, dev, X), _t(torch, dev, R), _t(torch, dev, c32), _t(torch, dev, t32),
+                             bits, mode)
+    torch.cuda.synchronize()
+    check_encode(codes.cpu().numpy(), scale.cpu().numpy(), X, enc, c32, t32, d, bits, mode)
+    assert np.all(codes.cpu().numpy()[5] == enc.packed[5]) and scale.cpu().numpy()[5] == 0.0
+
+
+@pytest.mark.parametrize("d", [32, 96, 160, 2048])
+def test_encode_parity_dims(cuda_lib, torch_dev, d):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    n, bits = 300, 4
+    X = synth.mixture_corpus(n, d, 8, seed=7)
+    R = O.rotation(d, 11).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    enc = O.encode(X, R, c32, t32, bits)
+    codes, scale = tq.encode(_t(torch, dev, X), _t(torch, dev, R), _t(torch, dev, c32), _t(torch, dev, t32), bits)
+    torch.cuda.synchronize()
+    check_encode(codes.cpu().numpy(), scale.cpu().numpy(), X, enc, c32, t32, d, bits, "norm")
+
+
+def test_encode_empty_and_single(cuda_lib, torch_dev):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, bits = 64, 4
+    R = O.rotation(d, 3).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    X = synth.mixture_corpus(1, d, 2, seed=1)
+    enc = O.encode(X, R, c32, t32, bits)
+    codes, scale = tq.encode(_t(torch, dev, X), _t(torch, dev, R), _t(torch, dev, c32), _t(torch, dev, t32), bits)
+    check_encode(codes.cpu().numpy(), scale.cpu().numpy(), X, enc, c32, t32, d, bits, "norm")
+    empty = torch.empty((0, d), dtype=torch.float32, device=dev)
+    codes, scale = tq.encode(empty, _t(torch, dev, R), _t(torch, dev, c32), _t(torch, dev, t32), bits)
+    assert codes.shape == (0, d * bits // 8)
+
+
+# ------------------------------------------------------------------- search --
+@pytest.fixture(scope="module")
+def tiny_config():
+    """The tiny exact-check workload: N=10,000, d=1536, 64-component mixture,
+    100 perturbed-corpus queries, 4-bit codes, top-10, no filtering."""
+    d, n, nq, bits = 1536, 10_000, 100, 4
+    X = synth.mixture_corpus(n, d, 64)
+    R = O.rotation(d, synth.SEED_ROTATION).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    enc = O.encode(X, R, c32, t32, bits)
+    src = synth.query_sources(n, nq)
+    Q = synth.perturb(X[src])
+    return dict(X=X, R=R, c32=c32, t32=t32, enc=enc, Q=Q, d=d, n=n, bits=bits)
+
+
+def _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, **kw):
+    ids, sc = tq.search(_t(torch, dev, Q), _t(torch, dev, R), _t(torch, dev, c32), bits,
+                        _t(torch, dev, packed), None if scale is None else _t(torch, dev, scale), k, **kw)
+    torch.cuda.synchronize()
+    return ids.cpu().numpy(), sc.cpu().numpy()
+
+
+@pytest.mark.parametrize("path", ["lut"])
+def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = tiny_config
+    k = 10
+    tq.set_search_path(path)
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                              c["enc"].scale, k)
+    finally:
+        tq.set_search_path("auto")
+    ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"])
+    allowed = np.ones_like(ref.scores64, dtype=bool)
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT)
+    exact, _ = O.exact_knn(c["X"], c["Q"], k)
+    assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
+
+
+@pytest.mark.parametrize("bits", [2, 3, 8])
+def test_search_bit_widths(cuda_lib, torch_dev, bits):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, n, nq, k = 1536, 4000, 20, 10
+    X = synth.mixture_corpus(n, d, 64, seed=42)
+    R = O.rotation(d, 1536).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    enc = O.encode(X, R, c32, t32, bits)
+    Q = synth.perturb(X[synth.query_sources(n, nq)])
+    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, enc.packed, enc.scale, k)
+    ref = O.search(Q, R, c32, bits, enc.packed, enc.scale, k, d)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_LUT)
+
+
+@pytest.mark.parametrize("d,n,nq,k", [(32, 5, 3, 10), (64, 64 * 3 + 17, 9, 7), (96, 1000, 8, 1),
+                                      (160, 777, 2, 256), (2048, 1500, 1, 5)])
+def test_search_shapes_and_edges(cuda_lib, torch_dev, d, n, nq, k):
+    """n below one block, ragged blocks, small d (lanes idle), k = 1 and 256,
+    the GEMV (nq <= 8) and GEMM (nq > 8) query rotations, d = 2048."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    bits = 4
+    rng = np.random.default_rng(d + n)
+    packed = synth.random_codes(n, d * bits // 8, seed=d)
+    scale = synth.random_scales(n, seed=n)
+    scale[0] = 0.0
+    R = O.rotation(d, 5).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    Q = synth.gaussian_rows(nq, d, seed=nq)
+    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    ref = O.search(Q, R, c32, bits, packed, scale, k, d)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_LUT)
+    del rng
+
+
+def test_search_unit_scale_and_ties(cuda_lib, torch_dev):
+    """scale=NULL means 1; duplicated rows tie exactly and come back by id."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, bits, k = 64, 4, 6
+    packed = synth.random_codes(300, d * bits // 8, seed=3)
+    packed = np.concatenate([packed, packed[[17, 17, 250]]])
+    R = O.rotation(d, 2).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    C = c32.astype(np.float64)[O.unpack(packed, d, bits)]
+    Q = (C[17] @ R.astype(np.float64))[None].astype(np.float32)   # R q = c[row 17]
+    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, None, k)
+    ref = O.search(Q, R, c32, bits, packed, None, k, d)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_LUT)
+    assert ids[0][:3].tolist() == [17, 300, 301]
+
+
+# ---------------------------------------------------------------- filtering --
+@pytest.fixture(scope="module")
+def filtered_corpus():
+    d, n, bits = 1536, 20_000, 4
+    X = synth.mixture_corpus(n, d, 256, seed=42)
+    R = O.rotation(d, 1536).astype(np.float32)
+    c32, t32 = _cb(d, bits)
+    enc = O.encode(X, R, c32, t32, bits)
+    src = synth.query_sources(n, 200)
+    Q = synth.perturb(X[src])
+    return dict(X=X, R=R, c32=c32, enc=enc, src=src, Q=Q, d=d, n=n, bits=bits)
+
+
+@pytest.mark.parametrize("T", [10, 100, 1000])
+@pytest.mark.parametrize("block", [64, 32])
+def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
+    """Zipf(1.1) tenants in interleaved order; 1 allowed tenant per query, 10%
+    of queries with 5 (Sec. III-B, the filtered workload)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    k = 10
+    tid, values = synth.zipf_tenants(c["n"], T)
+    off, allow = synth.allowlists(c["src"], tid, values)
+    filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=block)
+    assert filt.info() == {"n": c["n"], "block": block, "n_tenants": T}
+    ids, sc = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale,
+                          k, filter=filt, allow_off=_t(torch, dev, off),
+                          allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"],
+                   tid, off, allow)
+    allowed = O.allowed_mask(tid, off, allow, len(c["Q"]), c["n"])
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT)
+    exact, _ = O.exact_knn(c["X"], c["Q"], k, tid, off, allow)
+    assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
+    filt.close()
+
+
+def test_filter_edge_cases(cuda_lib, torch_dev):
+    """Empty allowlists, ids absent from the corpus, a tenant smaller than k,
+    and a filter allowing every tenant equal to no filter."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, n, bits, k = 64, 500, 4, 12
+    packed = synth.random_codes(n, d * bits // 8, seed=9)
+    scale = synth.random_scales(n, seed=9)
+    R = O.rotation(d, 9).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    tid = np.full(n, 7, np.uint32)
+    tid[::50] = 99                           # a tenant of 10 vectors (< k)
+    tid[3] = 12345
+    Q = synth.gaussian_rows(4, d, seed=4)
+    off = np.array([0, 0, 1, 3, 5], np.int64)
+    allow = np.array([99, 555, 12345, 7, 99], np.uint32)
+    filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=32)
+    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, filter=filt,
+                          allow_off=_t(torch, dev, off), allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    ref = O.search(Q, R, c32, bits, packed, scale, k, d, tid, off, allow)
+    allowed = O.allowed_mask(tid, off, allow, 4, n)
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT)
+    assert np.all(ids[0] == -1)              # empty allowlist
+    assert np.sum(ids[1] >= 0) == 10         # tenant of 10 vectors, k = 12
+    # every tenant allowed == unfiltered
+    off2 = np.array([0, 3, 6, 9, 12], np.int64)
+    allow2 = np.tile(np.array([7, 99, 12345], np.uint32), 4)
+    ids_f, sc_f = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, filter=filt,
+                              allow_off=_t(torch, dev, off2), allow_tenants=_t(torch, dev, allow2.view(np.int32)))
+    ids_u, sc_u = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    assert np.array_equal(ids_f, ids_u) and np.array_equal(sc_f, sc_u)
+    filt.close()
+
+
+def test_invalid_calls_on_gpu(cuda_lib, torch_dev):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, bits = 64, 4
+    Q = torch.zeros((2, d), device=dev)
+    R = torch.eye(d, device=dev)
+    c = torch.zeros(16, device=dev)
+    codes = torch.zeros((10, 32), dtype=torch.uint8, device=dev)
+    with pytest.raises(tq.TQError, match="workspace"):
+        tq.search(Q, R, c, bits, codes, None, 5, workspace=torch.zeros(16, dtype=torch.uint8, device=dev))
+    tid = torch.zeros(11, dtype=torch.int32, device=dev)
+    f = tq.Filter(tid)
+    with pytest.raises(tq.TQError, match="filter built for n=11"):
+        tq.search(Q, R, c, bits, codes, None, 5, filter=f, allow_off=torch.zeros(3, dtype=torch.int64, device=dev),
+                  allow_tenants=torch.zeros(1, dtype=torch.int32, device=dev))
+    f.close()

@@ -1,0 +1,137 @@
+"""libtq.so on the CPU: it loads, exports every symbol include/tq.h declares,
+its host-only math (tq_codebook, tq_rotation) matches the oracle, and every
+device call rejects invalid arguments before touching CUDA."""
+import ctypes as C
+import json
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as O
+import paper_2607_16973_gb300 as tq
+from paper_2607_16973_gb300 import _lib
+from paper_2607_16973_gb300.build import build
+from conftest import GOLDEN, ROOT
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build()
+    return tq.load()
+
+
+def _header_functions():
+    with open(os.path.join(ROOT, "include", "tq.h")) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(tq_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _header_functions()
+    assert "tq_search" in names and "tq_encode" in names and "tq_codebook" in names
+    for name in names:
+        assert hasattr(lib, name), name
+    assert set(names) == set(_lib.SIGNATURES), "binding and header disagree"
+    assert lib.tq_version() == 100
+
+
+@pytest.mark.parametrize("marginal", ["beta", "gauss"])
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_codebook_matches_oracle_golden(lib, marginal, bits):
+    with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+        e = [e for e in json.load(f)["entries"] if e["bits"] == bits and e["marginal"] == marginal][0]
+    c, t, D = tq.codebook(1536, bits, marginal)
+    want_c = np.asarray(e["centroids"])
+    want_t = np.asarray(e["boundaries"])
+    # float32 outputs: within one float32 ulp of the float64 oracle (the oracle's
+    # own fixed-point error is < 1e-9 relative at 8 bits)
+    ulp_c = np.spacing(np.abs(want_c).astype(np.float32)).astype(np.float64)
+    ulp_t = np.spacing(np.abs(want_t).astype(np.float32)).astype(np.float64)
+    assert np.all(np.abs(c - want_c) <= ulp_c + 2e-9 * np.abs(want_c))
+    assert np.all(np.abs(t - want_t) <= ulp_t + 2e-9 * np.abs(want_t) + 1e-30)
+    assert D == pytest.approx(e["distortion"], rel=1e-8)
+    assert t[len(t) // 2] == 0.0 and np.array_equal(c, -c[::-1])
+
+
+@pytest.mark.parametrize("d", [32, 96, 512])
+@pytest.mark.parametrize("bits", [2, 4])
+def test_codebook_matches_oracle_small_d(lib, d, bits):
+    c, t, D = tq.codebook(d, bits)
+    ref = O.codebook(d, bits)
+    assert np.allclose(c, ref.centroids, rtol=1.5e-7, atol=0)
+    assert np.allclose(t, ref.boundaries, rtol=1.5e-7, atol=1e-30)
+    assert D == pytest.approx(ref.distortion, rel=1e-9)
+
+
+def test_codebook_is_data_free_and_deterministic(lib):
+    a = tq.codebook(1536, 4)
+    b = tq.codebook(1536, 4)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1]) and a[2] == b[2]
+
+
+@pytest.mark.parametrize("d", [32, 160, 1536])
+def test_rotation_matches_oracle(lib, d):
+    R = tq.rotation(d, 1536)
+    ref = O.rotation(d, 1536).astype(np.float32)
+    diff = np.abs(R.astype(np.float64) - ref.astype(np.float64))
+    assert np.all(diff <= np.spacing(np.abs(ref)).astype(np.float64))
+    assert np.mean(R == ref) > 0.999
+
+
+def _status(fn, *args):
+    return fn(*args)
+
+
+def test_invalid_arguments_rejected_without_gpu(lib):
+    null = None
+    # codebook / rotation
+    assert lib.tq_codebook(4, 4, 0, null, null, null) == _lib.TQ_EINVAL
+    assert lib.tq_codebook(64, 9, 0, null, null, null) == _lib.TQ_EINVAL
+    assert lib.tq_codebook(64, 4, 7, null, null, null) == _lib.TQ_EINVAL
+    assert lib.tq_rotation(1, 0, null) == _lib.TQ_EINVAL
+    assert b"d=1" in lib.tq_last_error()
+    # encode: d not a multiple of 32, bad bits, bad scale mode, NULL pointers, misalignment
+    p = 4096
+    assert lib.tq_encode(p, 10, 48, p, p, p, 4, 0, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode(p, 10, 64, p, p, p, 5, 0, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode(p, 10, 64, p, p, p, 4, 9, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode(null, 10, 64, p, p, p, 4, 0, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode(p + 4, 10, 64, p, p, p, 4, 0, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode(null, 0, 64, null, null, null, 4, 0, null, null, null) == _lib.TQ_OK
+    # search
+    args = [p, 1, 64, p, p, 4, p, p, 100, null, null, null, 10, p, p, p, 1 << 20, null]
+
+    def search(**kw):
+        a = list(args)
+        names = ["Q", "nq", "d", "R", "cen", "bits", "codes", "scale", "n", "filter", "off",
+                 "ten", "k", "ids", "scores", "ws", "wsb", "stream"]
+        for k_, v in kw.items():
+            a[names.index(k_)] = v
+        return lib.tq_search(*a)
+
+    assert search(k=0) == _lib.TQ_EINVAL
+    assert search(k=257) == _lib.TQ_EINVAL
+    assert search(bits=1) == _lib.TQ_EINVAL
+    assert search(d=40) == _lib.TQ_EINVAL
+    assert search(n=0) == _lib.TQ_EINVAL
+    assert search(Q=null) == _lib.TQ_EINVAL
+    assert search(codes=p + 8) == _lib.TQ_EINVAL
+    assert search(ws=null) == _lib.TQ_EINVAL
+    assert search(nq=0) == _lib.TQ_OK
+    # filter
+    h = C.c_void_p()
+    assert lib.tq_filter_build(p, 10, 48, C.byref(h), null) == _lib.TQ_EINVAL
+    assert lib.tq_filter_build(p, 0, 64, C.byref(h), null) == _lib.TQ_EINVAL
+    assert lib.tq_filter_destroy(null) == _lib.TQ_OK
+    assert lib.tq_set_search_path(7) == _lib.TQ_EINVAL
+    assert lib.tq_profile_events(p, null) == _lib.TQ_EINVAL
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    monkeypatch.setattr(_lib, "_lib", None)
+    monkeypatch.setattr(_lib, "LIB_PATH", str(tmp_path / "libtq.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        _lib.load()
