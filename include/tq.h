@@ -191,6 +191,29 @@ tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
                     int k, int64_t* out_ids, float* out_scores, void* workspace,
                     size_t ws_bytes, void* stream);
 
+/*
+ * tq_search_static - tq_search without a workspace, for callers that cannot
+ * allocate device memory (for example a C host program or plugin that is
+ * handed device pointers for its inputs and outputs but owns no allocator, or
+ * a serving loop that must not call cudaMalloc, which can block, synchronise
+ * the device or fail under memory pressure mid-request).  The paper has no
+ * counterpart: it is an interface convenience of this library.
+ * Same arguments and results as tq_search (always the lookup scan), minus
+ * workspace/ws_bytes.  Its scratch is one 8 MiB device array per GPU,
+ * reserved when the library is loaded and held until the process exits; the
+ * call allocates nothing.  Sizes whose scratch (about nq*d*4 bytes of rotated
+ * queries plus nq*k*8 bytes per scan CTA of candidates) exceeds 8 MiB return
+ * TQ_EINVAL with the byte counts.  The first call on each device looks the
+ * array's device address up (make it before any stream capture).  All calls on
+ * a device share the array: calls whose work overlaps on the GPU (two streams
+ * or two threads) race and must be serialised by the caller.  Limit on d: 2048.
+ */
+tq_status tq_search_static(const float* Q, int64_t nq, int d, const float* R,
+                           const float* centroids, int bits, const uint8_t* codes,
+                           const float* scale, int64_t n, const tq_filter* filter,
+                           const int64_t* allow_off, const uint32_t* allow_tenants,
+                           int k, int64_t* out_ids, float* out_scores, void* stream);
+
 /* Selects the search kernels for later tq_search calls of the calling thread
  * (TQ_PATH_*).  AUTO is the default. */
 tq_status tq_set_search_path(int path);

@@ -11,11 +11,6 @@
 #include "tq_internal.h"
 #include "tq_kernels.h"
 
-struct tq_filter {
-  tq::FilterDev f;
-  int device = 0;
-};
-
 namespace tq {
 namespace {
 

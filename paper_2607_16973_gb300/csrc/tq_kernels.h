@@ -58,3 +58,10 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
 int device_sm_count();
 
 }  // namespace tq
+
+// Opaque handle of the C ABI (include/tq.h): the filter's device arrays and
+// the device they live on.
+struct tq_filter {
+  tq::FilterDev f;
+  int device = 0;
+};
