@@ -29,22 +29,31 @@ constexpr size_t kAlign = 256;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct SearchPlan {
-  int grid_x = 1;
-  size_t off_rot = 0, off_allow = 0, off_cs = 0, off_ci = 0, total = 0;
+  int grid_lut = 1, grid_mma = 0;
+  size_t off_status = 0, off_rot = 0, off_allow = 0, off_qpack = 0, off_cs = 0, off_ci = 0, total = 0;
 };
 
+// Workspace layout (both scan paths): status word | rotated queries | allow
+// bitmaps | fp16 query tiles (tensor-core path) | candidate scores | ids.
 SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
   SearchPlan p;
-  p.grid_x = scan_lut_grid_x(nq, n, k, bits, d);
+  p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
+  const bool mma = mma_supported(bits, d, k) && !filter;
+  p.grid_mma = mma ? scan_mma_grid_x(nq, n) : 0;
+  const int per_query = std::max(p.grid_lut, p.grid_mma) * k;
   size_t off = 0;
+  p.off_status = off;
+  off = align_up(off + sizeof(int));
   p.off_rot = off;
   off = align_up(off + (size_t)nq * d * sizeof(float));
   p.off_allow = off;
   if (filter) off = align_up(off + (size_t)nq * filter->f.words * sizeof(uint32_t));
+  p.off_qpack = off;
+  if (mma) off = align_up(off + mma_qpack_bytes(nq, d));
   p.off_cs = off;
-  off = align_up(off + (size_t)nq * p.grid_x * k * sizeof(float));
+  off = align_up(off + (size_t)nq * per_query * sizeof(float));
   p.off_ci = off;
-  off = align_up(off + (size_t)nq * p.grid_x * k * sizeof(int32_t));
+  off = align_up(off + (size_t)nq * per_query * sizeof(int32_t));
   p.total = off;
   return p;
 }
@@ -186,23 +195,36 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
       return fail(TQ_EINVAL, "tq_search: misaligned allowlist pointers");
   }
   const int path = tq::search_path();
-  if (path == TQ_PATH_MMA) return fail(TQ_EUNSUPPORTED, "tq_search: the MMA path is not built yet");
+  const bool can_mma = tq::mma_supported(bits, d, k) && !filter;
+  if (path == TQ_PATH_MMA && !can_mma)
+    return fail(TQ_EUNSUPPORTED, "tq_search: the tensor-core scan needs bits 2/4/8, k <= %d and no filter",
+                tq::kMaxKMma);
+  const bool use_mma = can_mma && (path == TQ_PATH_MMA || (path == TQ_PATH_AUTO && nq >= tq::kMmaMinBatch));
   const tq::SearchPlan p = tq::plan_search(nq, n, d, bits, k, filter);
   if (ws_bytes < p.total)
     return fail(TQ_EINVAL, "tq_search: workspace of %zu bytes, %zu needed", ws_bytes, p.total);
   cudaStream_t s = (cudaStream_t)stream;
   char* ws = static_cast<char*>(workspace);
+  int* status = reinterpret_cast<int*>(ws + p.off_status);
   float* qrot = reinterpret_cast<float*>(ws + p.off_rot);
   uint32_t* allow = filter ? reinterpret_cast<uint32_t*>(ws + p.off_allow) : nullptr;
   float* cs = reinterpret_cast<float*>(ws + p.off_cs);
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
   cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, s);
-  if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
-  if (e == cudaSuccess)
-    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, filter ? &filter->f : nullptr, allow,
-                            k, p.grid_x, cs, ci, s, (cudaEvent_t)tq::profile_start(),
-                            (cudaEvent_t)tq::profile_stop());
-  if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_x * k, k, out_ids, out_scores, s);
+  if (use_mma) {
+    if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int), s);
+    if (e == cudaSuccess)
+      e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, k, p.grid_mma, ws + p.off_qpack, cs, ci,
+                              status, s, (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
+    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, out_ids, out_scores, s);
+  } else {
+    if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
+    if (e == cudaSuccess)
+      e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, filter ? &filter->f : nullptr, allow,
+                              k, p.grid_lut, cs, ci, s, (cudaEvent_t)tq::profile_start(),
+                              (cudaEvent_t)tq::profile_stop());
+    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_lut * k, k, out_ids, out_scores, s);
+  }
   if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
   return tq::ok();
 }

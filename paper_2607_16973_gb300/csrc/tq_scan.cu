@@ -1,10 +1,10 @@
 // Search-side kernels: the lookup scan with fused top-k (Sec. II-B step 5,
 // Sec. III-B), per-query allow bitmaps, the filter build and the final merge.
 //
-// Lookup scan layout.  One warp scores one vector at a time.  The packed row
-// is cut into chunks of 16 codes (2*bits bytes); lane l owns chunks l, l+32,
-// l+64, ... of every row, so each load instruction of a warp reads a
-// contiguous run of the row and every lane always handles the same
+// Lookup scan layout.  One warp scores 8 consecutive vectors per step.  Each
+// packed row is cut into chunks of 16 codes (2*bits bytes); lane l owns chunks
+// l, l+32, l+64, ... of every row, so each load instruction of a warp reads a
+// contiguous run of one row and every lane always handles the same
 // coordinates.  Lane l keeps the rotated query's values for its coordinates
 // in registers and looks the centroid of each code up in a table replicated
 // across the 32 shared-memory banks (entry (code, lane) lives in bank lane), so
@@ -107,6 +107,7 @@ struct Chunk<4> {
     w0 = v.x;
     w1 = v.y;
   }
+  __device__ __forceinline__ void zero() { w0 = w1 = 0; }
   __device__ __forceinline__ uint32_t code(int t) const { return ((t < 8 ? w0 : w1) >> (4 * (t & 7))) & 15u; }
 };
 
@@ -114,6 +115,7 @@ template <>
 struct Chunk<2> {
   uint32_t w;
   __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const unsigned int*>(p)); }
+  __device__ __forceinline__ void zero() { w = 0; }
   __device__ __forceinline__ uint32_t code(int t) const { return (w >> (2 * t)) & 3u; }
 };
 
@@ -121,6 +123,7 @@ template <>
 struct Chunk<8> {
   uint4 w;
   __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const uint4*>(p)); }
+  __device__ __forceinline__ void zero() { w = make_uint4(0, 0, 0, 0); }
   __device__ __forceinline__ uint32_t code(int t) const {
     const uint32_t x = t < 4 ? w.x : t < 8 ? w.y : t < 12 ? w.z : w.w;
     return (x >> (8 * (t & 3))) & 255u;
@@ -134,9 +137,37 @@ struct Chunk<3> {
     const unsigned short* h = reinterpret_cast<const unsigned short*>(p);
     v = (uint64_t)__ldcs(h) | ((uint64_t)__ldcs(h + 1) << 16) | ((uint64_t)__ldcs(h + 2) << 32);
   }
+  __device__ __forceinline__ void zero() { v = 0; }
   __device__ __forceinline__ uint32_t code(int t) const { return (uint32_t)(v >> (3 * t)) & 7u; }
 };
 
+// Sums p[0..7] across the warp: afterwards lanes 4i..4i+3 hold the total of
+// p[i] (a transposed butterfly: 4 + 2 + 1 + 1 + 1 shuffles for 8 values).
+__device__ __forceinline__ float warp_sum8(float (&p)[8]) {
+  const int lane = threadIdx.x & 31;
+  const bool h16 = lane & 16, h8 = lane & 8, h4 = lane & 4;
+  float a[4], b[2];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float send = h16 ? p[i] : p[i + 4];
+    const float keep = h16 ? p[i + 4] : p[i];
+    a[i] = keep + __shfl_xor_sync(FULL, send, 16);
+  }
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float send = h8 ? a[i] : a[i + 2];
+    const float keep = h8 ? a[i + 2] : a[i];
+    b[i] = keep + __shfl_xor_sync(FULL, send, 8);
+  }
+  float c = (h4 ? b[1] : b[0]) + __shfl_xor_sync(FULL, h4 ? b[0] : b[1], 4);
+  c += __shfl_xor_sync(FULL, c, 2);
+  c += __shfl_xor_sync(FULL, c, 1);
+  return c;
+}
+
+// Each warp scores 8 consecutive vectors per step: all their code loads (and
+// their scales and tenants) are issued before any arithmetic, so a warp keeps
+// 8 x d*bits/8 bytes in flight.
 template <int BITS, int S>
 __global__ void __launch_bounds__(SCAN_NT, 2)
 k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
@@ -146,6 +177,7 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
            float* __restrict__ cand_s, int* __restrict__ cand_i) {
   constexpr int L = 1 << BITS;
   constexpr int CB = 2 * BITS;
+  constexpr int V = 8;  // vectors per warp step; a CTA step covers 64
   extern __shared__ __align__(16) unsigned char smem_raw[];
   float* ctab = reinterpret_cast<float*>(smem_raw);  // [L][32], entry (c, lane) in bank lane
   float* ls = ctab + L * 32;                          // [P] scores; warp w's list at [w*k, w*k+k)
@@ -175,37 +207,61 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
   int cnt = 0;
   float th_s = -INFINITY;
   int th_i = INT_MAX;
-  const int nfb = (n + fblock - 1) / fblock;
-  for (int b = blockIdx.x; b < nfb; b += gridDim.x) {
-    if (ab) {
+  const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
+  const int my = (lane >> 2) & 7;  // the vector whose total this lane ends up holding
+  for (int st = blockIdx.x; st < nsteps; st += gridDim.x) {
+    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+    if (v0 >= n) continue;
+    if (ab) {  // the warp's 8 vectors lie in one filter block (block is 32 or 64)
+      const int fb = v0 / fblock;
       uint32_t any = 0;
-      for (int w = lane; w < words; w += 32) any |= __ldg(block_bits + (size_t)b * words + w) & __ldg(ab + w);
-      if (!__any_sync(FULL, any != 0u)) continue;  // no allowed vector in this block
+      for (int w = lane; w < words; w += 32) any |= __ldg(block_bits + (size_t)fb * words + w) & __ldg(ab + w);
+      if (!__any_sync(FULL, any != 0u)) continue;  // no allowed vector: skip before reading codes
     }
-    const int v_end = min(n, (b + 1) * fblock);
-    for (int v = b * fblock + warp; v < v_end; v += SCAN_WARPS) {
-      const uint8_t* row = codes + (size_t)v * row_bytes;
-      float acc = 0.f;
+    const int vm = v0 + my;
+    float sc_my = 0.f;
+    uint32_t ten_my = 0;
+    if ((lane & 3) == 0 && vm < n) {
+      sc_my = scale ? __ldg(scale + vm) : 1.0f;
+      if (ab) ten_my = __ldg(dense + vm);
+    }
+    Chunk<BITS> ch[V][S];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      const uint8_t* row = codes + (size_t)(v0 + i) * row_bytes;
 #pragma unroll
       for (int s = 0; s < S; ++s) {
         const int chunk = lane + 32 * s;
-        if (chunk < nchunks) {
-          Chunk<BITS> c;
-          c.load(row + chunk * CB);
-#pragma unroll
-          for (int t = 0; t < 16; ++t) acc = fmaf(qr[s][t], ctab[(c.code(t) << 5) | lane], acc);
-        }
+        if (v0 + i < n && chunk < nchunks) ch[i][s].load(row + chunk * CB);
+        else ch[i][s].zero();
       }
+    }
+    float p[V];
 #pragma unroll
-      for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(FULL, acc, o);
-      const float score = scale ? acc * __ldg(scale + v) : acc;
-      bool allowed = true;
-      if (ab) {
-        const uint32_t t = __ldg(dense + v);
-        allowed = (__ldg(ab + (t >> 5)) >> (t & 31)) & 1u;
-      }
-      if (allowed && better(score, v, th_s, th_i)) {
-        warp_insert(wl_s, wl_i, k, cnt, score, v);
+    for (int i = 0; i < V; ++i) {
+      float acc = 0.f;
+#pragma unroll
+      for (int s = 0; s < S; ++s)
+#pragma unroll
+        for (int t = 0; t < 16; ++t) acc = fmaf(qr[s][t], ctab[(ch[i][s].code(t) << 5) | lane], acc);
+      p[i] = acc;
+    }
+    const float total = warp_sum8(p);
+    float score = -INFINITY;
+    bool cand = false;
+    if ((lane & 3) == 0 && vm < n) {
+      score = total * sc_my;
+      const bool allowed = !ab || ((__ldg(ab + (ten_my >> 5)) >> (ten_my & 31)) & 1u);
+      cand = allowed && better(score, vm, th_s, th_i);
+    }
+    unsigned m = __ballot_sync(FULL, cand);
+    while (m) {  // in vector order; re-checked against the moving threshold
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      const float s = __shfl_sync(FULL, score, src);
+      const int vv = v0 + ((src >> 2) & 7);
+      if (better(s, vv, th_s, th_i)) {
+        warp_insert(wl_s, wl_i, k, cnt, s, vv);
         cnt = min(cnt + 1, k);
         if (cnt == k) {
           th_s = wl_s[k - 1];

@@ -9,7 +9,7 @@ import pytest
 
 import oracle as O
 from paper_2607_16973_gb300 import synth
-from parity import TOL_LUT, check_encode, check_topk
+from parity import TOL_LUT, TOL_MMA, check_encode, check_topk
 
 pytestmark = pytest.mark.gpu
 
@@ -30,19 +30,21 @@ def corpus(cuda_lib):
                 d_packed=T(packed), d_scale=T(scale), d_R=T(R), d_c=T(cb.centroids32), T=T)
 
 
-@pytest.mark.parametrize("batch,sampled", [(1, [0]), (1024, [0, 517, 1023])])
-def test_fullsize_search_sampled(cuda_lib, corpus, batch, sampled):
+@pytest.mark.parametrize("batch,sampled,tol", [(1, [0], TOL_LUT), (1024, [0, 517, 1023], TOL_MMA)])
+def test_fullsize_search_sampled(cuda_lib, corpus, batch, sampled, tol):
+    """Batch 1 runs the lookup scan, batch 1024 the tensor-core scan (AUTO)."""
     import torch
     tq = cuda_lib
     c = corpus
     Q = synth.gaussian_rows(batch, D, seed=batch)
+    Q /= np.linalg.norm(Q, axis=1, keepdims=True)   # unit queries, as in the workload
     ids, sc = tq.search(c["T"](Q), c["d_R"], c["d_c"], BITS, c["d_packed"], c["d_scale"], K)
     torch.cuda.synchronize()
     ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
     assert np.all(ids >= 0) and np.all(ids < N)
     for q in sampled:
         ref = O.search(Q[q:q + 1], c["R"], c["c32"], BITS, c["packed"], c["scale"], K, D)
-        check_topk(ids[q:q + 1], sc[q:q + 1], ref.ids, ref.scores64, np.ones((1, N), bool), K, TOL_LUT)
+        check_topk(ids[q:q + 1], sc[q:q + 1], ref.ids, ref.scores64, np.ones((1, N), bool), K, tol)
 
 
 def test_fullsize_encode_sampled_rows(cuda_lib, corpus):

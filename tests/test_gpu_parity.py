@@ -10,7 +10,7 @@ import pytest
 import oracle as O
 from paper_2607_16973_gb300 import synth
 from conftest import GOLDEN
-from parity import TOL_LUT, check_encode, check_topk, recall
+from parity import TOL_LUT, TOL_MMA, check_encode, check_topk, recall
 
 pytestmark = pytest.mark.gpu
 
@@ -105,7 +105,7 @@ def _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, **kw):
     return ids.cpu().numpy(), sc.cpu().numpy()
 
 
-@pytest.mark.parametrize("path", ["lut"])
+@pytest.mark.parametrize("path", ["lut", "mma"])
 def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
     torch, dev = torch_dev
     tq = cuda_lib
@@ -119,13 +119,13 @@ def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
         tq.set_search_path("auto")
     ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"])
     allowed = np.ones_like(ref.scores64, dtype=bool)
-    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT)
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT if path == "lut" else TOL_MMA)
     exact, _ = O.exact_knn(c["X"], c["Q"], k)
     assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
 
 
-@pytest.mark.parametrize("bits", [2, 3, 8])
-def test_search_bit_widths(cuda_lib, torch_dev, bits):
+@pytest.mark.parametrize("bits,path", [(2, "lut"), (3, "lut"), (8, "lut"), (2, "mma"), (8, "mma")])
+def test_search_bit_widths(cuda_lib, torch_dev, bits, path):
     torch, dev = torch_dev
     tq = cuda_lib
     d, n, nq, k = 1536, 4000, 20, 10
@@ -134,9 +134,14 @@ def test_search_bit_widths(cuda_lib, torch_dev, bits):
     c32, t32 = _cb(d, bits)
     enc = O.encode(X, R, c32, t32, bits)
     Q = synth.perturb(X[synth.query_sources(n, nq)])
-    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, enc.packed, enc.scale, k)
+    tq.set_search_path(path)
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, enc.packed, enc.scale, k)
+    finally:
+        tq.set_search_path("auto")
     ref = O.search(Q, R, c32, bits, enc.packed, enc.scale, k, d)
-    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_LUT)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k,
+               TOL_LUT if path == "lut" else TOL_MMA)
 
 
 @pytest.mark.parametrize("d,n,nq,k", [(32, 5, 3, 10), (64, 64 * 3 + 17, 9, 7), (96, 1000, 8, 1),
@@ -265,3 +270,46 @@ def test_invalid_calls_on_gpu(cuda_lib, torch_dev):
         tq.search(Q, R, c, bits, codes, None, 5, filter=f, allow_off=torch.zeros(3, dtype=torch.int64, device=dev),
                   allow_tenants=torch.zeros(1, dtype=torch.int32, device=dev))
     f.close()
+
+
+# ------------------------------------------------------- tensor-core scan --
+@pytest.mark.parametrize("bits,d,n,nq,k", [(4, 1536, 3000, 130, 10), (2, 1536, 1000, 17, 5),
+                                           (8, 1536, 777, 64, 8), (4, 64, 513, 200, 1),
+                                           (4, 2048, 2049, 129, 64), (4, 128, 255, 1, 3)])
+def test_search_mma_parity(cuda_lib, torch_dev, bits, d, n, nq, k):
+    """Query tiles of 128 with a ragged last tile, vector tiles of 256 with a
+    ragged tail (rows past n are filled with zeros by the tensor map), one
+    query, k = 1 and 64, 2/4/8-bit codes (fp16 products, float32 sums)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    packed = synth.random_codes(n, d * bits // 8, seed=bits * n)
+    scale = synth.random_scales(n, seed=n + 1)
+    R = O.rotation(d, 7).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    Q = synth.gaussian_rows(nq, d, seed=nq + d)
+    Q /= np.linalg.norm(Q, axis=1, keepdims=True)   # unit queries, as in the workloads (fp16 error ~ |q|)
+    tq.set_search_path("mma")
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    finally:
+        tq.set_search_path("auto")
+    ref = O.search(Q, R, c32, bits, packed, scale, k, d)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_MMA)
+
+
+def test_search_mma_unsupported(cuda_lib, torch_dev):
+    """Forcing the tensor-core scan where it does not apply is an error, not a
+    silent switch: 3-bit codes, k > 64, d not a multiple of 64, a filter."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    tq.set_search_path("mma")
+    try:
+        for bits, d, k in ((3, 1536, 5), (4, 1536, 65), (4, 96, 5)):
+            Q = torch.zeros((4, d), device=dev)
+            R = torch.eye(d, device=dev)
+            c = torch.zeros(1 << bits, device=dev)
+            codes = torch.zeros((100, d * bits // 8), dtype=torch.uint8, device=dev)
+            with pytest.raises(tq.TQError, match="TQ_EUNSUPPORTED"):
+                tq.search(Q, R, c, bits, codes, None, k)
+    finally:
+        tq.set_search_path("auto")
