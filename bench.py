@@ -42,7 +42,11 @@ CONFIGS = {
     "scale": dict(n=999_000, d=1536, bits=4, clusters=1024, pool=10_000, k=5, batches=[1, 1024]),
     "c2": dict(n=100_000, d=1536, bits=4, clusters=256, pool=1_000, k=10, batches=[1, 256]),
     "tiny": dict(n=10_000, d=1536, bits=4, clusters=64, pool=100, k=10, batches=[1, 100]),
+    # profiling case: codes (192 MB) larger than L2, a few GB on the device at most
+    "prof": dict(n=250_000, d=1536, bits=4, clusters=256, pool=2_048, k=5, batches=[1, 1024]),
 }
+
+MMA_MIN_BATCH = 16  # tq_search's AUTO switch to the tensor-core scan (bits 2/4/8, k <= 64, no filter)
 
 METRIC = "queries/sec at 999Kx1536 4-bit top-5 (batch 1 / 1024); % of HBM / TC roofline"
 
@@ -72,21 +76,27 @@ def source_hash(*files):
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel_file: str, profile_md: str):
+def recorded_traffic(kernel_file: str, profile_md: str, scale_to: int):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
-    the current kernel source (the summary records the source hash)."""
+    the current kernel source (the summary records the source hash).  The
+    summary is captured on a smaller corpus of `captured_n` vectors; traffic
+    grows with the corpus, so it is scaled to `scale_to` vectors."""
     path = os.path.join(ROOT, "profiles", profile_md)
     if not os.path.exists(path):
         return None
     want = source_hash(kernel_file)
-    got_hash, traffic = None, None
+    got_hash, traffic, cap_n = None, None, None
     with open(path) as f:
         for line in f:
             if line.startswith("source_sha256_16:"):
                 got_hash = line.split(":", 1)[1].strip()
             if line.startswith("dram_bytes_per_launch:"):
                 traffic = float(line.split(":", 1)[1].strip())
-    return traffic if got_hash == want else None
+            if line.startswith("captured_n:"):
+                cap_n = int(line.split(":", 1)[1].strip())
+    if got_hash != want or traffic is None or not cap_n:
+        return None
+    return traffic * scale_to / cap_n
 
 
 class ClockSampler:
@@ -360,15 +370,28 @@ def run_ours(args, cfg, rank, world):
             ms = float(tt.item())
         scan_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
         qps = B * args.steps * world / (ms / 1e3)
-        # roofline of the scan kernel: the corpus (codes + scales) read once per launch
         alg_bytes = n * (d * bits // 8 + 4)
-        achieved = alg_bytes / (scan_ms / 1e3) / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
-                "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu",
-                                            f"scan_lut_{n // 1000}k_b{B}.md"),
-                "kernel": "k_scan_lut", "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
-                "frac_of_8tbs_nominal": achieved / 8000.0}
+        if B >= MMA_MIN_BATCH and bits in (2, 4, 8) and k <= 64:
+            # tensor-core scan: 2*n*d*B flops per launch against the dense fp16/bf16
+            # peak (same rate), sustained figure since it runs inside a long loop
+            flops = 2.0 * n * d * B
+            achieved = flops / (scan_ms / 1e3) / 1e12
+            peak = pk["bf16_tflops_sustained"]
+            roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "frac_of": pk["source"] + " (sustained bf16 = fp16 dense rate)",
+                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_mma.cu", "scan_mma_prof.md",
+                                                scale_to=n),
+                    "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": scan_ms,
+                    "hbm_gbs_of_corpus": alg_bytes / (scan_ms / 1e3) / 1e9}
+        else:
+            # lookup scan: the corpus (codes + scales) read once per launch
+            achieved = alg_bytes / (scan_ms / 1e3) / 1e9
+            roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                    "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
+                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu", "scan_lut_prof.md",
+                                                scale_to=n),
+                    "kernel": "k_scan_lut", "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
+                    "frac_of_8tbs_nominal": achieved / 8000.0}
         # e2e through the public API with host buffers
         qh = torch.empty((B, d), dtype=torch.float32).pin_memory()
         qh.copy_(torch.from_numpy(Qpool[:B]))

@@ -39,7 +39,7 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   SearchPlan p;
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
   const bool mma = mma_supported(bits, d, k) && !filter;
-  p.grid_mma = mma ? scan_mma_grid_x(nq, n) : 0;
+  p.grid_mma = mma ? scan_mma_grid_x(nq, n, k, bits) : 0;
   const int per_query = std::max(p.grid_lut, p.grid_mma) * k;
   size_t off = 0;
   p.off_status = off;

@@ -48,7 +48,7 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
 
 // Tensor-core decode-GEMM scan (bits 2, 4, 8; k <= kMaxKMma; unfiltered).
 bool mma_supported(int bits, int d, int k);
-int scan_mma_grid_x(int64_t nq, int64_t n);
+int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits);
 size_t mma_qpack_bytes(int64_t nq, int d);
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, int k, int grid_x,

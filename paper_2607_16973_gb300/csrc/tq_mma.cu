@@ -4,16 +4,16 @@
 // vectors on N (256 per MMA), fp16 operands and fp32 accumulation in tensor
 // memory (TMEM).  One CTA owns one query tile and a strided set of 256-vector
 // tiles.  Roles (warp-specialised, 10 warps):
-//   warps 0-3  decoders: expand one K-block (64 coordinates) of packed codes,
+//   warps 0-7  decoders: expand one K-block (64 coordinates) of packed codes,
 //              brought to shared memory by TMA, into fp16 centroid values laid
 //              out as the K-major, 128-byte-swizzled B operand;
-//   warps 4-7  epilogue: read the 128 x 256 fp32 accumulator from TMEM (one
+//   warps 8-11 epilogue: read the 128 x 256 fp32 accumulator from TMEM (one
 //              query per thread), apply the per-vector scale and keep each
 //              query's top-k in a thread-private sorted list;
-//   warp 8     producer: TMA of the code tile and a 1-D bulk copy of the
+//   warp 12    producer: TMA of the code tile and a 1-D bulk copy of the
 //              pre-swizzled fp16 query block, one mbarrier per stage;
 //              allocates TMEM;
-//   warp 9     MMA issuer: one thread issues tcgen05.mma (M=128, N=256, K=16)
+//   warp 13    MMA issuer: one thread issues tcgen05.mma (M=128, N=256, K=16)
 //              and commits completion to mbarriers.
 // TMEM holds two 256-column accumulators so the epilogue of one vector tile
 // overlaps the MMAs of the next.  Every wait is bounded: on timeout the CTA
@@ -37,8 +37,14 @@ namespace {
 constexpr int MMA_M = 128;            // queries per tile
 constexpr int MMA_N = 256;            // vectors per tile
 constexpr int KB = 64;                // coordinates per K-block (128 B of fp16)
-constexpr int STAGES = 2;
-constexpr int NTHREADS = 320;
+constexpr int MAX_CST = 8;  // raw code tiles in flight (HBM latency)
+constexpr int RAW_ROW_MAX = 128;  // bytes of each row one code tile carries (one 128-B line)
+constexpr int MAX_AST = 4;  // query blocks in flight (L2-resident)
+constexpr int BST = 2;      // decoded fp16 tiles
+constexpr int NTHREADS = 480;
+constexpr int DEC_WARPS = 8, DEC_THREADS = DEC_WARPS * 32;
+constexpr int EPI_WARP0 = 8, CODE_WARP = 12, MMA_WARP = 13, QUERY_WARP = 14;
+constexpr uint32_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
 constexpr int A_BYTES = MMA_M * KB * 2;   // 16 KB
 constexpr int B_BYTES = MMA_N * KB * 2;   // 32 KB
 constexpr long long WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
@@ -171,110 +177,197 @@ __device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
 }
 
 struct MmaSmem {
-  uint32_t a, b, raw, tab, scale, lists_s, lists_i, bars, total;
+  uint32_t a, b, raw, tab, scale, scr, lists_s, lists_i, bars, total;
 };
 
 template <int BITS>
 __host__ __device__ constexpr int raw_bytes_per_row() { return KB * BITS / 8; }
 
+// 4-bit codes decode in registers (no table); 2- and 8-bit use a table
+// replicated in all 32 banks (entry e of lane l at e*32 + l).
 template <int BITS>
 __host__ __device__ constexpr int tab_bytes() {
-  return BITS == 4 ? 256 * 32 * 4 : BITS == 2 ? 16 * 32 * 4 : 256 * 32 * 2;
+  return BITS == 4 ? 0 : BITS == 2 ? 16 * 32 * 4 : 256 * 32 * 2;
 }
 
-template <int BITS>
-__host__ __device__ inline MmaSmem mma_smem_layout(int k) {
+// Shared-memory plan for QT query tiles per CTA, `cst` raw code stages and
+// `ast` query stages.
+template <int BITS, int QT>
+__host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int rr) {
   MmaSmem L{};
   uint32_t off = 0;
   L.a = off;
-  off += STAGES * A_BYTES;
+  off += (uint32_t)ast * QT * A_BYTES;
   L.b = off;
-  off += STAGES * B_BYTES;
+  off += BST * B_BYTES;
   L.raw = off;
-  off += STAGES * MMA_N * raw_bytes_per_row<BITS>();
+  off += (uint32_t)cst * MMA_N * rr;
   L.tab = off;
   off += tab_bytes<BITS>();
   L.scale = off;
   off += MMA_N * 4;
+  L.scr = off;  // epilogue: 32 candidate scores per thread, [32][128]
+  off += 32 * MMA_M * 4;
   L.lists_s = off;
-  off += (uint32_t)k * MMA_M * 4;
+  off += (uint32_t)QT * k * MMA_M * 4;
   L.lists_i = off;
-  off += (uint32_t)k * MMA_M * 4;
+  off += (uint32_t)QT * k * MMA_M * 4;
   off = (off + 15) & ~15u;
   L.bars = off;
-  off += 16 * 8;
+  off += 48 * 8;
   L.total = off + 1024;  // slack to align the base to 1024 bytes
   // at most one CTA per SM: each allocates all 512 TMEM columns
   if (L.total < 116u * 1024u) L.total = 116u * 1024u;
   return L;
 }
 
+struct MmaPlan {
+  int qt = 1, cst = 2, ast = 2, rr = RAW_ROW_MAX;  // rr: bytes of each row per code tile
+  uint32_t smem = 0;
+};
+
+// Picks query tiles per CTA and ring depths that fit in shared memory:
+// prefer two query tiles per decoded code tile, then deep code prefetch.
 template <int BITS>
+MmaPlan mma_plan(int64_t nq, int k) {
+  MmaPlan best;
+  for (int qt = (nq > MMA_M ? 2 : 1); qt >= 1; --qt) {
+    for (int rr = RAW_ROW_MAX; rr >= 64; rr >>= 1) {
+      for (int ast = 3; ast >= 2; --ast) {
+        for (int cst = MAX_CST; cst >= 2; --cst) {
+          const uint32_t need = qt == 2 ? mma_smem_layout<BITS, 2>(k, cst, ast, rr).total
+                                        : mma_smem_layout<BITS, 1>(k, cst, ast, rr).total;
+          if (need <= kMaxDynSmem) {
+            best.qt = qt;
+            best.cst = cst;
+            best.ast = ast;
+            best.rr = rr;
+            best.smem = need;
+            return best;
+          }
+        }
+      }
+    }
+  }
+  best.smem = 0;  // does not fit
+  return best;
+}
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+  return d;
+}
+
+// Eight 4-bit codes (nibble i of w is code i) -> eight fp16 centroids, in
+// registers.  tl[j] / th[j] hold the low / high bytes of the fp16 centroids
+// 4j .. 4j+3.  A byte permute picks table bytes by the code's low 3 bits from
+// entries 0-7 and 8-15; the sign-replicate selector mode turns each code's
+// bit 3 into a 0x00/0xFF byte mask that chooses between the two.
+__device__ __forceinline__ uint4 decode8_4bit(uint32_t w, const uint32_t (&tl)[4], const uint32_t (&th)[4]) {
+  const uint32_t sel = w & 0x77777777u;
+  const uint32_t w4 = w << 4;
+  uint32_t o[4];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const uint32_t sh = h ? sel >> 16 : sel;
+    const uint32_t m = prmt(w4, w, h ? 0xFBEAu : 0xD9C8u);  // byte i = 0xFF iff code 4h+i >= 8
+    const uint32_t lo = (prmt(tl[0], tl[1], sh) & ~m) | (prmt(tl[2], tl[3], sh) & m);
+    const uint32_t hi = (prmt(th[0], th[1], sh) & ~m) | (prmt(th[2], th[3], sh) & m);
+    o[2 * h] = prmt(lo, hi, 0x5140u);
+    o[2 * h + 1] = prmt(lo, hi, 0x7362u);
+  }
+  return make_uint4(o[0], o[1], o[2], o[3]);
+}
+
+// Lane 0 polls the barrier for the whole warp.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
+                                          int where) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort_flag, err, where) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+template <int BITS, int QT>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,
            const float* __restrict__ centroids, const float* __restrict__ scale, int n, int nq, int d,
-           int k, float* __restrict__ cand_s, int* __restrict__ cand_i, int* __restrict__ err) {
+           int k, int cst, int ast, int rr, int sub, float* __restrict__ cand_s, int* __restrict__ cand_i,
+           int* __restrict__ err) {
   constexpr int RAWB = raw_bytes_per_row<BITS>();
+  // A code tile carries `sub` consecutive K-blocks of 256 rows: rows of
+  // sub*RAWB bytes (128 B, one full line, when d allows), stored with the
+  // 128-B swizzle in that case so the decoders' reads do not conflict.
+  const int rrow = sub * RAWB;
+  const bool swz = rrow == 128;
+  constexpr int NSETS = 2 / QT;  // accumulator sets in TMEM (2 = double buffered)
   extern __shared__ unsigned char smem_dyn[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_dyn) + 1023) & ~(uintptr_t)1023);
-  const MmaSmem L = mma_smem_layout<BITS>(k);
+  const MmaSmem L = mma_smem_layout<BITS, QT>(k, cst, ast, rr);
   unsigned char* sA = base + L.a;
   unsigned char* sB = base + L.b;
   unsigned char* sRaw = base + L.raw;
   float* sScale = reinterpret_cast<float*>(base + L.scale);
+  float* scr = reinterpret_cast<float*>(base + L.scr);
   float* lst_s = reinterpret_cast<float*>(base + L.lists_s);
   int* lst_i = reinterpret_cast<int*>(base + L.lists_i);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
-  uint64_t* full = bars;                 // [STAGES] TMA bytes landed
-  uint64_t* empty = bars + 2;            // [STAGES] MMAs done reading the stage
-  uint64_t* dec = bars + 4;              // [STAGES] decoded B written
-  uint64_t* acc_full = bars + 6;         // [2] accumulator complete
-  uint64_t* acc_empty = bars + 8;        // [2] accumulator read out
-  uint64_t* fin = bars + 10;             // all MMAs of this CTA complete
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 12);
+  uint64_t* cfull = bars;                      // [MAX_CST] code tile landed
+  uint64_t* cempty = bars + 8;                 // [MAX_CST] code tile decoded (stage free)
+  uint64_t* afull = bars + 16;                 // [MAX_AST] query block(s) landed
+  uint64_t* aempty = bars + 20;                // [MAX_AST] MMAs done with the query block(s)
+  uint64_t* dec = bars + 24;                   // [BST] decoded B tile written
+  uint64_t* bempty = bars + 26;                // [BST] MMAs done with the decoded tile
+  uint64_t* acc_full = bars + 28;              // [NSETS] accumulators complete
+  uint64_t* acc_empty = bars + 30;             // [NSETS] accumulators read out
+  uint64_t* fin = bars + 32;                   // all MMAs of this CTA complete
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 33);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 34);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int qt = blockIdx.y;
+  const int qt0 = blockIdx.y * QT;                     // first query tile of this CTA
+  const int nqt = (nq + MMA_M - 1) / MMA_M;
+  const int qts = min(QT, nqt - qt0);                  // query tiles present (1..QT)
   const int kblocks = d / KB;
   const int ntiles = (n + MMA_N - 1) / MMA_N;
   const int my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
-  // decode table, replicated in all 32 banks: entry e for lane l at e*32 + l
-  if (BITS == 4) {
-    uint32_t* tab = reinterpret_cast<uint32_t*>(base + L.tab);
-    for (int i = tid; i < 256 * 32; i += NTHREADS) {
-      const int e = i >> 5;
-      const __half2 h = __floats2half2_rn(centroids[e & 15], centroids[e >> 4]);
-      tab[i] = *reinterpret_cast<const uint32_t*>(&h);
-    }
-  } else if (BITS == 2) {
+  if (BITS == 2) {
     uint32_t* tab = reinterpret_cast<uint32_t*>(base + L.tab);
     for (int i = tid; i < 16 * 32; i += NTHREADS) {
       const int e = i >> 5;
       const __half2 h = __floats2half2_rn(centroids[e & 3], centroids[e >> 2]);
       tab[i] = *reinterpret_cast<const uint32_t*>(&h);
     }
-  } else {
+  } else if (BITS == 8) {
     __half* tab = reinterpret_cast<__half*>(base + L.tab);
     for (int i = tid; i < 256 * 32; i += NTHREADS) tab[i] = __float2half_rn(centroids[i >> 5]);
   }
   if (tid == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(full + s, 1);
-      mbar_init(empty + s, 1);
-      mbar_init(dec + s, 128);
+    for (int s = 0; s < MAX_CST; ++s) {
+      mbar_init(cfull + s, 1);
+      mbar_init(cempty + s, DEC_WARPS);  // one arrival per decoder warp
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int s = 0; s < MAX_AST; ++s) {
+      mbar_init(afull + s, 1);
+      mbar_init(aempty + s, 1);
+    }
+    for (int s = 0; s < BST; ++s) {
+      mbar_init(dec + s, DEC_WARPS);
+      mbar_init(bempty + s, 1);
+    }
+    for (int b = 0; b < NSETS; ++b) {
       mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, 128);
+      mbar_init(acc_empty + b, 4);       // one arrival per epilogue warp
     }
     mbar_init(fin, 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 8) {
+  if (warp == CODE_WARP) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 512;" ::"r"(smem_u32(tmem_slot)));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
@@ -284,105 +377,169 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
   const uint32_t tmem = *tmem_slot;
   const int total_it = my_tiles * kblocks;
 
-  if (warp == 8) {
-    // ---------------------------------------------------------- producer
+  if (warp == CODE_WARP) {
+    // ------------------------------------------------- code tiles (TMA, HBM)
+    if (lane == 0) {
+      int issued = 0;
+      const int total_loads = total_it / sub;
+      for (int ld = 0; ld < total_loads; ++ld) {
+        const int s = ld % cst, use = ld / cst;
+        if (use > 0 && !mbar_wait(cempty + s, (use - 1) & 1, abort_flag, err, 1)) break;
+        const int it = ld * sub;
+        const int t = blockIdx.x + (it / kblocks) * gridDim.x;
+        const int kb = it % kblocks;
+        mbar_arrive_expect_tx(cfull + s, MMA_N * rrow);
+        tma_load_2d(sRaw + s * MMA_N * rr, &codes_map, kb * RAWB, t * MMA_N, cfull + s);
+        issued = ld + 1;
+      }
+      // never leave with copies in flight: wait (bounded) for the last one of each stage
+      for (int s = 0; s < cst && s < issued; ++s) mbar_wait_drain(cfull + s, ((issued - 1 - s) / cst) & 1);
+    }
+  } else if (warp == QUERY_WARP) {
+    // ------------------------------------------ query blocks (bulk copy, L2)
     if (lane == 0) {
       int issued = 0;
       for (int it = 0; it < total_it; ++it) {
-        const int s = it % STAGES;
-        const int use = it / STAGES;
-        if (use > 0 && !mbar_wait(empty + s, (use - 1) & 1, abort_flag, err, 1)) break;
-        const int t = blockIdx.x + (it / kblocks) * gridDim.x;
+        const int s = it % ast, use = it / ast;
+        if (use > 0 && !mbar_wait(aempty + s, (use - 1) & 1, abort_flag, err, 6)) break;
         const int kb = it % kblocks;
-        mbar_arrive_expect_tx(full + s, A_BYTES + MMA_N * RAWB);
-        tma_load_2d(sRaw + s * MMA_N * RAWB, &codes_map, kb * RAWB, t * MMA_N, full + s);
-        bulk_load(sA + s * A_BYTES, qpack + ((size_t)qt * kblocks + kb) * (A_BYTES / 2), A_BYTES, full + s);
+        mbar_arrive_expect_tx(afull + s, qts * A_BYTES);
+        for (int j = 0; j < qts; ++j)
+          bulk_load(sA + (s * QT + j) * A_BYTES, qpack + ((size_t)(qt0 + j) * kblocks + kb) * (A_BYTES / 2),
+                    A_BYTES, afull + s);
         issued = it + 1;
       }
-      // never leave with copies in flight: wait (bounded) for the last one of each stage
-      for (int s = 0; s < STAGES && s < issued; ++s) {
-        const int last_use = (issued - 1 - s) / STAGES;
-        mbar_wait_drain(full + s, last_use & 1);
-      }
+      for (int s = 0; s < ast && s < issued; ++s) mbar_wait_drain(afull + s, ((issued - 1 - s) / ast) & 1);
     }
-  } else if (warp == 9) {
+  } else if (warp == MMA_WARP) {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
+      int bs = 0, bpar = 0, as = 0, apar = 0, kb = 0, tile_i = 0, set = 0, spar = 0;
       for (int it = 0; it < total_it; ++it) {
-        const int s = it % STAGES;
-        const int tile_i = it / kblocks;
-        const int kb = it % kblocks;
-        const int buf = tile_i & 1;
-        if (kb == 0 && tile_i >= 2 && !mbar_wait(acc_empty + buf, ((tile_i >> 1) - 1) & 1, abort_flag, err, 2))
-          break;
-        if (!mbar_wait(dec + s, (it / STAGES) & 1, abort_flag, err, 3)) break;
+        if (kb == 0 && tile_i >= NSETS && !mbar_wait(acc_empty + set, spar ^ 1, abort_flag, err, 2)) break;
+        if (!mbar_wait(dec + bs, bpar, abort_flag, err, 3)) break;
+        if (!mbar_wait(afull + as, apar, abort_flag, err, 7)) break;
         tc_fence_after();
-        const uint32_t a0 = smem_u32(sA + s * A_BYTES);
-        const uint32_t b0 = smem_u32(sB + s * B_BYTES);
+        const uint32_t b0 = smem_u32(sB + bs * B_BYTES);
+        for (int j = 0; j < qts; ++j) {
+          const uint32_t a0 = smem_u32(sA + (as * QT + j) * A_BYTES);
+          const uint32_t dt = tmem + (uint32_t)((set * QT + j) * MMA_N);
 #pragma unroll
-        for (int kk = 0; kk < KB / 16; ++kk)
-          mma_f16(tmem + buf * MMA_N, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), (kb | kk) != 0);
-        mma_commit(empty + s);
-        if (kb == kblocks - 1) mma_commit(acc_full + buf);
+          for (int kk = 0; kk < KB / 16; ++kk)
+            mma_f16(dt, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), (kb | kk) != 0);
+        }
+        mma_commit(bempty + bs);
+        mma_commit(aempty + as);
+        if (kb == kblocks - 1) mma_commit(acc_full + set);
+        if (++bs == BST) {
+          bs = 0;
+          bpar ^= 1;
+        }
+        if (++as == ast) {
+          as = 0;
+          apar ^= 1;
+        }
+        if (++kb == kblocks) {
+          kb = 0;
+          ++tile_i;
+          if (++set == NSETS) {
+            set = 0;
+            spar ^= 1;
+          }
+        }
       }
       mma_commit(fin);
       mbar_wait_drain(fin, 0);
     }
-  } else if (warp < 4) {
+  } else if (warp < DEC_WARPS) {
     // ---------------------------------------------------------- decoders
     constexpr int PARTS = RAWB / 16;                 // 16-byte parts per row per K-block
     constexpr int CODES = 16 * 8 / BITS;             // codes per part
     constexpr int CHUNKS = CODES / 8;                // 16-byte fp16 chunks per part
+    uint32_t tl[4] = {0, 0, 0, 0}, th[4] = {0, 0, 0, 0};
+    if (BITS == 4) {
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        const __half h = __float2half_rn(centroids[e]);
+        const uint32_t bitsv = (uint32_t)__half_as_ushort(h);
+        tl[e >> 2] |= (bitsv & 0xFFu) << (8 * (e & 3));
+        th[e >> 2] |= (bitsv >> 8) << (8 * (e & 3));
+      }
+    }
+    int sb = 0, cs = 0, cpar = 0, bs = 0, bpar = 0;  // sub-block, code stage + parity, B stage + parity
     for (int it = 0; it < total_it; ++it) {
-      const int s = it % STAGES;
-      if (!mbar_wait(full + s, (it / STAGES) & 1, abort_flag, err, 4)) break;
-      const unsigned char* raw = sRaw + s * MMA_N * RAWB;
-      unsigned char* bdst = sB + s * B_BYTES;
-      for (int item = tid; item < MMA_N * PARTS; item += 128) {
+      if (!warp_wait(cfull + cs, cpar, abort_flag, err, 4)) break;
+      if (it >= BST && !warp_wait(bempty + bs, bpar ^ 1, abort_flag, err, 8)) break;
+      const unsigned char* raw = sRaw + cs * MMA_N * rr;
+      unsigned char* bdst = sB + bs * B_BYTES;
+      for (int item = tid; item < MMA_N * PARTS; item += DEC_THREADS) {
         const int r = item / PARTS, p = item % PARTS;
-        const uint4 w4 = *reinterpret_cast<const uint4*>(raw + r * RAWB + p * 16);
+        const int chunk = sb * PARTS + p;  // 16-byte chunk of the row in this code tile
+        const uint4 w4 = *reinterpret_cast<const uint4*>(
+            raw + r * rrow + ((swz ? (chunk ^ (r & 7)) : chunk) << 4));
         const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
 #pragma unroll
         for (int c = 0; c < CHUNKS; ++c) {
-          uint32_t o[4];
+          uint4 out;
           if (BITS == 4) {          // chunk c: bytes 4c..4c+3, 8 codes
-            const uint32_t* tab = reinterpret_cast<const uint32_t*>(base + L.tab);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) o[j] = tab[(((w[c] >> (8 * j)) & 0xFFu) << 5) | lane];
+            out = decode8_4bit(w[c], tl, th);
           } else if (BITS == 2) {   // chunk c: bytes 2c, 2c+1, 8 codes
             const uint32_t* tab = reinterpret_cast<const uint32_t*>(base + L.tab);
             const uint32_t x = w[c >> 1] >> (16 * (c & 1));
+            uint32_t o[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) o[j] = tab[(((x >> (4 * j)) & 0xFu) << 5) | lane];
+            out = make_uint4(o[0], o[1], o[2], o[3]);
           } else {                  // chunk c: bytes 8c..8c+7, 8 codes
             const unsigned short* tab = reinterpret_cast<const unsigned short*>(base + L.tab);
+            uint32_t o[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
               const uint32_t x = w[2 * c + (j >> 1)] >> (16 * (j & 1));
               o[j] = (uint32_t)tab[((x & 0xFFu) << 5) | lane] | ((uint32_t)tab[(((x >> 8) & 0xFFu) << 5) | lane] << 16);
             }
+            out = make_uint4(o[0], o[1], o[2], o[3]);
           }
-          *reinterpret_cast<uint4*>(bdst + sw128_offset(r, p * CHUNKS + c)) = make_uint4(o[0], o[1], o[2], o[3]);
+          *reinterpret_cast<uint4*>(bdst + sw128_offset(r, p * CHUNKS + c)) = out;
         }
       }
-      fence_proxy_async();
-      mbar_arrive(dec + s);
+      fence_proxy_async();  // make this thread's writes visible to the tensor core
+      __syncwarp();
+      if (lane == 0) {
+        if (sb == sub - 1) mbar_arrive(cempty + cs);  // the whole code tile is decoded
+        mbar_arrive(dec + bs);
+      }
+      if (++sb == sub) {
+        sb = 0;
+        if (++cs == cst) {
+          cs = 0;
+          cpar ^= 1;
+        }
+      }
+      if (++bs == BST) {
+        bs = 0;
+        bpar ^= 1;
+      }
     }
   } else {
     // ---------------------------------------------------------- epilogue
-    const int e = warp - 4;                 // TMEM lanes 32e .. 32e+31
-    const int row = tid - 128;              // query row within the tile
-    const int q = qt * MMA_M + row;
-    for (int i = 0; i < k; ++i) {
+    const int e = warp - EPI_WARP0;         // TMEM lanes 32e .. 32e+31 (warp % 4 == e)
+    const int row = tid - EPI_WARP0 * 32;   // query row within each tile
+    for (int i = 0; i < QT * k; ++i) {
       lst_s[i * MMA_M + row] = -INFINITY;
       lst_i[i * MMA_M + row] = INT_MAX;
     }
-    float th_s = -INFINITY;
-    int th_i = INT_MAX;
+    float th_s[QT];
+    int th_i[QT];
+#pragma unroll
+    for (int j = 0; j < QT; ++j) {
+      th_s[j] = -INFINITY;
+      th_i[j] = INT_MAX;
+    }
     for (int tile_i = 0; tile_i < my_tiles; ++tile_i) {
       const int t = blockIdx.x + tile_i * gridDim.x;
       const int v0 = t * MMA_N;
-      const int buf = tile_i & 1;
+      const int set = tile_i % NSETS;
       // scales of this tile's vectors (the previous tile's readers are done:
       // they passed the named barrier below)
       for (int j = row; j < MMA_N; j += 128) {
@@ -391,7 +548,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       }
       asm volatile("bar.sync 1, 128;" ::: "memory");
       // all four epilogue warps take the same decision, so none is left at bar.sync
-      const int ok = mbar_wait(acc_full + buf, (tile_i >> 1) & 1, abort_flag, err, 5) ? 1 : 0;
+      const int ok = warp_wait(acc_full + set, (tile_i / NSETS) & 1, abort_flag, err, 5) ? 1 : 0;
       int all_ok;
       asm volatile(
           "{\n .reg .pred p, q;\n setp.ne.s32 p, %1, 0;\n bar.red.and.pred q, 1, 128, p;\n"
@@ -401,45 +558,67 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
           : "memory");
       if (!all_ok) break;
       tc_fence_after();
-      for (int c0 = 0; c0 < MMA_N; c0 += 32) {
-        uint32_t r[32];
-        tmem_ld32(tmem + ((uint32_t)(32 * e) << 16) + buf * MMA_N + c0, r);
-        if (q < nq) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
-            const int v = v0 + c0 + j;
-            const float sc = __uint_as_float(r[j]) * sScale[c0 + j];
-            if (v < n && better(sc, v, th_s, th_i)) {
-              int pos = k - 1;
-              while (pos > 0 && better(sc, v, lst_s[(pos - 1) * MMA_M + row], lst_i[(pos - 1) * MMA_M + row])) {
-                lst_s[pos * MMA_M + row] = lst_s[(pos - 1) * MMA_M + row];
-                lst_i[pos * MMA_M + row] = lst_i[(pos - 1) * MMA_M + row];
-                --pos;
-              }
-              lst_s[pos * MMA_M + row] = sc;
-              lst_i[pos * MMA_M + row] = v;
-              th_s = lst_s[(k - 1) * MMA_M + row];
-              th_i = lst_i[(k - 1) * MMA_M + row];
+      for (int j = 0; j < QT; ++j) {
+        const int q = (qt0 + j) * MMA_M + row;
+        if (j >= qts) break;
+        float* ls = lst_s + j * k * MMA_M;
+        int* li = lst_i + j * k * MMA_M;
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld32(tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + j) * MMA_N + c0), r);
+          if (q >= nq) continue;
+          // branch-free pass: scale and flag scores that may enter the list
+          const int valid = min(32, n - (v0 + c0));
+          uint32_t m = 0;
+#pragma unroll
+          for (int jj = 0; jj < 32; ++jj) {
+            const float sc = __uint_as_float(r[jj]) * sScale[c0 + jj];
+            r[jj] = __float_as_uint(sc);
+            m |= (sc >= th_s[j] ? 1u : 0u) << jj;
+          }
+          if (valid < 32) m &= valid > 0 ? (1u << valid) - 1u : 0u;
+          if (m == 0u) continue;
+#pragma unroll
+          for (int jj = 0; jj < 32; ++jj) scr[jj * MMA_M + row] = __uint_as_float(r[jj]);
+          while (m) {  // rare after the first tiles
+            const int jj = __ffs(m) - 1;
+            m &= m - 1;
+            const float sc = scr[jj * MMA_M + row];
+            const int v = v0 + c0 + jj;
+            if (!better(sc, v, th_s[j], th_i[j])) continue;
+            int pos = k - 1;
+            while (pos > 0 && better(sc, v, ls[(pos - 1) * MMA_M + row], li[(pos - 1) * MMA_M + row])) {
+              ls[pos * MMA_M + row] = ls[(pos - 1) * MMA_M + row];
+              li[pos * MMA_M + row] = li[(pos - 1) * MMA_M + row];
+              --pos;
             }
+            ls[pos * MMA_M + row] = sc;
+            li[pos * MMA_M + row] = v;
+            th_s[j] = ls[(k - 1) * MMA_M + row];
+            th_i[j] = li[(k - 1) * MMA_M + row];
           }
         }
       }
       tc_fence_before();
-      mbar_arrive(acc_empty + buf);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty + set);
       asm volatile("bar.sync 1, 128;" ::: "memory");
     }
-    if (q < nq) {
+    for (int j = 0; j < qts; ++j) {
+      const int q = (qt0 + j) * MMA_M + row;
+      if (q >= nq) continue;
       for (int i = 0; i < k; ++i) {
         const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
-        cand_s[o] = lst_s[i * MMA_M + row];
-        cand_i[o] = lst_i[i * MMA_M + row];
+        cand_s[o] = lst_s[(j * k + i) * MMA_M + row];
+        cand_i[o] = lst_i[(j * k + i) * MMA_M + row];
       }
     }
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 8) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
+  if (warp == CODE_WARP) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
 }
 
 // Rotated queries (float32 [nq, d]) -> fp16 A blocks [qtile][kblock][128 x 64],
@@ -478,28 +657,37 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
   return fn;
 }
 
-template <int BITS>
-cudaError_t launch_typed(const CUtensorMap& map, const __half* qpack, const float* centroids,
-                         const float* scale, int n, int nq, int d, int k, int grid_x, float* cs, int* ci,
-                         int* err, cudaStream_t s) {
-  const MmaSmem L = mma_smem_layout<BITS>(k);
-  cudaError_t e = cudaFuncSetAttribute(k_scan_mma<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)L.total);
+template <int BITS, int QT>
+cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half* qpack, const float* centroids,
+                         const float* scale, int n, int nq, int d, int k, int sub, int grid_x, float* cs,
+                         int* ci, int* err, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(k_scan_mma<BITS, QT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)P.smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)grid_x, (unsigned)((nq + MMA_M - 1) / MMA_M));
-  k_scan_mma<BITS><<<grid, NTHREADS, L.total, s>>>(map, qpack, centroids, scale, n, nq, d, k, cs, ci, err);
+  const int nqt = (nq + MMA_M - 1) / MMA_M;
+  const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));
+  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, n, nq, d, k, P.cst, P.ast,
+                                                         P.rr, sub, cs, ci, err);
   return cudaGetLastError();
+}
+
+MmaPlan plan_for(int bits, int64_t nq, int k) {
+  return bits == 2 ? mma_plan<2>(nq, k) : bits == 4 ? mma_plan<4>(nq, k) : mma_plan<8>(nq, k);
 }
 
 }  // namespace
 
 bool mma_supported(int bits, int d, int k) {
-  return (bits == 2 || bits == 4 || bits == 8) && d % KB == 0 && k <= kMaxKMma;
+  return (bits == 2 || bits == 4 || bits == 8) && d % KB == 0 && k >= 1 && k <= kMaxKMma &&
+         plan_for(bits, 1, k).smem != 0;
 }
 
-int scan_mma_grid_x(int64_t nq, int64_t n) {
+int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits) {
   const int64_t qtiles = (nq + MMA_M - 1) / MMA_M;
+  const int qt = plan_for(bits, nq, k).qt;
+  const int64_t groups = (qtiles + qt - 1) / qt;
   const int64_t ntiles = (n + MMA_N - 1) / MMA_N;
-  int64_t gx = ((int64_t)device_sm_count() + qtiles - 1) / qtiles;
+  int64_t gx = ((int64_t)device_sm_count() + groups - 1) / groups;
   if (gx > ntiles) gx = ntiles;
   if (gx < 1) gx = 1;
   return (int)gx;
@@ -517,13 +705,20 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
   if (!enc) return cudaErrorNotSupported;
   const int rawb = KB * bits / 8;
+  const MmaPlan P = plan_for(bits, nq, k);
+  if (P.smem == 0) return cudaErrorInvalidValue;
+  // K-blocks per code tile: up to P.rr bytes of each row, dividing the row's K-blocks
+  const int kblocks = d / KB;
+  int sub = P.rr / rawb;
+  while (sub > 1 && kblocks % sub != 0) sub >>= 1;
   CUtensorMap map;
   const cuuint64_t gdim[2] = {(cuuint64_t)row_bytes(d, bits), (cuuint64_t)n};
   const cuuint64_t gstride[1] = {(cuuint64_t)row_bytes(d, bits)};
-  const cuuint32_t box[2] = {(cuuint32_t)rawb, (cuuint32_t)MMA_N};
+  const cuuint32_t box[2] = {(cuuint32_t)(sub * rawb), (cuuint32_t)MMA_N};
   const cuuint32_t estride[2] = {1, 1};
   CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(codes), gdim, gstride, box,
-                   estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                   estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   sub * rawb == RAW_ROW_MAX ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   const dim3 pgrid((unsigned)(d / KB), (unsigned)((nq + MMA_M - 1) / MMA_M));
@@ -532,12 +727,20 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   if (e != cudaSuccess) return e;
   if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;
   const __half* qp = static_cast<const __half*>(qpack);
+#define TQ_MMA_CASE(B)                                                                                        \
+  case B:                                                                                                     \
+    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, (int)n, (int)nq, d, k, sub, grid_x,      \
+                                       cand_s, cand_i, err, s)                                                \
+                  : launch_typed<B, 1>(P, map, qp, centroids, scale, (int)n, (int)nq, d, k, sub, grid_x,      \
+                                       cand_s, cand_i, err, s);                                               \
+    break;
   switch (bits) {
-    case 2: e = launch_typed<2>(map, qp, centroids, scale, (int)n, (int)nq, d, k, grid_x, cand_s, cand_i, err, s); break;
-    case 4: e = launch_typed<4>(map, qp, centroids, scale, (int)n, (int)nq, d, k, grid_x, cand_s, cand_i, err, s); break;
-    case 8: e = launch_typed<8>(map, qp, centroids, scale, (int)n, (int)nq, d, k, grid_x, cand_s, cand_i, err, s); break;
+    TQ_MMA_CASE(2)
+    TQ_MMA_CASE(4)
+    TQ_MMA_CASE(8)
     default: return cudaErrorInvalidValue;
   }
+#undef TQ_MMA_CASE
   if (e != cudaSuccess) return e;
   if (ev1 && (e = cudaEventRecord(ev1, s)) != cudaSuccess) return e;
   return cudaSuccess;

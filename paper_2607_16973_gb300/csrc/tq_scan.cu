@@ -95,7 +95,14 @@ __device__ __forceinline__ void warp_insert(float* ws, int* wi, int k, int cnt, 
   __syncwarp();
 }
 
-// 16 codes of `BITS` bits starting at a chunk boundary.
+// Shifts x so that the bit at position p lands at bit 7 (p is a compile-time
+// constant after unrolling).
+__device__ __forceinline__ uint32_t to_bit7(uint32_t x, int p) { return p >= 7 ? x >> (p - 7) : x << (7 - p); }
+
+// 16 codes of `BITS` bits starting at a chunk boundary.  off(t, lane4) is the
+// byte offset of code t's entry for this lane in the bank-replicated centroid
+// table (entry (c, lane) at (c * 32 + lane) * 4): one shift and one
+// three-input logic op per code.
 template <int BITS>
 struct Chunk;
 
@@ -108,7 +115,9 @@ struct Chunk<4> {
     w1 = v.y;
   }
   __device__ __forceinline__ void zero() { w0 = w1 = 0; }
-  __device__ __forceinline__ uint32_t code(int t) const { return ((t < 8 ? w0 : w1) >> (4 * (t & 7))) & 15u; }
+  __device__ __forceinline__ uint32_t off(int t, uint32_t lane4) const {
+    return (to_bit7(t < 8 ? w0 : w1, 4 * (t & 7)) & 0x780u) | lane4;
+  }
 };
 
 template <>
@@ -116,7 +125,7 @@ struct Chunk<2> {
   uint32_t w;
   __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const unsigned int*>(p)); }
   __device__ __forceinline__ void zero() { w = 0; }
-  __device__ __forceinline__ uint32_t code(int t) const { return (w >> (2 * t)) & 3u; }
+  __device__ __forceinline__ uint32_t off(int t, uint32_t lane4) const { return (to_bit7(w, 2 * t) & 0x180u) | lane4; }
 };
 
 template <>
@@ -124,9 +133,9 @@ struct Chunk<8> {
   uint4 w;
   __device__ __forceinline__ void load(const uint8_t* p) { w = __ldcs(reinterpret_cast<const uint4*>(p)); }
   __device__ __forceinline__ void zero() { w = make_uint4(0, 0, 0, 0); }
-  __device__ __forceinline__ uint32_t code(int t) const {
+  __device__ __forceinline__ uint32_t off(int t, uint32_t lane4) const {
     const uint32_t x = t < 4 ? w.x : t < 8 ? w.y : t < 12 ? w.z : w.w;
-    return (x >> (8 * (t & 3))) & 255u;
+    return (to_bit7(x, 8 * (t & 3)) & 0x7F80u) | lane4;
   }
 };
 
@@ -138,7 +147,11 @@ struct Chunk<3> {
     v = (uint64_t)__ldcs(h) | ((uint64_t)__ldcs(h + 1) << 16) | ((uint64_t)__ldcs(h + 2) << 32);
   }
   __device__ __forceinline__ void zero() { v = 0; }
-  __device__ __forceinline__ uint32_t code(int t) const { return (uint32_t)(v >> (3 * t)) & 7u; }
+  __device__ __forceinline__ uint32_t off(int t, uint32_t lane4) const {
+    const int p = 3 * t;
+    const uint32_t x = (uint32_t)(p >= 7 ? v >> (p - 7) : v << (7 - p));
+    return (x & 0x380u) | lane4;
+  }
 };
 
 // Sums p[0..7] across the warp: afterwards lanes 4i..4i+3 hold the total of
@@ -209,6 +222,7 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
   int th_i = INT_MAX;
   const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
   const int my = (lane >> 2) & 7;  // the vector whose total this lane ends up holding
+  const uint32_t lane4 = (uint32_t)lane * 4u;
   for (int st = blockIdx.x; st < nsteps; st += gridDim.x) {
     const int v0 = st * (SCAN_WARPS * V) + warp * V;
     if (v0 >= n) continue;
@@ -236,14 +250,18 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
         else ch[i][s].zero();
       }
     }
+    // keep every load above in flight before the first lookup below
+    asm volatile("" ::: "memory");
     float p[V];
+    const char* tab = reinterpret_cast<const char*>(ctab);
 #pragma unroll
     for (int i = 0; i < V; ++i) {
       float acc = 0.f;
 #pragma unroll
       for (int s = 0; s < S; ++s)
 #pragma unroll
-        for (int t = 0; t < 16; ++t) acc = fmaf(qr[s][t], ctab[(ch[i][s].code(t) << 5) | lane], acc);
+        for (int t = 0; t < 16; ++t)
+          acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + ch[i][s].off(t, lane4)), acc);
       p[i] = acc;
     }
     const float total = warp_sum8(p);
@@ -279,8 +297,144 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
   }
 }
 
+// Sums p[0..3] across the warp: afterwards lanes 8i..8i+7 hold the total of
+// p[i] (2 + 1 + 1 + 1 + 1 shuffles for 4 values).
+__device__ __forceinline__ float warp_sum4(float (&p)[4]) {
+  const int lane = threadIdx.x & 31;
+  const bool h16 = lane & 16, h8 = lane & 8;
+  float a[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    const float send = h16 ? p[i] : p[i + 2];
+    const float keep = h16 ? p[i + 2] : p[i];
+    a[i] = keep + __shfl_xor_sync(FULL, send, 16);
+  }
+  float c = (h8 ? a[1] : a[0]) + __shfl_xor_sync(FULL, h8 ? a[0] : a[1], 8);
+  c += __shfl_xor_sync(FULL, c, 4);
+  c += __shfl_xor_sync(FULL, c, 2);
+  c += __shfl_xor_sync(FULL, c, 1);
+  return c;
+}
+
+// Unfiltered lookup scan with a register double buffer: each warp scores 4
+// consecutive vectors per step and issues the next step's code loads before
+// it starts on the current ones, so every warp always has loads in flight.
+template <int BITS, int S>
+__global__ void __launch_bounds__(SCAN_NT, 2)
+k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
+                  const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n, int k, int P,
+                  float* __restrict__ cand_s, int* __restrict__ cand_i) {
+  constexpr int L = 1 << BITS;
+  constexpr int CB = 2 * BITS;
+  constexpr int V = 4;  // vectors per warp step; a CTA step covers 32
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float* ctab = reinterpret_cast<float*>(smem_raw);  // [L][32], entry (c, lane) in bank lane
+  float* ls = ctab + L * 32;                          // [P] scores; warp w's list at [w*k, w*k+k)
+  int* li = reinterpret_cast<int*>(ls + P);           // [P] ids
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int q = blockIdx.y;
+  for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  for (int i = tid; i < P; i += SCAN_NT) {
+    ls[i] = -INFINITY;
+    li[i] = INT_MAX;
+  }
+  const int nchunks = d >> 4;
+  const float* qq = qrot + (size_t)q * d;
+  float qr[S][16];
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    const int chunk = lane + 32 * s;
+#pragma unroll
+    for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+  }
+  __syncthreads();
+
+  const int64_t row_bytes = (int64_t)d * BITS / 8;
+  float* wl_s = ls + warp * k;
+  int* wl_i = li + warp * k;
+  int cnt = 0;
+  float th_s = -INFINITY;
+  int th_i = INT_MAX;
+  const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
+  const int my = (lane >> 3) & 3;  // the vector whose total this lane ends up holding
+  const uint32_t lane4 = (uint32_t)lane * 4u;
+  const char* tab = reinterpret_cast<const char*>(ctab);
+
+  Chunk<BITS> cur[V][S], nxt[V][S];
+  float sc_cur = 0.f, sc_nxt = 0.f;
+  auto load_step = [&](int st, Chunk<BITS> (&buf)[V][S], float& sc) {
+    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      const uint8_t* row = codes + (size_t)(v0 + i) * row_bytes;
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        const int chunk = lane + 32 * s;
+        if (st < nsteps && v0 + i < n && chunk < nchunks) buf[i][s].load(row + chunk * CB);
+        else buf[i][s].zero();
+      }
+    }
+    const int vm = v0 + my;
+    sc = 0.f;
+    if (st < nsteps && (lane & 7) == 0 && vm < n) sc = scale ? __ldg(scale + vm) : 1.0f;
+  };
+  int st = blockIdx.x;
+  load_step(st, cur, sc_cur);
+  for (; st < nsteps; st += gridDim.x) {
+    load_step(st + gridDim.x, nxt, sc_nxt);   // next step's loads go out first
+    asm volatile("" ::: "memory");
+    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+    float p[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      float acc = 0.f;
+#pragma unroll
+      for (int s = 0; s < S; ++s)
+#pragma unroll
+        for (int t = 0; t < 16; ++t)
+          acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + cur[i][s].off(t, lane4)), acc);
+      p[i] = acc;
+    }
+    const float total = warp_sum4(p);
+    const int vm = v0 + my;
+    float score = -INFINITY;
+    bool cand = false;
+    if ((lane & 7) == 0 && vm < n) {
+      score = total * sc_cur;
+      cand = better(score, vm, th_s, th_i);
+    }
+    unsigned m = __ballot_sync(FULL, cand);
+    while (m) {  // in vector order; re-checked against the moving threshold
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      const float sv = __shfl_sync(FULL, score, src);
+      const int vv = v0 + ((src >> 3) & 3);
+      if (better(sv, vv, th_s, th_i)) {
+        warp_insert(wl_s, wl_i, k, cnt, sv, vv);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = wl_s[k - 1];
+          th_i = wl_i[k - 1];
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < V; ++i)
+#pragma unroll
+      for (int s = 0; s < S; ++s) cur[i][s] = nxt[i][s];
+    sc_cur = sc_nxt;
+  }
+  __syncthreads();
+  block_sort(ls, li, P);
+  for (int i = tid; i < k; i += SCAN_NT) {
+    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
+    cand_s[o] = ls[i];
+    cand_i[o] = li[i];
+  }
+}
+
 // Merges per_query candidates of each query into its sorted top-k.
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(1024)
 k_merge(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int per_query, int k,
         int P, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -355,7 +509,14 @@ cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* 
                            const float* centroids, const uint8_t* codes, const float* scale, int n,
                            const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
                            const uint32_t* allow, int k, int P, float* cs, int* ci) {
-  cudaError_t e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e;
+  if (!allow) {
+    e = cudaFuncSetAttribute(k_scan_lut_stream<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
+    return cudaGetLastError();
+  }
+  e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_scan_lut<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
                                                   words, fblock, allow, k, P, cs, ci);
@@ -382,7 +543,8 @@ int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d) {
   (void)k;
   (void)bits;
   (void)d;
-  const int64_t target = (int64_t)device_sm_count() * 4;
+  // one resident wave (two CTAs per SM) for a single query
+  const int64_t target = (int64_t)device_sm_count() * 2;
   int64_t gx = (target + nq - 1) / (nq > 0 ? nq : 1);
   const int64_t blocks = (n + 31) / 32;
   if (gx > blocks) gx = blocks;
@@ -422,7 +584,7 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
   if (nq == 0) return cudaSuccess;
   const int P = std::min(MERGE_P, next_pow2(std::max(per_query + k, 64)));
   const size_t smem = (size_t)P * (sizeof(float) + sizeof(int));
-  k_merge<<<(unsigned)nq, 256, smem, s>>>(cand_s, cand_i, per_query, k, P, out_ids, out_scores);
+  k_merge<<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, per_query, k, P, out_ids, out_scores);
   return cudaGetLastError();
 }
 

@@ -275,7 +275,8 @@ def test_invalid_calls_on_gpu(cuda_lib, torch_dev):
 # ------------------------------------------------------- tensor-core scan --
 @pytest.mark.parametrize("bits,d,n,nq,k", [(4, 1536, 3000, 130, 10), (2, 1536, 1000, 17, 5),
                                            (8, 1536, 777, 64, 8), (4, 64, 513, 200, 1),
-                                           (4, 2048, 2049, 129, 64), (4, 128, 255, 1, 3)])
+                                           (4, 2048, 2049, 129, 64), (4, 128, 255, 1, 3),
+                                           (8, 1536, 777, 300, 8), (4, 1536, 1500, 257, 5)])
 def test_search_mma_parity(cuda_lib, torch_dev, bits, d, n, nq, k):
     """Query tiles of 128 with a ragged last tile, vector tiles of 256 with a
     ragged tail (rows past n are filled with zeros by the tensor map), one
