@@ -15,9 +15,15 @@ step streams it from HBM.  The headline `value` is queries/s at the first batch
 size; every batch size measured is reported under "batches".
 
 --impl reference times the CPU oracle (float64 numpy) on the host cores on a
-bounded sample of the same workload.  Under torchrun every rank runs an
-independent replica (the search path needs no collective), the timed region is
-bracketed by barriers and the slowest rank's time is used.
+bounded sample of the same workload.
+
+Under torchrun (N > 1 ranks, one GPU each) the corpus is N x 999,000 rows, one
+999,000-row shard per rank (rows [r N0, (r+1) N0) of the same seeded
+generator), and the queries of rank 0 are broadcast once.  A step is then the
+sharded search: tq_search on the rank's shard, an all-gather of every rank's
+top-k (the exchange step), and tq_merge_topk.  Work per GPU is fixed (weak
+scaling); `value` counts query x shard scans per second, summed over ranks.
+The timed region is bracketed by barriers and the slowest rank's time is used.
 """
 from __future__ import annotations
 
@@ -187,13 +193,16 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------- workloads --
-def make_corpus(cfg, workers):
+def make_corpus(cfg, workers, shard=0):
+    """Rows [shard n, (shard+1) n) of the seeded mixture corpus and the query
+    pool drawn from them (shard 0 is the single-GPU workload)."""
     from paper_2607_16973_gb300 import synth
     t0 = time.time()
-    X = synth.mixture_corpus(cfg["n"], cfg["d"], cfg["clusters"], workers=workers)
-    src = synth.query_sources(cfg["n"], cfg["pool"])
+    n = cfg["n"]
+    X = synth.mixture_rows(shard * n, (shard + 1) * n, cfg["d"], cfg["clusters"], workers=workers)
+    src = synth.query_sources(n, cfg["pool"])
     Q = synth.perturb(X[src])
-    log(f"[bench] generated corpus {X.shape} + {len(Q)} queries in {time.time() - t0:.1f}s")
+    log(f"[bench] generated corpus shard {shard} {X.shape} + {len(Q)} queries in {time.time() - t0:.1f}s")
     return X, Q
 
 
@@ -280,7 +289,7 @@ def run_reference(args, cfg, rank, world):
 def run_ours(args, cfg, rank, world):
     import torch
     import paper_2607_16973_gb300 as tq
-    from paper_2607_16973_gb300 import synth
+    from paper_2607_16973_gb300 import shard, synth
     from paper_2607_16973_gb300.build import build
 
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -302,7 +311,12 @@ def run_ours(args, cfg, rank, world):
         torch.cuda.synchronize(dev)
 
     # ---- index build: codebook + rotation on the host, encode on the GPU
-    X, Qpool = make_corpus(cfg, workers=min(16, os.cpu_count() or 4))
+    X, Qpool = make_corpus(cfg, workers=min(16, os.cpu_count() or 4), shard=rank)
+    if world > 1:  # every rank searches rank 0's queries
+        qb = torch.from_numpy(Qpool).to(dev)
+        dist.broadcast(qb, src=0)
+        Qpool = qb.cpu().numpy()
+        del qb
     cen, bnd, _ = tq.codebook(d, bits)
     R = tq.rotation(d, synth.SEED_ROTATION)
     with torch.cuda.stream(stream):
@@ -341,11 +355,22 @@ def run_ours(args, cfg, rank, world):
         ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
         ids = torch.empty((B, k), dtype=torch.int64, device=dev)
         scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+        gids = torch.empty((B, k), dtype=torch.int64, device=dev)
+        gscs = torch.empty((B, k), dtype=torch.float32, device=dev)
+
+        def exchange():
+            # the sharded search's exchange step: all-gather of every rank's
+            # top-k (global ids) and the exact merge, queued on `stream`
+            with torch.cuda.stream(stream):
+                ci, cs = shard.gather_topk(ids, scs, rank * n)
+                tq.merge_topk(ci, cs, k, out_ids=gids, out_scores=gscs, stream=stream)
 
         def step(i):
             j = (i % nbatches) * B
             tq.search(Qd[j:j + B], Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids,
                       out_scores=scs, stream=stream)
+            if world > 1:
+                exchange()
 
         for i in range(args.warmup):
             step(i)
@@ -399,15 +424,25 @@ def run_ours(args, cfg, rank, world):
         ih = torch.empty((B, k), dtype=torch.int64).pin_memory()
         sh = torch.empty((B, k), dtype=torch.float32).pin_memory()
         with torch.cuda.stream(stream):
+            def e2e_step():
+                if world == 1:
+                    tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
+                                        out_ids=ids, out_scores=scs, stream=stream)
+                else:
+                    qdev.copy_(qh, non_blocking=True)
+                    tq.search(qdev, Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids,
+                              out_scores=scs, stream=stream)
+                    exchange()
+                    ih.copy_(gids, non_blocking=True)
+                    sh.copy_(gscs, non_blocking=True)
+
             for _ in range(max(1, args.warmup)):
-                tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
-                                    out_ids=ids, out_scores=scs, stream=stream)
+                e2e_step()
             barrier()
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(stream)
             for _ in range(args.steps):
-                tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
-                                    out_ids=ids, out_scores=scs, stream=stream)
+                e2e_step()
             b.record(stream)
             b.synchronize()
         e2e_ms = a.elapsed_time(b)
@@ -431,9 +466,10 @@ def run_ours(args, cfg, rank, world):
                                f"codes {n * d * bits // 8 / 1e6:.1f} MB resident in HBM",
                    "n": n, "d": d, "bits": bits, "k": k, "batch": head,
                    "l2": "inputs larger than L2 (corpus streamed from HBM every step)",
-                   "parallelism": f"replicas x{world}"},
+                   "parallelism": "single GPU" if world == 1 else
+                   f"corpus sharded by rows over {world} GPUs ({n} rows each), all-gather of top-k + merge"},
         "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (3 if world == 1 else 4) * args.steps,  # rotate, scan, merge (+ shard merge)
         "batches": {str(b): {"value": v["value"], "ms_per_step": v["ms_per_step"],
                              "roofline": v["roofline"], "e2e": v["e2e"]} for b, v in results.items()},
         "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,

@@ -214,6 +214,29 @@ tq_status tq_search_static(const float* Q, int64_t nq, int d, const float* R,
                            const int64_t* allow_off, const uint32_t* allow_tenants,
                            int k, int64_t* out_ids, float* out_scores, void* stream);
 
+/*
+ * tq_merge_topk - exact merge of per-shard top-k lists.  When the corpus is
+ * split by contiguous row ranges (one shard per device, each searched with
+ * tq_search), the k best of the whole corpus are the k best, by the same
+ * (score descending, id ascending) order tq_search uses (Sec. III-B top-k),
+ * of the union of every shard's k best with ids shifted to global rows.
+ *   cand_ids     device [n_src*nq*m] int64 global ids, laid out [n_src][nq][m]
+ *                (what an all-gather of every shard's [nq][m] result gives):
+ *                candidate j of source s for query q is at (s*nq + q)*m + j;
+ *                -1 marks an empty slot, which never displaces a real candidate
+ *   cand_scores  device [n_src*nq*m] float32, same layout
+ *   n_src        sources (1..4096)
+ *   nq           queries (>= 0; 0 is a no-op)
+ *   m            candidates per source and query (0..2^20)
+ *   k            1..256
+ *   out_ids      device out [nq*k] int64, -1 where fewer than k real candidates
+ *   out_scores   device out [nq*k] float32, -INFINITY where out_ids is -1
+ * Candidates are read-only; a (score, id) pair given twice is kept twice.
+ */
+tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_scores,
+                        int64_t n_src, int64_t nq, int64_t m, int k,
+                        int64_t* out_ids, float* out_scores, void* stream);
+
 /* Selects the search kernels for later tq_search calls of the calling thread
  * (TQ_PATH_*).  AUTO is the default. */
 tq_status tq_set_search_path(int path);

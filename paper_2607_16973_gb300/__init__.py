@@ -14,7 +14,7 @@ import numpy as np
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
 __all__ = ["codebook", "rotation", "encode", "Filter", "search", "search_workspace",
-           "search_from_host", "set_search_path", "profile_events", "row_bytes", "load",
+           "search_from_host", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
            "TQError"]
 
 
@@ -158,6 +158,27 @@ def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, q_de
     ids_host.copy_(ids, non_blocking=True)
     scores_host.copy_(scores, non_blocking=True)
     return ids_host, scores_host
+
+
+def merge_topk(cand_ids, cand_scores, k: int, out_ids=None, out_scores=None, stream=None):
+    """tq_merge_topk on CUDA tensors laid out [n_src, nq, m] (or [nq, m] for a
+    single source): returns (ids int64 [nq, k], scores f32 [nq, k])."""
+    torch = _torch()
+    if cand_ids.dim() == 2:
+        cand_ids, cand_scores = cand_ids.unsqueeze(0), cand_scores.unsqueeze(0)
+    if cand_ids.shape != cand_scores.shape or cand_ids.dim() != 3:
+        raise ValueError("cand_ids and cand_scores must both be [n_src, nq, m]")
+    n_src, nq, m = cand_ids.shape
+    dev = cand_ids.device
+    if out_ids is None:
+        out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    if out_scores is None:
+        out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    check(load().tq_merge_topk(
+        _dev_ptr(cand_ids, "cand_ids", torch.int64), _dev_ptr(cand_scores, "cand_scores", torch.float32),
+        n_src, nq, m, k, _dev_ptr(out_ids, "out_ids", torch.int64),
+        _dev_ptr(out_scores, "out_scores", torch.float32), _stream_handle(stream)))
+    return out_ids, out_scores
 
 
 def set_search_path(path: str) -> None:

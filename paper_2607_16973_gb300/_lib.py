@@ -34,6 +34,8 @@ SIGNATURES = {
     "tq_search_static": (C.c_int, [C.c_void_p, C.c_int64, C.c_int, C.c_void_p, C.c_void_p, C.c_int,
                                    C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p, C.c_void_p,
                                    C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "tq_merge_topk": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int64, C.c_int64, C.c_int, C.c_void_p,
+                                C.c_void_p, C.c_void_p]),
     "tq_set_search_path": (C.c_int, [C.c_int]),
     "tq_profile_events": (C.c_int, [C.c_void_p, C.c_void_p]),
 }

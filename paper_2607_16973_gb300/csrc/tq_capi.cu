@@ -228,3 +228,21 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
   if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
   return tq::ok();
 }
+
+extern "C" tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_scores, int64_t n_src, int64_t nq,
+                                   int64_t m, int k, int64_t* out_ids, float* out_scores, void* stream) {
+  if (nq < 0 || nq > (1 << 24)) return fail(TQ_EINVAL, "tq_merge_topk: nq=%lld outside [0, 2^24]", (long long)nq);
+  if (n_src < 1 || n_src > 4096) return fail(TQ_EINVAL, "tq_merge_topk: n_src=%lld outside [1, 4096]", (long long)n_src);
+  if (m < 0 || m > (1 << 20)) return fail(TQ_EINVAL, "tq_merge_topk: m=%lld outside [0, 2^20]", (long long)m);
+  if (k < 1 || k > tq::kMaxK) return fail(TQ_EINVAL, "tq_merge_topk: k=%d outside [1, %d]", k, tq::kMaxK);
+  if (nq == 0) return tq::ok();
+  if (!out_ids || !out_scores || (m > 0 && (!cand_ids || !cand_scores)))
+    return fail(TQ_EINVAL, "tq_merge_topk: NULL device pointer");
+  if (((uintptr_t)cand_ids & 7u) || ((uintptr_t)out_ids & 7u) || ((uintptr_t)cand_scores & 3u) ||
+      ((uintptr_t)out_scores & 3u))
+    return fail(TQ_EINVAL, "tq_merge_topk: misaligned pointers");
+  const cudaError_t e =
+      tq::launch_merge_global(cand_scores, cand_ids, n_src, nq, m, k, out_ids, out_scores, (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_merge_topk", e);
+  return tq::ok();
+}

@@ -46,6 +46,11 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
 cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
                          int k, int64_t* out_ids, float* out_scores, cudaStream_t s);
 
+// Merge of S sources x m candidates per query ([S][nq][m]) with global int64
+// ids (-1 = padding).
+cudaError_t launch_merge_global(const float* cand_s, const int64_t* cand_i, int64_t S, int64_t nq, int64_t m,
+                                int k, int64_t* out_ids, float* out_scores, cudaStream_t s);
+
 // Tensor-core decode-GEMM scan (bits 2, 4, 8; k <= kMaxKMma; unfiltered).
 bool mma_supported(int bits, int d, int k);
 int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits);

@@ -18,6 +18,7 @@
 #include <cuda_runtime.h>
 
 #include <climits>
+#include <limits>
 #include <cmath>
 #include <cstdint>
 
@@ -32,20 +33,22 @@ constexpr int SCAN_NT = 256;
 constexpr int SCAN_WARPS = SCAN_NT / 32;
 constexpr int MERGE_P = 2048;
 
-__device__ __forceinline__ bool better(float s1, int i1, float s2, int i2) {
+template <typename I>
+__device__ __forceinline__ bool better(float s1, I i1, float s2, I i2) {
   return s1 > s2 || (s1 == s2 && i1 < i2);
 }
 
 // Bitonic sort of P (a power of two) (score, id) pairs in shared memory, best
 // first.  All threads of the block take part.
-__device__ void block_sort(float* s, int* id, int P) {
+template <typename I>
+__device__ void block_sort(float* s, I* id, int P) {
   for (int size = 2; size <= P; size <<= 1) {
     for (int stride = size >> 1; stride > 0; stride >>= 1) {
       for (int t = threadIdx.x; t < P / 2; t += blockDim.x) {
         const int i = 2 * t - (t & (stride - 1));
         const int j = i + stride;
         const float si = s[i], sj = s[j];
-        const int ii = id[i], ij = id[j];
+        const I ii = id[i], ij = id[j];
         const bool best_first = (i & size) == 0;
         const bool swap = best_first ? better(sj, ij, si, ii) : better(si, ii, sj, ij);
         if (swap) {
@@ -434,33 +437,48 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
 }
 
 // Merges per_query candidates of each query into its sorted top-k.
+// Merges the candidates of each query into its sorted top-k, P - k at a time.
+// Candidates come from S sources laid out [S][nq][m]: candidate j of source
+// src for query q is cand_*[(src * nq + q) * m + j].  Candidates whose id is
+// `pad` never beat a real one and come out as (-1, -INFINITY).
+template <typename I>
 __global__ void __launch_bounds__(1024)
-k_merge(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int per_query, int k,
-        int P, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t S, int64_t nq, int64_t m, int k,
+        int P, I pad, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* s = reinterpret_cast<float*>(smem_raw);
-  int* id = reinterpret_cast<int*>(s + P);
-  const int q = blockIdx.x;
-  const float* cs = cand_s + (size_t)q * per_query;
-  const int* ci = cand_i + (size_t)q * per_query;
+  I* id = reinterpret_cast<I*>(smem_raw);
+  float* s = reinterpret_cast<float*>(id + P);
+  const int64_t q = blockIdx.x;
+  const int64_t total = S * m;
+  constexpr I kWorst = std::numeric_limits<I>::max();
   for (int i = threadIdx.x; i < k; i += blockDim.x) {
     s[i] = -INFINITY;
-    id[i] = INT_MAX;
+    id[i] = kWorst;
   }
   const int chunk = P - k;
-  for (int c0 = 0; c0 < per_query; c0 += chunk) {
+  for (int64_t c0 = 0; c0 < total; c0 += chunk) {
     for (int i = threadIdx.x; i < chunk; i += blockDim.x) {
-      const int j = c0 + i;
-      s[k + i] = j < per_query ? cs[j] : -INFINITY;
-      id[k + i] = j < per_query ? ci[j] : INT_MAX;
+      const int64_t c = c0 + i;
+      float sv = -INFINITY;
+      I v = kWorst;
+      if (c < total) {
+        const int64_t src = c / m, j = c - src * m;
+        const int64_t o = (src * nq + q) * m + j;
+        if (cand_i[o] != pad) {
+          v = cand_i[o];
+          sv = cand_s[o];
+        }
+      }
+      s[k + i] = sv;
+      id[k + i] = v;
     }
     __syncthreads();
     block_sort(s, id, P);
   }
   for (int i = threadIdx.x; i < k; i += blockDim.x) {
-    const bool pad = id[i] == INT_MAX;
-    out_ids[(size_t)q * k + i] = pad ? -1 : (int64_t)id[i];
-    out_scores[(size_t)q * k + i] = pad ? -INFINITY : s[i];
+    const bool empty = id[i] == kWorst;
+    out_ids[q * k + i] = empty ? -1 : (int64_t)id[i];
+    out_scores[q * k + i] = empty ? -INFINITY : s[i];
   }
 }
 
@@ -583,8 +601,21 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
                          int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   const int P = std::min(MERGE_P, next_pow2(std::max(per_query + k, 64)));
-  const size_t smem = (size_t)P * (sizeof(float) + sizeof(int));
-  k_merge<<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, per_query, k, P, out_ids, out_scores);
+  const size_t smem = (size_t)P * (sizeof(float) + sizeof(int32_t));
+  k_merge<int32_t><<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, 1, nq, per_query, k, P, INT_MAX, out_ids,
+                                                     out_scores);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_global(const float* cand_s, const int64_t* cand_i, int64_t S, int64_t nq, int64_t m,
+                                int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  const int64_t total = S * m;
+  int P = next_pow2((int)std::min<int64_t>(total + k, MERGE_P));
+  P = std::max(P, next_pow2(std::max(2 * k, 64)));  // at least k new candidates per pass
+  const size_t smem = (size_t)P * (sizeof(float) + sizeof(int64_t));
+  k_merge<int64_t><<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, S, nq, m, k, P, (int64_t)-1, out_ids,
+                                                     out_scores);
   return cudaGetLastError();
 }
 

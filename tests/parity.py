@@ -90,3 +90,21 @@ def check_topk(gpu_ids, gpu_scores, oracle_ids, scores64, allowed, k, tol):
 
 def recall(ids, exact_ids):
     return O.recall_at_k(np.asarray(ids), np.asarray(exact_ids))
+
+
+def merge_candidates(cand_ids, cand_scores, k):
+    """Top-k of the union of candidate lists [S, nq, m] by (score desc, id asc),
+    padding (id -1) dropped, result padded with (-1, -inf): the ranking rule of
+    the search, applied to the gathered lists."""
+    S, nq, m = cand_ids.shape
+    ids = np.full((nq, k), -1, np.int64)
+    sc = np.full((nq, k), -np.inf, np.float32)
+    for q in range(nq):
+        i = cand_ids[:, q, :].reshape(-1)
+        s = cand_scores[:, q, :].reshape(-1)
+        keep = i >= 0
+        i, s = i[keep], s[keep]
+        order = np.lexsort((i, -s.astype(np.float64)))[:k]
+        ids[q, :len(order)] = i[order]
+        sc[q, :len(order)] = s[order]
+    return ids, sc

@@ -126,6 +126,14 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert lib.tq_filter_build(p, 10, 48, C.byref(h), null) == _lib.TQ_EINVAL
     assert lib.tq_filter_build(p, 0, 64, C.byref(h), null) == _lib.TQ_EINVAL
     assert lib.tq_filter_destroy(null) == _lib.TQ_OK
+    # merge: sources, candidates per source, k, NULL and misaligned pointers
+    assert lib.tq_merge_topk(p, p, 0, 4, 10, 5, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(p, p, 2, 4, -1, 5, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(p, p, 2, 4, 10, 0, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(p, p, 2, 4, 10, 257, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(null, p, 2, 4, 10, 5, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(p + 4, p, 2, 4, 10, 5, p, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_merge_topk(null, null, 2, 0, 10, 5, null, null, null) == _lib.TQ_OK
     assert lib.tq_set_search_path(7) == _lib.TQ_EINVAL
     assert lib.tq_profile_events(p, null) == _lib.TQ_EINVAL
 
