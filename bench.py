@@ -409,14 +409,18 @@ def run_ours(args, cfg, rank, world):
                     "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": scan_ms,
                     "hbm_gbs_of_corpus": alg_bytes / (scan_ms / 1e3) / 1e9}
         else:
-            # lookup scan: the corpus (codes + scales) read once per launch
+            # lookup scan: the corpus (codes + scales) read once per launch; 4-bit
+            # codes take the byte-pair kernel, other widths the per-code one
+            kname = "k_scan_pair_stream" if bits == 4 else "k_scan_lut_stream"
             achieved = alg_bytes / (scan_ms / 1e3) / 1e9
             roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                     "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
-                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu", "scan_lut_prof.md",
-                                                scale_to=n),
-                    "kernel": "k_scan_lut", "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
-                    "frac_of_8tbs_nominal": achieved / 8000.0}
+                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu",
+                                                "k_scan_pair_stream_250k_batch1.md", scale_to=n)
+                    if bits == 4 else None,
+                    "kernel": kname, "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
+                    "frac_of_8tbs_nominal": achieved / 8000.0,
+                    "smem_lookup_ceiling_gbs": 4950.0 if bits == 4 else None}
         # e2e through the public API with host buffers
         qh = torch.empty((B, d), dtype=torch.float32).pin_memory()
         qh.copy_(torch.from_numpy(Qpool[:B]))

@@ -259,15 +259,28 @@ k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, f
 #pragma unroll
   for (int q = 0; q < NQ; ++q) acc[q] = 0.f;
   const float4* r4 = reinterpret_cast<const float4*>(R + (int64_t)i * d);
-  for (int j = lane; j < d / 4; j += 32) {
-    const float4 rv = __ldg(r4 + j);
+  const int d4 = d / 4;
+  // R (d*d*4 bytes) is usually evicted from L2 by the corpus stream between
+  // searches, so issue 8 row loads per lane before using any of them
+  for (int j0 = lane; j0 < d4; j0 += 32 * 8) {
+    float4 rv[8];
 #pragma unroll
-    for (int q = 0; q < NQ; ++q) {
-      const float4 qv = __ldg(reinterpret_cast<const float4*>(Q + (int64_t)q * d) + j);
-      acc[q] = fmaf(rv.x, qv.x, acc[q]);
-      acc[q] = fmaf(rv.y, qv.y, acc[q]);
-      acc[q] = fmaf(rv.z, qv.z, acc[q]);
-      acc[q] = fmaf(rv.w, qv.w, acc[q]);
+    for (int t = 0; t < 8; ++t) {
+      const int j = j0 + 32 * t;
+      rv[t] = j < d4 ? __ldg(r4 + j) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+#pragma unroll
+    for (int t = 0; t < 8; ++t) {
+      const int j = j0 + 32 * t;
+      if (j >= d4) break;
+#pragma unroll
+      for (int q = 0; q < NQ; ++q) {
+        const float4 qv = __ldg(reinterpret_cast<const float4*>(Q + (int64_t)q * d) + j);
+        acc[q] = fmaf(rv[t].x, qv.x, acc[q]);
+        acc[q] = fmaf(rv[t].y, qv.y, acc[q]);
+        acc[q] = fmaf(rv[t].z, qv.z, acc[q]);
+        acc[q] = fmaf(rv[t].w, qv.w, acc[q]);
+      }
     }
   }
 #pragma unroll

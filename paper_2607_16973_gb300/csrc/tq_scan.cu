@@ -157,6 +157,54 @@ struct Chunk<3> {
   }
 };
 
+// Byte-pair lookups for 4-bit codes.  A packed byte x holds two codes, so one
+// 8-byte load of T[x] = (c[x & 15], c[x >> 4]) fetches both centroids and one
+// paired FMA adds q'_{2m} c[x & 15] and q'_{2m+1} c[x >> 4] into a float2
+// accumulator: per two codes one byte permute (the byte moved to bits 8..15
+// next to lane * 8, which is the entry's address), one shared load and one
+// FMA instruction.  T is replicated per lane, entry (x, lane) at
+// (x * 32 + lane) * 8 bytes, so a warp's 32 loads hit 32 different 8-byte
+// bank pairs in two wavefronts whatever the bytes are.
+constexpr int PAIR_TAB_BYTES = 256 * 32 * 8;
+
+__device__ __forceinline__ void pair_table_init(float2* ptab, const float* __restrict__ centroids, int tid, int nt) {
+  for (int i = tid; i < 256 * 32; i += nt) {
+    const int x = i >> 5;
+    ptab[i] = make_float2(__ldg(centroids + (x & 15)), __ldg(centroids + (x >> 4)));
+  }
+}
+
+// This lane's part of one vector's score: its S chunks of 16 codes against
+// the matching (q'_{2m}, q'_{2m+1}) pairs.  Both 4-bit scans use exactly this
+// order of operations, so filtered and unfiltered scores agree bit for bit.
+template <int S>
+__device__ __forceinline__ float pair_dot(const Chunk<4> (&ch)[S], const float2 (&q2)[S][8], const char* tab,
+                                          uint32_t lane8) {
+  float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+#pragma unroll
+    for (int b = 0; b < 8; ++b) {
+      const uint32_t w = b < 4 ? ch[s].w0 : ch[s].w1;
+      const uint32_t addr = __byte_perm(w, lane8, 0x5504u | ((uint32_t)(b & 3) << 4));
+      acc = __ffma2_rn(q2[s][b], *reinterpret_cast<const float2*>(tab + addr), acc);
+    }
+  }
+  return acc.x + acc.y;
+}
+
+template <int S>
+__device__ __forceinline__ void load_q2(float2 (&q2)[S][8], const float* qq, int nchunks, int lane) {
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+    const int chunk = lane + 32 * s;
+#pragma unroll
+    for (int m = 0; m < 8; ++m)
+      q2[s][m] = chunk < nchunks ? make_float2(qq[chunk * 16 + 2 * m], qq[chunk * 16 + 2 * m + 1])
+                                 : make_float2(0.f, 0.f);
+  }
+}
+
 // Sums p[0..7] across the warp: afterwards lanes 4i..4i+3 hold the total of
 // p[i] (a transposed butterfly: 4 + 2 + 1 + 1 + 1 shuffles for 8 values).
 __device__ __forceinline__ float warp_sum8(float (&p)[8]) {
@@ -194,25 +242,35 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
   constexpr int L = 1 << BITS;
   constexpr int CB = 2 * BITS;
   constexpr int V = 8;  // vectors per warp step; a CTA step covers 64
+  // 4-bit codes use the byte-pair table (pair_dot), other widths the
+  // per-code table [L][32] with entry (c, lane) in bank lane
+  constexpr int TAB_BYTES = BITS == 4 ? PAIR_TAB_BYTES : L * 32 * 4;
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* ctab = reinterpret_cast<float*>(smem_raw);  // [L][32], entry (c, lane) in bank lane
-  float* ls = ctab + L * 32;                          // [P] scores; warp w's list at [w*k, w*k+k)
-  int* li = reinterpret_cast<int*>(ls + P);           // [P] ids
+  float* ctab = reinterpret_cast<float*>(smem_raw);
+  float* ls = reinterpret_cast<float*>(smem_raw + TAB_BYTES);  // [P] scores; warp w's list at [w*k, w*k+k)
+  int* li = reinterpret_cast<int*>(ls + P);                     // [P] ids
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int q = blockIdx.y;
-  for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  if constexpr (BITS == 4) pair_table_init(reinterpret_cast<float2*>(smem_raw), centroids, tid, SCAN_NT);
+  else
+    for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
   for (int i = tid; i < P; i += SCAN_NT) {
     ls[i] = -INFINITY;
     li[i] = INT_MAX;
   }
   const int nchunks = d >> 4;
   const float* qq = qrot + (size_t)q * d;
-  float qr[S][16];
+  float qr[BITS == 4 ? 1 : S][16];
+  float2 q2[BITS == 4 ? S : 1][8];
+  if constexpr (BITS == 4) {
+    load_q2(q2, qq, nchunks, lane);
+  } else {
 #pragma unroll
-  for (int s = 0; s < S; ++s) {
-    const int chunk = lane + 32 * s;
+    for (int s = 0; s < S; ++s) {
+      const int chunk = lane + 32 * s;
 #pragma unroll
-    for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+      for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+    }
   }
   __syncthreads();
 
@@ -259,13 +317,17 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
     const char* tab = reinterpret_cast<const char*>(ctab);
 #pragma unroll
     for (int i = 0; i < V; ++i) {
-      float acc = 0.f;
+      if constexpr (BITS == 4) {
+        p[i] = pair_dot<S>(ch[i], q2, tab, lane4 * 2u);
+      } else {
+        float acc = 0.f;
 #pragma unroll
-      for (int s = 0; s < S; ++s)
+        for (int s = 0; s < S; ++s)
 #pragma unroll
-        for (int t = 0; t < 16; ++t)
-          acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + ch[i][s].off(t, lane4)), acc);
-      p[i] = acc;
+          for (int t = 0; t < 16; ++t)
+            acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + ch[i][s].off(t, lane4)), acc);
+        p[i] = acc;
+      }
     }
     const float total = warp_sum8(p);
     float score = -INFINITY;
@@ -436,7 +498,106 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
   }
 }
 
-// Merges per_query candidates of each query into its sorted top-k.
+// Unfiltered 4-bit scan with byte-pair lookups (pair_dot); otherwise as
+// k_scan_lut_stream: 4 vectors per warp step, next step's loads in flight.
+template <int S>
+__global__ void __launch_bounds__(SCAN_NT, 2)
+k_scan_pair_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
+                   const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n, int k, int P,
+                   float* __restrict__ cand_s, int* __restrict__ cand_i) {
+  constexpr int V = 4;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  float2* ptab = reinterpret_cast<float2*>(smem_raw);  // [256][32]
+  float* ls = reinterpret_cast<float*>(smem_raw + PAIR_TAB_BYTES);
+  int* li = reinterpret_cast<int*>(ls + P);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int q = blockIdx.y;
+  pair_table_init(ptab, centroids, tid, SCAN_NT);
+  for (int i = tid; i < P; i += SCAN_NT) {
+    ls[i] = -INFINITY;
+    li[i] = INT_MAX;
+  }
+  const int nchunks = d >> 4;
+  float2 q2[S][8];  // (q'_{2m}, q'_{2m+1}) of the 16 coordinates of chunk lane + 32 s
+  load_q2(q2, qrot + (size_t)q * d, nchunks, lane);
+  __syncthreads();
+
+  const int64_t row_bytes = (int64_t)d / 2;
+  float* wl_s = ls + warp * k;
+  int* wl_i = li + warp * k;
+  int cnt = 0;
+  float th_s = -INFINITY;
+  int th_i = INT_MAX;
+  const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
+  const int my = (lane >> 3) & 3;
+  const uint32_t lane8 = (uint32_t)lane * 8u;
+  const char* tab = reinterpret_cast<const char*>(ptab);
+
+  Chunk<4> cur[V][S], nxt[V][S];
+  float sc_cur = 0.f, sc_nxt = 0.f;
+  auto load_step = [&](int st, Chunk<4> (&buf)[V][S], float& sc) {
+    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+#pragma unroll
+    for (int i = 0; i < V; ++i) {
+      const uint8_t* row = codes + (size_t)(v0 + i) * row_bytes;
+#pragma unroll
+      for (int s = 0; s < S; ++s) {
+        const int chunk = lane + 32 * s;
+        if (st < nsteps && v0 + i < n && chunk < nchunks) buf[i][s].load(row + chunk * 8);
+        else buf[i][s].zero();
+      }
+    }
+    const int vm = v0 + my;
+    sc = 0.f;
+    if (st < nsteps && (lane & 7) == 0 && vm < n) sc = scale ? __ldg(scale + vm) : 1.0f;
+  };
+  int st = blockIdx.x;
+  load_step(st, cur, sc_cur);
+  for (; st < nsteps; st += gridDim.x) {
+    load_step(st + gridDim.x, nxt, sc_nxt);
+    asm volatile("" ::: "memory");
+    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+    float p[V];
+#pragma unroll
+    for (int i = 0; i < V; ++i) p[i] = pair_dot<S>(cur[i], q2, tab, lane8);
+    const float total = warp_sum4(p);
+    const int vm = v0 + my;
+    float score = -INFINITY;
+    bool cand = false;
+    if ((lane & 7) == 0 && vm < n) {
+      score = total * sc_cur;
+      cand = better(score, vm, th_s, th_i);
+    }
+    unsigned m = __ballot_sync(FULL, cand);
+    while (m) {
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      const float sv = __shfl_sync(FULL, score, src);
+      const int vv = v0 + ((src >> 3) & 3);
+      if (better(sv, vv, th_s, th_i)) {
+        warp_insert(wl_s, wl_i, k, cnt, sv, vv);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = wl_s[k - 1];
+          th_i = wl_i[k - 1];
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < V; ++i)
+#pragma unroll
+      for (int s = 0; s < S; ++s) cur[i][s] = nxt[i][s];
+    sc_cur = sc_nxt;
+  }
+  __syncthreads();
+  block_sort(ls, li, P);
+  for (int i = tid; i < k; i += SCAN_NT) {
+    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
+    cand_s[o] = ls[i];
+    cand_i[o] = li[i];
+  }
+}
+
 // Merges the candidates of each query into its sorted top-k, P - k at a time.
 // Candidates come from S sources laid out [S][nq][m]: candidate j of source
 // src for query q is cand_*[(src * nq + q) * m + j].  Candidates whose id is
@@ -477,6 +638,117 @@ k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t 
   }
   for (int i = threadIdx.x; i < k; i += blockDim.x) {
     const bool empty = id[i] == kWorst;
+    out_ids[q * k + i] = empty ? -1 : (int64_t)id[i];
+    out_scores[q * k + i] = empty ? -INFINITY : s[i];
+  }
+}
+
+// Merge of per-CTA candidate lists that are each sorted best first and hold
+// exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
+// any one list is beaten or matched by that list's k entries, so the global
+// k-th best is at least as good as the best such T, and only candidates at
+// least as good as it can be in the global top-k.  Those survivors (at least
+// k of them, usually few more) are compacted; each then finds its rank by
+// counting the survivors ahead of it (equal pairs, which only padding can
+// form, are ordered by slot) and the first k ranks are written out.  If more
+// survive than the P slots hold, the block sorts everything in chunks.
+__global__ void __launch_bounds__(1024)
+k_merge_sorted_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k, int P,
+                     int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  int* id = reinterpret_cast<int*>(smem_raw);
+  float* s = reinterpret_cast<float*>(id + P);
+  __shared__ float red_s[32];
+  __shared__ int red_i[32];
+  __shared__ int count;
+  const int64_t q = blockIdx.x;
+  const int total = nlists * k;
+  const float* cs = cand_s + q * total;
+  const int* ci = cand_i + q * total;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  // 1. T = best k-th entry over the lists
+  float ts = -INFINITY;
+  int ti = INT_MAX;
+  for (int l = tid; l < nlists; l += blockDim.x) {
+    const float a = cs[l * k + k - 1];
+    const int b = ci[l * k + k - 1];
+    if (better(a, b, ts, ti)) {
+      ts = a;
+      ti = b;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float a = __shfl_xor_sync(FULL, ts, o);
+    const int b = __shfl_xor_sync(FULL, ti, o);
+    if (better(a, b, ts, ti)) {
+      ts = a;
+      ti = b;
+    }
+  }
+  if (lane == 0) {
+    red_s[warp] = ts;
+    red_i[warp] = ti;
+  }
+  if (tid == 0) count = 0;
+  __syncthreads();
+  ts = red_s[0];
+  ti = red_i[0];
+  for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+    if (better(red_s[w], red_i[w], ts, ti)) {
+      ts = red_s[w];
+      ti = red_i[w];
+    }
+  // 2. compact the candidates at least as good as T
+  for (int c = tid; c < total; c += blockDim.x) {
+    const float a = cs[c];
+    const int b = ci[c];
+    if (!better(ts, ti, a, b)) {
+      const int pos = atomicAdd(&count, 1);
+      if (pos < P) {
+        s[pos] = a;
+        id[pos] = b;
+      }
+    }
+  }
+  __syncthreads();
+  const int m = count;
+  if (m > P) {  // 3a. too many survivors (e.g. mostly padding): sort everything in chunks
+    for (int i = tid; i < k; i += blockDim.x) {
+      s[i] = -INFINITY;
+      id[i] = INT_MAX;
+    }
+    const int chunk = P - k;
+    for (int c0 = 0; c0 < total; c0 += chunk) {
+      __syncthreads();
+      for (int i = tid; i < chunk; i += blockDim.x) {
+        const int c = c0 + i;
+        s[k + i] = c < total ? cs[c] : -INFINITY;
+        id[k + i] = c < total ? ci[c] : INT_MAX;
+      }
+      __syncthreads();
+      block_sort(s, id, P);
+    }
+  } else {  // 3b. rank the survivors
+    for (int i = tid; i < m; i += blockDim.x) {
+      const float a = s[i];
+      const int b = id[i];
+      int r = 0;
+      for (int j = 0; j < m; ++j) {
+        const float sj = s[j];
+        const int ij = id[j];
+        r += better(sj, ij, a, b) || (sj == a && ij == b && j < i);
+      }
+      if (r < k) {
+        const bool empty = b == INT_MAX;
+        out_ids[q * k + r] = empty ? -1 : (int64_t)b;
+        out_scores[q * k + r] = empty ? -INFINITY : a;
+      }
+    }
+    return;
+  }
+  for (int i = tid; i < k; i += blockDim.x) {
+    const bool empty = id[i] == INT_MAX;
     out_ids[q * k + i] = empty ? -1 : (int64_t)id[i];
     out_scores[q * k + i] = empty ? -INFINITY : s[i];
   }
@@ -528,16 +800,24 @@ cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* 
                            const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
                            const uint32_t* allow, int k, int P, float* cs, int* ci) {
   cudaError_t e;
+  if (BITS == 4 && !allow) {
+    const size_t psmem = (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int));
+    e = cudaFuncSetAttribute(k_scan_pair_stream<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+    if (e != cudaSuccess) return e;
+    k_scan_pair_stream<S><<<grid, SCAN_NT, psmem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
+    return cudaGetLastError();
+  }
   if (!allow) {
     e = cudaFuncSetAttribute(k_scan_lut_stream<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
     return cudaGetLastError();
   }
-  e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const size_t fsmem = BITS == 4 ? (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int)) : smem;
+  e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
   if (e != cudaSuccess) return e;
-  k_scan_lut<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
-                                                  words, fblock, allow, k, P, cs, ci);
+  k_scan_lut<BITS, S><<<grid, SCAN_NT, fsmem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
+                                                   words, fblock, allow, k, P, cs, ci);
   return cudaGetLastError();
 }
 
@@ -600,10 +880,10 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
 cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
                          int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
+  // per_query = grid_x * k: one sorted list of k per scan CTA
   const int P = std::min(MERGE_P, next_pow2(std::max(per_query + k, 64)));
   const size_t smem = (size_t)P * (sizeof(float) + sizeof(int32_t));
-  k_merge<int32_t><<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, 1, nq, per_query, k, P, INT_MAX, out_ids,
-                                                     out_scores);
+  k_merge_sorted_lists<<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, per_query / k, k, P, out_ids, out_scores);
   return cudaGetLastError();
 }
 
