@@ -237,6 +237,30 @@ tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_scores,
                         int64_t n_src, int64_t nq, int64_t m, int k,
                         int64_t* out_ids, float* out_scores, void* stream);
 
+/*
+ * tq_search_check - waits for `stream` and reports how the last tq_search that
+ * used `workspace` ended on the GPU.  tq_search validates its arguments and
+ * queues its kernels; the tensor-core scan's waits on its pipelines are
+ * bounded (about 2 s of SM clock), and a wait that gives up stops the kernel
+ * and records where in the workspace's status word instead of hanging.
+ *   workspace  the device workspace passed to tq_search (16-byte aligned)
+ * Returns TQ_OK, TQ_ETIMEOUT (the results of that search are invalid; the
+ * context and the library stay usable) or TQ_ECUDA.  Every tq_search clears
+ * the word before its kernels run.
+ */
+tq_status tq_search_check(const void* workspace, void* stream);
+
+/* Testing hooks.  They exercise the failure paths without faulting the GPU.
+ * tq_debug_fail_allocs(count): the calling thread's next `count` library-owned
+ * device allocations (tq_filter_build) fail as out of memory (TQ_ENOMEM).
+ * tq_debug_bounded_wait(budget_cycles, workspace, stream): queues one CTA that
+ * waits, with the scans' bounded wait and a budget of budget_cycles SM cycles
+ * (1 .. 4e9), on an mbarrier nothing completes; the wait gives up and records
+ * its timeout in the workspace's status word, which tq_search_check reports. */
+tq_status tq_debug_fail_allocs(int count);
+tq_status tq_debug_bounded_wait(long long budget_cycles, void* workspace,
+                                void* stream);
+
 /* Selects the search kernels for later tq_search calls of the calling thread
  * (TQ_PATH_*).  AUTO is the default. */
 tq_status tq_set_search_path(int path);

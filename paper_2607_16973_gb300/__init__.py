@@ -14,7 +14,7 @@ import numpy as np
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
 __all__ = ["codebook", "rotation", "encode", "Filter", "search", "search_workspace",
-           "search_from_host", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
+           "search_from_host", "search_check", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
            "TQError"]
 
 
@@ -179,6 +179,12 @@ def merge_topk(cand_ids, cand_scores, k: int, out_ids=None, out_scores=None, str
         n_src, nq, m, k, _dev_ptr(out_ids, "out_ids", torch.int64),
         _dev_ptr(out_scores, "out_scores", torch.float32), _stream_handle(stream)))
     return out_ids, out_scores
+
+
+def search_check(workspace, stream=None) -> None:
+    """tq_search_check: waits for the stream; raises TQError (TQ_ETIMEOUT) if
+    the last search that used `workspace` gave up on a bounded wait."""
+    check(load().tq_search_check(_dev_ptr(workspace, "workspace"), _stream_handle(stream)))
 
 
 def set_search_path(path: str) -> None:

@@ -36,6 +36,9 @@ SIGNATURES = {
                                    C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]),
     "tq_merge_topk": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_int64, C.c_int64, C.c_int, C.c_void_p,
                                 C.c_void_p, C.c_void_p]),
+    "tq_search_check": (C.c_int, [C.c_void_p, C.c_void_p]),
+    "tq_debug_fail_allocs": (C.c_int, [C.c_int]),
+    "tq_debug_bounded_wait": (C.c_int, [C.c_longlong, C.c_void_p, C.c_void_p]),
     "tq_set_search_path": (C.c_int, [C.c_int]),
     "tq_profile_events": (C.c_int, [C.c_void_p, C.c_void_p]),
 }

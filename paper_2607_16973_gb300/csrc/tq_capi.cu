@@ -108,9 +108,10 @@ extern "C" tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int 
     f.n_tenants = (int64_t)ids.size();
     f.words = (int)((f.n_tenants + 31) / 32);
     const int64_t nblocks = (n + block - 1) / block;
-    e = cudaMalloc(&f.tenants, ids.size() * sizeof(uint32_t));
-    if (e == cudaSuccess) e = cudaMalloc(&f.dense, (size_t)n * sizeof(uint32_t));
-    if (e == cudaSuccess) e = cudaMalloc(&f.block_bits, (size_t)nblocks * f.words * sizeof(uint32_t));
+    e = tq::dev_malloc(reinterpret_cast<void**>(&f.tenants), ids.size() * sizeof(uint32_t));
+    if (e == cudaSuccess) e = tq::dev_malloc(reinterpret_cast<void**>(&f.dense), (size_t)n * sizeof(uint32_t));
+    if (e == cudaSuccess)
+      e = tq::dev_malloc(reinterpret_cast<void**>(&f.block_bits), (size_t)nblocks * f.words * sizeof(uint32_t));
     if (e != cudaSuccess) {
       tq_filter_destroy(h);
       cudaGetLastError();
@@ -210,9 +211,8 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
   uint32_t* allow = filter ? reinterpret_cast<uint32_t*>(ws + p.off_allow) : nullptr;
   float* cs = reinterpret_cast<float*>(ws + p.off_cs);
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
-  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, s);
+  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, s);  // also zeroes the status word
   if (use_mma) {
-    if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int), s);
     if (e == cudaSuccess)
       e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, k, p.grid_mma, ws + p.off_qpack, cs, ci,
                               status, s, (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
@@ -244,5 +244,31 @@ extern "C" tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_sc
   const cudaError_t e =
       tq::launch_merge_global(cand_scores, cand_ids, n_src, nq, m, k, out_ids, out_scores, (cudaStream_t)stream);
   if (e != cudaSuccess) return tq::cuda_fail("tq_merge_topk", e);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_search_check(const void* workspace, void* stream) {
+  if (!workspace) return fail(TQ_EINVAL, "tq_search_check: NULL workspace");
+  if (!tq::aligned16(workspace)) return fail(TQ_EINVAL, "tq_search_check: workspace must be 16-byte aligned");
+  cudaStream_t s = (cudaStream_t)stream;
+  int word = 0;
+  cudaError_t e = cudaMemcpyAsync(&word, workspace, sizeof(int), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_search_check", e);
+  if (word == 0) return tq::ok();
+  if (word / 1000 == TQ_ETIMEOUT)
+    return fail(TQ_ETIMEOUT, "tq_search_check: a bounded wait (site %d) gave up; the results are invalid",
+                word % 1000);
+  return fail(TQ_ECUDA, "tq_search_check: unexpected status word %d", word);
+}
+
+extern "C" tq_status tq_debug_bounded_wait(long long budget_cycles, void* workspace, void* stream) {
+  if (!workspace || !tq::aligned16(workspace))
+    return fail(TQ_EINVAL, "tq_debug_bounded_wait: NULL or misaligned workspace");
+  if (budget_cycles < 1 || budget_cycles > tq::kWaitCyclesMax)
+    return fail(TQ_EINVAL, "tq_debug_bounded_wait: budget %lld outside [1, %lld]", budget_cycles,
+                tq::kWaitCyclesMax);
+  const cudaError_t e = tq::launch_debug_wait(budget_cycles, static_cast<int*>(workspace), (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_debug_bounded_wait", e);
   return tq::ok();
 }

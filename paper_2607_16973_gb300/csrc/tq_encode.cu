@@ -230,8 +230,9 @@ k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict_
 // Q' = Q R^T, plain store epilogue (nq > 8).
 __global__ void __launch_bounds__(NT, 2)
 k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R,
-              float* __restrict__ out) {
+              float* __restrict__ out, int* __restrict__ status) {
   __shared__ GemmSmem sm;
+  if (status && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
   const int64_t row0 = (int64_t)blockIdx.x * BM;
   const int col0 = blockIdx.y * BN;
   float acc[8][8];
@@ -251,7 +252,9 @@ k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __res
 // Q' = Q R^T for nq <= 8: one warp per output coordinate, R read once.
 template <int NQ>
 __global__ void __launch_bounds__(256)
-k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, float* __restrict__ out) {
+k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, float* __restrict__ out,
+              int* __restrict__ status) {
+  if (status && blockIdx.x == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
   const int lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (i >= d) return;
@@ -317,14 +320,14 @@ cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, cons
   return cudaGetLastError();
 }
 
-cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out,
+cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out, int* status,
                           cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   if (nq <= 8) {
     const int grid = (d + 7) / 8;
     switch (nq) {
 #define TQ_GEMV_CASE(N) \
-  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, d, R, out); break;
+  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, d, R, out, status); break;
       TQ_GEMV_CASE(1) TQ_GEMV_CASE(2) TQ_GEMV_CASE(3) TQ_GEMV_CASE(4)
       TQ_GEMV_CASE(5) TQ_GEMV_CASE(6) TQ_GEMV_CASE(7) TQ_GEMV_CASE(8)
 #undef TQ_GEMV_CASE
@@ -332,7 +335,7 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
     return cudaGetLastError();
   }
   dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN));
-  k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out);
+  k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out, status);
   return cudaGetLastError();
 }
 

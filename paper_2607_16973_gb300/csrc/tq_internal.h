@@ -23,6 +23,10 @@ constexpr int kMaxK = 256;
 constexpr int kMaxKMma = 64;     // per-thread top-k lists of the tensor-core scan
 constexpr int kMmaMinBatch = 16; // AUTO uses the tensor-core scan from this batch size
 constexpr int kMaxD = 8192;
+constexpr long long kWaitCyclesMax = 4000000000LL;  // the kernels' wait budget (~2 s at 2 GHz)
+
+// Thread-local count of device allocations still to fail (tq_debug_fail_allocs).
+int& fail_allocs();
 
 inline bool valid_bits(int b) { return b == 2 || b == 3 || b == 4 || b == 8; }
 inline int64_t row_bytes(int d, int bits) { return (int64_t)d * bits / 8; }

@@ -24,7 +24,7 @@ cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, cons
                           float* scale, cudaStream_t s);
 
 // q' = R q for nq queries: out [nq * d] float32.
-cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out,
+cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out, int* status,
                           cudaStream_t s);
 
 // Per-query allow bitmaps over the dense tenant index: out [nq * words].
@@ -61,6 +61,14 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
                             cudaEvent_t ev0, cudaEvent_t ev1);
 
 int device_sm_count();
+
+// cudaMalloc that fails while the calling thread's tq_debug_fail_allocs
+// count is positive (testing hook for the out-of-memory paths).
+cudaError_t dev_malloc(void** p, size_t bytes);
+
+// One CTA that waits, with the scans' bounded wait, on an mbarrier nothing
+// completes (testing hook for the timeout path).
+cudaError_t launch_debug_wait(long long budget, int* status, cudaStream_t s);
 
 }  // namespace tq
 

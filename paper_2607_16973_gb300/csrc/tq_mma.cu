@@ -30,6 +30,7 @@
 
 #include "tq_internal.h"
 #include "tq_kernels.h"
+#include "tq_wait.cuh"
 
 namespace tq {
 namespace {
@@ -47,7 +48,7 @@ constexpr int EPI_WARP0 = 8, CODE_WARP = 12, MMA_WARP = 13, QUERY_WARP = 14;
 constexpr uint32_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
 constexpr int A_BYTES = MMA_M * KB * 2;   // 16 KB
 constexpr int B_BYTES = MMA_N * KB * 2;   // 32 KB
-constexpr long long WAIT_CYCLES = 4000000000LL;  // ~2 s at 2 GHz
+constexpr long long WAIT_CYCLES = kWaitCycles;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -79,18 +80,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // Waits for the phase with the given parity; false on timeout or abort.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                           int* err, int where) {
-  const long long t0 = clock64();
-  for (uint32_t i = 0;; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 63) == 63) {
-      if (*abort_flag) return false;
-      if (clock64() - t0 > WAIT_CYCLES) {
-        *abort_flag = 1;
-        atomicExch(err, TQ_ETIMEOUT * 1000 + where);
-        return false;
-      }
-    }
-  }
+  return bounded_wait(bar, parity, abort_flag, err, where, WAIT_CYCLES);
 }
 
 // Bounded wait that ignores `abort` (used to drain work already in flight).

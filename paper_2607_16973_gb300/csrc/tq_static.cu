@@ -110,7 +110,7 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
   uint32_t* allow_bits = f ? reinterpret_cast<uint32_t*>(base + rot) : nullptr;
   float* cand_s = reinterpret_cast<float*>(base + rot + allow);
   int32_t* cand_i = reinterpret_cast<int32_t*>(base + rot + allow + cs);
-  e = tq::launch_rotate(Q, nq, d, R, qrot, s);
+  e = tq::launch_rotate(Q, nq, d, R, qrot, nullptr, s);
   if (e == cudaSuccess && f) e = tq::launch_allow_bits(*f, allow_off, allow_tenants, nq, allow_bits, s);
   if (e == cudaSuccess)
     e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, f, allow_bits, k, gx, cand_s, cand_i, s,

@@ -134,6 +134,14 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert lib.tq_merge_topk(null, p, 2, 4, 10, 5, p, p, null) == _lib.TQ_EINVAL
     assert lib.tq_merge_topk(p + 4, p, 2, 4, 10, 5, p, p, null) == _lib.TQ_EINVAL
     assert lib.tq_merge_topk(null, null, 2, 0, 10, 5, null, null, null) == _lib.TQ_OK
+    # status check and testing hooks
+    assert lib.tq_search_check(null, null) == _lib.TQ_EINVAL
+    assert lib.tq_search_check(p + 4, null) == _lib.TQ_EINVAL
+    assert lib.tq_debug_fail_allocs(-1) == _lib.TQ_EINVAL
+    assert lib.tq_debug_fail_allocs(0) == _lib.TQ_OK
+    assert lib.tq_debug_bounded_wait(0, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_debug_bounded_wait(5_000_000_000, p, null) == _lib.TQ_EINVAL
+    assert lib.tq_debug_bounded_wait(1000, null, null) == _lib.TQ_EINVAL
     assert lib.tq_set_search_path(7) == _lib.TQ_EINVAL
     assert lib.tq_profile_events(p, null) == _lib.TQ_EINVAL
 

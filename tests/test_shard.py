@@ -99,3 +99,43 @@ def test_gloo_two_ranks_sharded_merge_equals_global(tmp_path, filtered):
     if filtered:  # query 0 allows only tenant 7: three rows, then padding
         assert sorted(ids[0, :3]) == [700, 701, 999]
         assert np.all(ids[0, 3:] == -1)
+
+
+def _rank_lost_main(rank, world, port, out_dir):
+    """Rank 1 dies before the exchange; rank 0 must learn of it from the
+    collective (process-group timeout or closed connection), not hang."""
+    import datetime
+    import torch
+    import torch.distributed as dist
+    from paper_2607_16973_gb300.shard import gather_topk
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank, world_size=world,
+                            timeout=datetime.timedelta(seconds=10))
+    if rank == 1:
+        os._exit(3)  # the shard is lost between steps, with nothing in flight
+    ids = torch.zeros((2, 5), dtype=torch.int64)
+    scores = torch.zeros((2, 5), dtype=torch.float32)
+    try:
+        gather_topk(ids, scores, 0)
+        outcome = "completed"
+    except Exception as e:  # noqa: BLE001 - any collective error is the detection
+        outcome = "detected: " + type(e).__name__
+    with open(os.path.join(out_dir, "rank0.txt"), "w") as f:
+        f.write(outcome)
+    os._exit(0)
+
+
+def test_gloo_lost_rank_is_detected(tmp_path):
+    import multiprocessing as mp
+    ctx = mp.get_context("spawn")
+    port = _free_port()
+    procs = [ctx.Process(target=_rank_lost_main, args=(r, 2, port, str(tmp_path))) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=60)
+    alive = [p for p in procs if p.is_alive()]
+    for p in alive:
+        p.kill()
+    assert not alive, "a rank hung after its peer was lost"
+    assert procs[1].exitcode == 3
+    assert (tmp_path / "rank0.txt").read_text().startswith("detected")
