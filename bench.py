@@ -52,6 +52,7 @@ CONFIGS = {
     "prof": dict(n=250_000, d=1536, bits=4, clusters=256, pool=2_048, k=5, batches=[1, 1024]),
 }
 
+RECALL_Q = 200       # queries whose Recall@k against exact kNN the bench reports
 MMA_MIN_BATCH = 16  # tq_search's AUTO switch to the tensor-core scan (bits 2/4/8, k <= 64, no filter)
 
 METRIC = "queries/sec at 999Kx1536 4-bit top-5 (batch 1 / 1024); % of HBM / TC roofline"
@@ -338,6 +339,20 @@ def run_ours(args, cfg, rank, world):
         e1.synchronize()
         enc_ms.append(e0.elapsed_time(e1))
     enc_ms = min(enc_ms[1:])
+    # ground truth for Recall@k: exact float32 inner products of the first
+    # RECALL_Q queries with the unquantised normalised corpus (torch matmul,
+    # outside the timed regions; TF32 off)
+    torch.backends.cuda.matmul.allow_tf32 = False
+    nrec = min(RECALL_Q, len(Qpool))
+    with torch.cuda.stream(stream):
+        exact = torch.empty((nrec, k), dtype=torch.int64, device=dev)
+        best = torch.full((nrec, k), float("-inf"), device=dev)
+        for r0 in range(0, n, 1 << 18):
+            sc = Qd[:nrec] @ Xd[r0:r0 + (1 << 18)].T
+            v, i = torch.topk(torch.cat([best, sc], dim=1), k, dim=1)
+            idx = torch.cat([exact, torch.arange(r0, r0 + sc.shape[1], device=dev).expand(nrec, -1)], dim=1)
+            exact, best = torch.gather(idx, 1, i), v
+    stream.synchronize()
     del Xd
     torch.cuda.empty_cache()
     log(f"[bench] encode {n} vectors: {enc_ms:.1f} ms ({n / enc_ms * 1e3:.3g} vec/s)")
@@ -404,7 +419,7 @@ def run_ours(args, cfg, rank, world):
             peak = pk["bf16_tflops_sustained"]
             roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                     "frac": achieved / peak, "frac_of": pk["source"] + " (sustained bf16 = fp16 dense rate)",
-                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_mma.cu", "scan_mma_prof.md",
+                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_mma.cu", "k_scan_mma_250k_batch1024.md",
                                                 scale_to=n),
                     "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": scan_ms,
                     "hbm_gbs_of_corpus": alg_bytes / (scan_ms / 1e3) / 1e9}
@@ -459,6 +474,23 @@ def run_ours(args, cfg, rank, world):
             f"= {achieved:.0f} GB/s ({100 * achieved / pk['hbm_gbs']:.1f}% of {pk['source']} HBM)")
         del ws
 
+    # Recall@k of both scan paths on the same queries
+    recall = {"k": k, "queries": nrec,
+              "exact": "float32 brute force over the unquantised normalised corpus"}
+    for path in ("lut", "mma"):
+        if path == "mma" and not (bits in (2, 4, 8) and k <= 64):
+            continue
+        tq.set_search_path(path)
+        try:
+            with torch.cuda.stream(stream):
+                got, _ = tq.search(Qd[:nrec], Rd, cd, bits, codes, scale, k, stream=stream)
+            stream.synchronize()
+        finally:
+            tq.set_search_path("auto")
+        hit = (got.unsqueeze(2) == exact.unsqueeze(1)).any(dim=2).float().sum(dim=1) / k
+        recall[path] = float(hit.mean())
+    log(f"[bench] Recall@{k} over {nrec} queries: {recall}")
+
     head = batches[0]
     r = results[head]
     line = {
@@ -473,6 +505,7 @@ def run_ours(args, cfg, rank, world):
                    "parallelism": "single GPU" if world == 1 else
                    f"corpus sharded by rows over {world} GPUs ({n} rows each), all-gather of top-k + merge"},
         "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
+        "recall": recall,
         "gpu_launches": (3 if world == 1 else 4) * args.steps,  # rotate, scan, merge (+ shard merge)
         "batches": {str(b): {"value": v["value"], "ms_per_step": v["ms_per_step"],
                              "roofline": v["roofline"], "e2e": v["e2e"]} for b, v in results.items()},

@@ -252,12 +252,17 @@ k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __res
 // Q' = Q R^T for nq <= 8: one warp per output coordinate, R read once.
 template <int NQ>
 __global__ void __launch_bounds__(256)
-k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, float* __restrict__ out,
+k_rotate_gemv(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R, float* __restrict__ out,
               int* __restrict__ status) {
-  if (status && blockIdx.x == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
+  if (status && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
   const int lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (i >= d) return;
+  // block row y handles queries NQ*y .. NQ*y + NQ - 1 (the last group may be short)
+  const int64_t q0 = (int64_t)blockIdx.y * NQ;
+  const int nqg = (int)min((int64_t)NQ, nq - q0);
+  Q += q0 * d;
+  out += q0 * d;
   float acc[NQ];
 #pragma unroll
   for (int q = 0; q < NQ; ++q) acc[q] = 0.f;
@@ -278,6 +283,7 @@ k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, f
       if (j >= d4) break;
 #pragma unroll
       for (int q = 0; q < NQ; ++q) {
+        if (q >= nqg) break;
         const float4 qv = __ldg(reinterpret_cast<const float4*>(Q + (int64_t)q * d) + j);
         acc[q] = fmaf(rv[t].x, qv.x, acc[q]);
         acc[q] = fmaf(rv[t].y, qv.y, acc[q]);
@@ -291,7 +297,7 @@ k_rotate_gemv(const float* __restrict__ Q, int d, const float* __restrict__ R, f
     float s = acc[q];
 #pragma unroll
     for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    if (lane == 0) out[(int64_t)q * d + i] = s;
+    if (lane == 0 && q < nqg) out[(int64_t)q * d + i] = s;
   }
 }
 
@@ -324,14 +330,19 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
                           cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   if (nq <= 8) {
-    const int grid = (d + 7) / 8;
+    const dim3 grid((unsigned)((d + 7) / 8), 1);
     switch (nq) {
 #define TQ_GEMV_CASE(N) \
-  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, d, R, out, status); break;
+  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status); break;
       TQ_GEMV_CASE(1) TQ_GEMV_CASE(2) TQ_GEMV_CASE(3) TQ_GEMV_CASE(4)
       TQ_GEMV_CASE(5) TQ_GEMV_CASE(6) TQ_GEMV_CASE(7) TQ_GEMV_CASE(8)
 #undef TQ_GEMV_CASE
     }
+    return cudaGetLastError();
+  }
+  if (nq <= 256) {  // groups of 8 queries: R stays in L2 across the groups; the GEMM would use few CTAs
+    const dim3 grid((unsigned)((d + 7) / 8), (unsigned)((nq + 7) / 8));
+    k_rotate_gemv<8><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status);
     return cudaGetLastError();
   }
   dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN));

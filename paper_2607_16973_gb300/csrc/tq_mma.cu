@@ -2,22 +2,24 @@
 //   S[q, v] = scale_v * sum_j q'_j c[code_vj]
 // with the rotated queries on the MMA's M dimension (128 per tile) and corpus
 // vectors on N (256 per MMA), fp16 operands and fp32 accumulation in tensor
-// memory (TMEM).  One CTA owns one query tile and a strided set of 256-vector
-// tiles.  Roles (warp-specialised, 10 warps):
-//   warps 0-7  decoders: expand one K-block (64 coordinates) of packed codes,
-//              brought to shared memory by TMA, into fp16 centroid values laid
-//              out as the K-major, 128-byte-swizzled B operand;
-//   warps 8-11 epilogue: read the 128 x 256 fp32 accumulator from TMEM (one
-//              query per thread), apply the per-vector scale and keep each
-//              query's top-k in a thread-private sorted list;
-//   warp 12    producer: TMA of the code tile and a 1-D bulk copy of the
-//              pre-swizzled fp16 query block, one mbarrier per stage;
-//              allocates TMEM;
-//   warp 13    MMA issuer: one thread issues tcgen05.mma (M=128, N=256, K=16)
-//              and commits completion to mbarriers.
-// TMEM holds two 256-column accumulators so the epilogue of one vector tile
-// overlaps the MMAs of the next.  Every wait is bounded: on timeout the CTA
-// raises `abort`, writes an error code to a flag in the workspace and exits.
+// memory (TMEM).  A CTA owns QT (1 or 2) query tiles and a strided set of
+// 256-vector tiles.  Roles (warp-specialised, 19 warps):
+//   warps 0-7   decoders: expand one K-block (64 coordinates) of packed codes,
+//               brought to shared memory by TMA, into fp16 centroid values
+//               laid out as the K-major, 128-byte-swizzled B operand;
+//   warps 8-15  epilogue: read the 128 x 256 fp32 accumulators from TMEM (one
+//               query per thread; warps 8-11 the first query tile, 12-15 the
+//               second), apply the per-vector scale and keep each query's
+//               top-k in a thread-private sorted list;
+//   warp 16     code producer: TMA of the code tiles; allocates TMEM;
+//   warp 17     MMA issuer: one thread issues tcgen05.mma (M=128, N=256,
+//               K=16) and commits completion to mbarriers;
+//   warp 18     query producer: 1-D bulk copies of pre-swizzled fp16 query
+//               blocks.
+// With one query tile TMEM holds two accumulator sets, so the epilogue of one
+// vector tile overlaps the MMAs of the next.  Every wait is bounded: on
+// timeout the CTA raises `abort`, writes an error code to the status word and
+// exits after draining what it has in flight.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -42,9 +44,10 @@ constexpr int MAX_CST = 8;  // raw code tiles in flight (HBM latency)
 constexpr int RAW_ROW_MAX = 128;  // bytes of each row one code tile carries (one 128-B line)
 constexpr int MAX_AST = 4;  // query blocks in flight (L2-resident)
 constexpr int BST = 2;      // decoded fp16 tiles
-constexpr int NTHREADS = 480;
 constexpr int DEC_WARPS = 8, DEC_THREADS = DEC_WARPS * 32;
-constexpr int EPI_WARP0 = 8, CODE_WARP = 12, MMA_WARP = 13, QUERY_WARP = 14;
+constexpr int EPI_WARP0 = 8, EPI_WARPS = 8, EPI_THREADS = EPI_WARPS * 32;
+constexpr int CODE_WARP = 16, MMA_WARP = 17, QUERY_WARP = 18;
+constexpr int NTHREADS = 19 * 32;
 constexpr uint32_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
 constexpr int A_BYTES = MMA_M * KB * 2;   // 16 KB
 constexpr int B_BYTES = MMA_N * KB * 2;   // 32 KB
@@ -143,6 +146,52 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
                ::"r"(smem_u32(bar)) : "memory");
 }
 
+// Issues a 32-column TMEM load without waiting; tmem_wait below must run
+// before any of r is read.
+__device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+
+// Waits for this thread's outstanding TMEM loads.  r is passed through so the
+// compiler cannot move a read of r above the wait.
+__device__ __forceinline__ void tmem_wait(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16_issue(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15])
+               :
+               : "memory");
+}
+
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
@@ -167,7 +216,7 @@ __device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
 }
 
 struct MmaSmem {
-  uint32_t a, b, raw, tab, scale, scr, lists_s, lists_i, bars, total;
+  uint32_t a, b, raw, tab, scale, lists_s, lists_i, bars, total;
 };
 
 template <int BITS>
@@ -196,8 +245,6 @@ __host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int 
   off += tab_bytes<BITS>();
   L.scale = off;
   off += MMA_N * 4;
-  L.scr = off;  // epilogue: 32 candidate scores per thread, [32][128]
-  off += 32 * MMA_M * 4;
   L.lists_s = off;
   off += (uint32_t)QT * k * MMA_M * 4;
   L.lists_i = off;
@@ -294,14 +341,14 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
   const bool swz = rrow == 128;
   constexpr int NSETS = 2 / QT;  // accumulator sets in TMEM (2 = double buffered)
   extern __shared__ unsigned char smem_dyn[];
-  unsigned char* base = reinterpret_cast<unsigned char*>(
-      (reinterpret_cast<uintptr_t>(smem_dyn) + 1023) & ~(uintptr_t)1023);
+  // pointer arithmetic on the shared array (not an integer round trip) keeps
+  // every access below a shared-memory access
+  unsigned char* base = smem_dyn + ((1024u - (smem_u32(smem_dyn) & 1023u)) & 1023u);
   const MmaSmem L = mma_smem_layout<BITS, QT>(k, cst, ast, rr);
   unsigned char* sA = base + L.a;
   unsigned char* sB = base + L.b;
   unsigned char* sRaw = base + L.raw;
   float* sScale = reinterpret_cast<float*>(base + L.scale);
-  float* scr = reinterpret_cast<float*>(base + L.scr);
   float* lst_s = reinterpret_cast<float*>(base + L.lists_s);
   int* lst_i = reinterpret_cast<int*>(base + L.lists_i);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
@@ -351,7 +398,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     }
     for (int b = 0; b < NSETS; ++b) {
       mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, 4);       // one arrival per epilogue warp
+      mbar_init(acc_empty + b, EPI_WARPS);  // one arrival per epilogue warp
     }
     mbar_init(fin, 1);
     *abort_flag = 0;
@@ -513,95 +560,129 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     }
   } else {
     // ---------------------------------------------------------- epilogue
-    const int e = warp - EPI_WARP0;         // TMEM lanes 32e .. 32e+31 (warp % 4 == e)
-    const int row = tid - EPI_WARP0 * 32;   // query row within each tile
-    for (int i = 0; i < QT * k; ++i) {
-      lst_s[i * MMA_M + row] = -INFINITY;
-      lst_i[i * MMA_M + row] = INT_MAX;
+    // Eight warps: warp 8 + g reads TMEM lanes 32 (g % 4) .. + 31 (a warp may
+    // only touch the lane quarter warp % 4) of query tile g / 4, so with two
+    // query tiles per CTA both tiles are read out at once.
+    const int g = warp - EPI_WARP0;
+    const int e = g & 3;
+    const int jsel = g >> 2;                 // this warp's query tile within the CTA
+    const int row = e * 32 + lane;           // query row within that tile
+    const int etid = g * 32 + lane;
+    const bool mine = jsel < qts;            // warps 12-15 idle with one query tile
+    const int q = (qt0 + jsel) * MMA_M + row;
+    float* ls = lst_s + jsel * k * MMA_M;
+    int* li = lst_i + jsel * k * MMA_M;
+    if (mine) {
+      for (int i = 0; i < k; ++i) {
+        ls[i * MMA_M + row] = -INFINITY;
+        li[i * MMA_M + row] = INT_MAX;
+      }
     }
-    float th_s[QT];
-    int th_i[QT];
-#pragma unroll
-    for (int j = 0; j < QT; ++j) {
-      th_s[j] = -INFINITY;
-      th_i[j] = INT_MAX;
-    }
+    float th_s = -INFINITY;
+    int th_i = INT_MAX;
     for (int tile_i = 0; tile_i < my_tiles; ++tile_i) {
       const int t = blockIdx.x + tile_i * gridDim.x;
       const int v0 = t * MMA_N;
       const int set = tile_i % NSETS;
       // scales of this tile's vectors (the previous tile's readers are done:
       // they passed the named barrier below)
-      for (int j = row; j < MMA_N; j += 128) {
+      for (int j = etid; j < MMA_N; j += EPI_THREADS) {
         const int v = v0 + j;
         sScale[j] = v < n ? (scale ? scale[v] : 1.0f) : 0.0f;
       }
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      // all four epilogue warps take the same decision, so none is left at bar.sync
+      asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
+      // all epilogue warps take the same decision, so none is left at bar.sync
       const int ok = warp_wait(acc_full + set, (tile_i / NSETS) & 1, abort_flag, err, 5) ? 1 : 0;
       int all_ok;
       asm volatile(
-          "{\n .reg .pred p, q;\n setp.ne.s32 p, %1, 0;\n bar.red.and.pred q, 1, 128, p;\n"
+          "{\n .reg .pred p, q;\n setp.ne.s32 p, %1, 0;\n bar.red.and.pred q, 1, %2, p;\n"
           " selp.s32 %0, 1, 0, q;\n}"
           : "=r"(all_ok)
-          : "r"(ok)
+          : "r"(ok), "n"(EPI_THREADS)
           : "memory");
       if (!all_ok) break;
       tc_fence_after();
-#pragma unroll
-      for (int j = 0; j < QT; ++j) {
-        const int q = (qt0 + j) * MMA_M + row;
-        if (j >= qts) break;
-        float* ls = lst_s + j * k * MMA_M;
-        int* li = lst_i + j * k * MMA_M;
-        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld32(tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + j) * MMA_N + c0), r);
-          if (q >= nq) continue;
-          // branch-free pass: scale and flag scores that may enter the list
-          const int valid = min(32, n - (v0 + c0));
+      if (mine) {
+        const uint32_t tb = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + jsel) * MMA_N);
+        // one 16-column chunk: scale, flag the scores that may enter the list
+        // (branch-free), then insert the flagged ones (rare after the first tiles)
+        auto chunk = [&](uint32_t (&r)[16], int c0) {
+          if (q >= nq) return;
+          const int valid = min(16, n - (v0 + c0));
           uint32_t m = 0;
 #pragma unroll
-          for (int jj = 0; jj < 32; ++jj) {
-            const float sc = __uint_as_float(r[jj]) * sScale[c0 + jj];
-            r[jj] = __float_as_uint(sc);
-            m |= (sc >= th_s[j] ? 1u : 0u) << jj;
+          for (int jj = 0; jj < 16; jj += 4) {
+            const float4 s4 = *reinterpret_cast<const float4*>(sScale + c0 + jj);
+            const float2 x = __fmul2_rn(make_float2(__uint_as_float(r[jj]), __uint_as_float(r[jj + 1])),
+                                        make_float2(s4.x, s4.y));
+            const float2 y = __fmul2_rn(make_float2(__uint_as_float(r[jj + 2]), __uint_as_float(r[jj + 3])),
+                                        make_float2(s4.z, s4.w));
+            r[jj] = __float_as_uint(x.x);
+            r[jj + 1] = __float_as_uint(x.y);
+            r[jj + 2] = __float_as_uint(y.x);
+            r[jj + 3] = __float_as_uint(y.y);
+            m |= (x.x >= th_s ? 1u : 0u) << jj;
+            m |= (x.y >= th_s ? 1u : 0u) << (jj + 1);
+            m |= (y.x >= th_s ? 1u : 0u) << (jj + 2);
+            m |= (y.y >= th_s ? 1u : 0u) << (jj + 3);
           }
-          if (valid < 32) m &= valid > 0 ? (1u << valid) - 1u : 0u;
-          if (m == 0u) continue;
-#pragma unroll
-          for (int jj = 0; jj < 32; ++jj) scr[jj * MMA_M + row] = __uint_as_float(r[jj]);
-          while (m) {  // rare after the first tiles
+          if (valid < 16) m &= valid > 0 ? (1u << valid) - 1u : 0u;
+          while (m) {  // rare after the first tiles; every step stays in registers but one load
             const int jj = __ffs(m) - 1;
             m &= m - 1;
-            const float sc = scr[jj * MMA_M + row];
+            float sc = 0.f;
+#pragma unroll
+            for (int t = 0; t < 16; ++t) sc = t == jj ? __uint_as_float(r[t]) : sc;
             const int v = v0 + c0 + jj;
-            if (!better(sc, v, th_s[j], th_i[j])) continue;
+            if (!better(sc, v, th_s, th_i)) continue;
+            // (sc, v) beats entry k-1: walk up while the entry above is worse,
+            // shifting it down; the new entry k-1 is the first one shifted, or
+            // (sc, v) itself if nothing moves
+            float nts = sc;
+            int nti = v;
             int pos = k - 1;
-            while (pos > 0 && better(sc, v, ls[(pos - 1) * MMA_M + row], li[(pos - 1) * MMA_M + row])) {
-              ls[pos * MMA_M + row] = ls[(pos - 1) * MMA_M + row];
-              li[pos * MMA_M + row] = li[(pos - 1) * MMA_M + row];
+            while (pos > 0) {
+              const float as = ls[(pos - 1) * MMA_M + row];
+              const int ai = li[(pos - 1) * MMA_M + row];
+              if (!better(sc, v, as, ai)) break;
+              ls[pos * MMA_M + row] = as;
+              li[pos * MMA_M + row] = ai;
+              if (pos == k - 1) {
+                nts = as;
+                nti = ai;
+              }
               --pos;
             }
             ls[pos * MMA_M + row] = sc;
             li[pos * MMA_M + row] = v;
-            th_s[j] = ls[(k - 1) * MMA_M + row];
-            th_i[j] = li[(k - 1) * MMA_M + row];
+            th_s = nts;
+            th_i = nti;
           }
+        };
+        // two chunks in flight: the next chunk's TMEM load overlaps this one's work
+        uint32_t ra[16], rb[16];
+        tmem_ld16_issue(tb, ra);
+        tmem_wait16(ra);
+#pragma unroll 1
+        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+          tmem_ld16_issue(tb + (uint32_t)(c0 + 16), rb);
+          chunk(ra, c0);
+          tmem_wait16(rb);
+          if (c0 + 32 < MMA_N) tmem_ld16_issue(tb + (uint32_t)(c0 + 32), ra);
+          chunk(rb, c0 + 16);
+          if (c0 + 32 < MMA_N) tmem_wait16(ra);
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty + set);
-      asm volatile("bar.sync 1, 128;" ::: "memory");
+      asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
     }
-    for (int j = 0; j < qts; ++j) {
-      const int q = (qt0 + j) * MMA_M + row;
-      if (q >= nq) continue;
+    if (mine && q < nq) {
       for (int i = 0; i < k; ++i) {
         const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
-        cand_s[o] = lst_s[(j * k + i) * MMA_M + row];
-        cand_i[o] = lst_i[(j * k + i) * MMA_M + row];
+        cand_s[o] = ls[i * MMA_M + row];
+        cand_i[o] = li[i * MMA_M + row];
       }
     }
   }
