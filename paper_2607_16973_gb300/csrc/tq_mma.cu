@@ -1,12 +1,15 @@
 // Tensor-core scan for query batches (Sec. II-B step 5 as a GEMM):
 //   S[q, v] = scale_v * sum_j q'_j c[code_vj]
 // with the rotated queries on the MMA's M dimension (128 per tile) and corpus
-// vectors on N (256 per MMA), fp16 operands and fp32 accumulation in tensor
+// vectors on N (256 per tile), fp16 operands and fp32 accumulation in tensor
 // memory (TMEM).  A CTA owns QT (1 or 2) query tiles and a strided set of
-// 256-vector tiles.  Roles (warp-specialised, 19 warps):
-//   warps 0-7   decoders: expand one K-block (64 coordinates) of packed codes,
-//               brought to shared memory by TMA, into fp16 centroid values
-//               laid out as the K-major, 128-byte-swizzled B operand;
+// vector tiles.  With one query tile TMEM holds two accumulator sets, so the
+// epilogue of one vector tile overlaps the MMAs of the next; with two, the
+// next tile's MMAs wait for the epilogue.  Roles (warp-specialised, 19 warps):
+//   warps 0-7   decoders, two groups of four on alternate K-blocks: expand
+//               one K-block (64 coordinates) of packed codes, brought to
+//               shared memory by TMA, into fp16 centroid values laid out as
+//               the K-major, 128-byte-swizzled B operand;
 //   warps 8-15  epilogue: read the 128 x 256 fp32 accumulators from TMEM (one
 //               query per thread; warps 8-11 the first query tile, 12-15 the
 //               second), apply the per-vector scale and keep each query's
@@ -16,8 +19,7 @@
 //               K=16) and commits completion to mbarriers;
 //   warp 18     query producer: 1-D bulk copies of pre-swizzled fp16 query
 //               blocks.
-// With one query tile TMEM holds two accumulator sets, so the epilogue of one
-// vector tile overlaps the MMAs of the next.  Every wait is bounded: on
+// Every wait is bounded: on
 // timeout the CTA raises `abort`, writes an error code to the status word and
 // exits after draining what it has in flight.
 #include <cuda.h>
@@ -43,14 +45,37 @@ constexpr int KB = 64;                // coordinates per K-block (128 B of fp16)
 constexpr int MAX_CST = 8;  // raw code tiles in flight (HBM latency)
 constexpr int RAW_ROW_MAX = 128;  // bytes of each row one code tile carries (one 128-B line)
 constexpr int MAX_AST = 4;  // query blocks in flight (L2-resident)
-constexpr int BST = 2;      // decoded fp16 tiles
-constexpr int DEC_WARPS = 8, DEC_THREADS = DEC_WARPS * 32;
-constexpr int EPI_WARP0 = 8, EPI_WARPS = 8, EPI_THREADS = EPI_WARPS * 32;
+constexpr int EPI_WARP0 = 8;
+// Decoders work in groups of four warps that take turns on K-blocks (group g
+// takes it = g, g + G, ...).  Warps 0-3, 4-7 and 19-22 are groups; with one
+// query tile the epilogue needs only warps 8-11, so warps 12-15 are a fourth.
+template <int QT>
+__host__ __device__ constexpr int dec_groups() { return QT == 1 ? 4 : 3; }
+// The plan runs ng <= dec_groups groups (as shared memory allows) and one
+// decoded fp16 stage per group: a group decodes its K-blocks in order, so it
+// is never more than one phase ahead on its stage's barriers (a shared stage
+// would let a group two phases ahead pass a parity wait early).
+// Decoder group of a warp, or -1.
+template <int QT>
+__device__ __forceinline__ int dec_group(int warp) {
+  if (warp < 8) return warp >> 2;
+  if (warp >= 19) return 2;
+  if (QT == 1 && warp >= 12 && warp < 16) return 3;
+  return -1;
+}
+template <int QT>
+__host__ __device__ constexpr int epi_warps() { return QT == 1 ? 4 : 8; }
 constexpr int CODE_WARP = 16, MMA_WARP = 17, QUERY_WARP = 18;
-constexpr int NTHREADS = 19 * 32;
+constexpr int NTHREADS = 23 * 32;  // warps 19-22: one more decoder group
 constexpr uint32_t kMaxDynSmem = 232448;  // 227 KB per block on sm_100-class GPUs
 constexpr int A_BYTES = MMA_M * KB * 2;   // 16 KB
-constexpr int B_BYTES = MMA_N * KB * 2;   // 32 KB
+// Vectors per tile.  (Tiles of 128 with two query tiles would leave room for
+// two accumulator sets, but M128 N128 MMAs ran at about two thirds of the
+// per-flop rate of N256 ones on this GPU, more than the overlap gains.)
+template <int QT>
+__host__ __device__ constexpr int tile_n() { return MMA_N; }
+template <int QT>
+__host__ __device__ constexpr int b_bytes() { return tile_n<QT>() * KB * 2; }
 constexpr long long WAIT_CYCLES = kWaitCycles;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -131,14 +156,17 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
 }
 
 // Instruction descriptor, kind::f16: D f32, A and B f16, both K-major, M x N.
-constexpr uint32_t IDESC = (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(MMA_N >> 3) << 17) |
-                           ((uint32_t)(MMA_M >> 4) << 24);
+template <int N>
+__host__ __device__ constexpr uint32_t idesc() {
+  return (1u << 4) | (0u << 7) | (0u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(MMA_M >> 4) << 24);
+}
 
+template <int N>
 __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
   asm volatile(
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}"
-      ::"r"(d_tmem), "l"(a), "l"(b), "r"(IDESC), "r"(accumulate));
+      ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc<N>()), "r"(accumulate));
 }
 
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -146,34 +174,9 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
                ::"r"(smem_u32(bar)) : "memory");
 }
 
-// Issues a 32-column TMEM load without waiting; tmem_wait below must run
-// before any of r is read.
-__device__ __forceinline__ void tmem_ld32_issue(uint32_t taddr, uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
-        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
-        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-}
-
-// Waits for this thread's outstanding TMEM loads.  r is passed through so the
-// compiler cannot move a read of r above the wait.
-__device__ __forceinline__ void tmem_wait(uint32_t (&r)[32]) {
-  asm volatile("tcgen05.wait::ld.sync.aligned;"
-               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
-                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
-                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
-                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
-                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
-               :
-               : "memory");
-}
-
+// Issues a 16-column TMEM load without waiting; tmem_wait16 must run before
+// any of r is read (r is passed through it, so the compiler cannot move a
+// read of r above the wait).
 __device__ __forceinline__ void tmem_ld16_issue(uint32_t taddr, uint32_t (&r)[16]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
@@ -190,20 +193,6 @@ __device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
                  "+r"(r[15])
                :
                : "memory");
-}
-
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
-        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
-        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
-        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
 __device__ __forceinline__ bool better(float s1, int i1, float s2, int i2) {
@@ -232,19 +221,19 @@ __host__ __device__ constexpr int tab_bytes() {
 // Shared-memory plan for QT query tiles per CTA, `cst` raw code stages and
 // `ast` query stages.
 template <int BITS, int QT>
-__host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int rr) {
+__host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int rr, int ng) {
   MmaSmem L{};
   uint32_t off = 0;
   L.a = off;
   off += (uint32_t)ast * QT * A_BYTES;
   L.b = off;
-  off += BST * B_BYTES;
+  off += (uint32_t)ng * b_bytes<QT>();
   L.raw = off;
-  off += (uint32_t)cst * MMA_N * rr;
+  off += (uint32_t)cst * tile_n<QT>() * rr;
   L.tab = off;
   off += tab_bytes<BITS>();
   L.scale = off;
-  off += MMA_N * 4;
+  off += tile_n<QT>() * 4;
   L.lists_s = off;
   off += (uint32_t)QT * k * MMA_M * 4;
   L.lists_i = off;
@@ -260,27 +249,55 @@ __host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int 
 
 struct MmaPlan {
   int qt = 1, cst = 2, ast = 2, rr = RAW_ROW_MAX;  // rr: bytes of each row per code tile
+  int ng = 2;                                      // decoder groups = decoded stages
   uint32_t smem = 0;
 };
 
-// Picks query tiles per CTA and ring depths that fit in shared memory:
-// prefer two query tiles per decoded code tile, then deep code prefetch.
+// Decoder groups that may run with code tiles of `sub` K-blocks in `cst`
+// stages.  Waits on a code stage use the phase parity, so a group must never
+// be two phases ahead on a stage: true when every group uses every tile
+// (sub >= g) or when each stage is always shared by the same groups
+// (cst * sub a multiple of g).
+int active_groups(int ng, int sub, int cst) {
+  int g = ng;
+  while (g > 2 && !(sub >= g || (cst * sub) % g == 0)) --g;
+  if (!(sub >= g || (cst * sub) % g == 0)) g = 1;
+  return g;
+}
+
+constexpr int MIN_PREFETCH_KB = 6;  // K-blocks of codes in flight (HBM latency)
+
+// Picks query tiles per CTA, decoder groups and ring depths that fit in shared
+// memory: prefer two query tiles per decoded code tile, then as many decoder
+// groups as the role layout has (all of them able to run), with at least
+// MIN_PREFETCH_KB K-blocks of codes in flight, then deeper rings.
 template <int BITS>
 MmaPlan mma_plan(int64_t nq, int k) {
   MmaPlan best;
-  for (int qt = (nq > MMA_M ? 2 : 1); qt >= 1; --qt) {
-    for (int rr = RAW_ROW_MAX; rr >= 64; rr >>= 1) {
-      for (int ast = 3; ast >= 2; --ast) {
-        for (int cst = MAX_CST; cst >= 2; --cst) {
-          const uint32_t need = qt == 2 ? mma_smem_layout<BITS, 2>(k, cst, ast, rr).total
-                                        : mma_smem_layout<BITS, 1>(k, cst, ast, rr).total;
-          if (need <= kMaxDynSmem) {
-            best.qt = qt;
-            best.cst = cst;
-            best.ast = ast;
-            best.rr = rr;
-            best.smem = need;
-            return best;
+  // first pass as above; the second relaxes the prefetch floor and allows
+  // fewer groups (large k at 8 bits needs the room for its lists)
+  for (int pass = 0; pass < 2; ++pass) {
+    const int min_pf = pass == 0 ? MIN_PREFETCH_KB : 2;
+    for (int qt = (nq > MMA_M ? 2 : 1); qt >= 1; --qt) {
+      const int gmax = qt == 2 ? dec_groups<2>() : dec_groups<1>();
+      for (int ng = gmax; ng >= 2; --ng) {
+        for (int rr = RAW_ROW_MAX; rr >= 64; rr >>= 1) {
+          const int sub = rr / raw_bytes_per_row<BITS>();  // for d a multiple of 256
+          for (int ast = 3; ast >= 2; --ast) {
+            for (int cst = MAX_CST; cst >= 2; --cst) {
+              if (cst * sub < min_pf || active_groups(ng, sub, cst) != ng) continue;
+              const uint32_t need = qt == 2 ? mma_smem_layout<BITS, 2>(k, cst, ast, rr, ng).total
+                                            : mma_smem_layout<BITS, 1>(k, cst, ast, rr, ng).total;
+              if (need <= kMaxDynSmem) {
+                best.qt = qt;
+                best.cst = cst;
+                best.ast = ast;
+                best.rr = rr;
+                best.ng = ng;
+                best.smem = need;
+                return best;
+              }
+            }
           }
         }
       }
@@ -331,20 +348,26 @@ template <int BITS, int QT>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,
            const float* __restrict__ centroids, const float* __restrict__ scale, int n, int nq, int d,
-           int k, int cst, int ast, int rr, int sub, float* __restrict__ cand_s, int* __restrict__ cand_i,
-           int* __restrict__ err) {
+           int k, int cst, int ast, int rr, int sub, int ng, int gact, float* __restrict__ cand_s,
+           int* __restrict__ cand_i, int* __restrict__ err) {
   constexpr int RAWB = raw_bytes_per_row<BITS>();
   // A code tile carries `sub` consecutive K-blocks of 256 rows: rows of
   // sub*RAWB bytes (128 B, one full line, when d allows), stored with the
   // 128-B swizzle in that case so the decoders' reads do not conflict.
   const int rrow = sub * RAWB;
   const bool swz = rrow == 128;
-  constexpr int NSETS = 2 / QT;  // accumulator sets in TMEM (2 = double buffered)
+  constexpr int NT = tile_n<QT>();       // vectors per tile
+  constexpr int B_BYTES = b_bytes<QT>();
+  constexpr int NSETS = 2 / QT;          // accumulator sets in TMEM (QT x NSETS x NT = 512 columns)
+  // gact <= ng decoder groups run (the launcher picks gact so that no group
+  // can get two phases ahead on a code stage); group g uses decoded stage g
+  const int G = gact, BST = gact;
+  constexpr int EPI_WARPS = epi_warps<QT>(), EPI_THREADS = EPI_WARPS * 32;
   extern __shared__ unsigned char smem_dyn[];
   // pointer arithmetic on the shared array (not an integer round trip) keeps
   // every access below a shared-memory access
   unsigned char* base = smem_dyn + ((1024u - (smem_u32(smem_dyn) & 1023u)) & 1023u);
-  const MmaSmem L = mma_smem_layout<BITS, QT>(k, cst, ast, rr);
+  const MmaSmem L = mma_smem_layout<BITS, QT>(k, cst, ast, rr, ng);
   unsigned char* sA = base + L.a;
   unsigned char* sB = base + L.b;
   unsigned char* sRaw = base + L.raw;
@@ -356,20 +379,20 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
   uint64_t* cempty = bars + 8;                 // [MAX_CST] code tile decoded (stage free)
   uint64_t* afull = bars + 16;                 // [MAX_AST] query block(s) landed
   uint64_t* aempty = bars + 20;                // [MAX_AST] MMAs done with the query block(s)
-  uint64_t* dec = bars + 24;                   // [BST] decoded B tile written
-  uint64_t* bempty = bars + 26;                // [BST] MMAs done with the decoded tile
-  uint64_t* acc_full = bars + 28;              // [NSETS] accumulators complete
-  uint64_t* acc_empty = bars + 30;             // [NSETS] accumulators read out
-  uint64_t* fin = bars + 32;                   // all MMAs of this CTA complete
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 33);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 34);
+  uint64_t* dec = bars + 24;                   // [BST <= 4] decoded B tile written
+  uint64_t* bempty = bars + 28;                // [BST] MMAs done with the decoded tile
+  uint64_t* acc_full = bars + 32;              // [NSETS] accumulators complete
+  uint64_t* acc_empty = bars + 34;             // [NSETS] accumulators read out
+  uint64_t* fin = bars + 36;                   // all MMAs of this CTA complete
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 37);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 38);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int qt0 = blockIdx.y * QT;                     // first query tile of this CTA
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const int qts = min(QT, nqt - qt0);                  // query tiles present (1..QT)
   const int kblocks = d / KB;
-  const int ntiles = (n + MMA_N - 1) / MMA_N;
+  const int ntiles = (n + NT - 1) / NT;
   const int my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
   if (BITS == 2) {
@@ -386,14 +409,16 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
   if (tid == 0) {
     for (int s = 0; s < MAX_CST; ++s) {
       mbar_init(cfull + s, 1);
-      mbar_init(cempty + s, DEC_WARPS);  // one arrival per decoder warp
+      // one arrival per decoder warp that uses the tile: a tile of `sub`
+      // consecutive K-blocks is used by min(sub, G) groups
+      mbar_init(cempty + s, 4 * min(sub, G));
     }
     for (int s = 0; s < MAX_AST; ++s) {
       mbar_init(afull + s, 1);
       mbar_init(aempty + s, 1);
     }
     for (int s = 0; s < BST; ++s) {
-      mbar_init(dec + s, DEC_WARPS);
+      mbar_init(dec + s, 4);  // the four warps of one decoder group
       mbar_init(bempty + s, 1);
     }
     for (int b = 0; b < NSETS; ++b) {
@@ -425,8 +450,8 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
         const int it = ld * sub;
         const int t = blockIdx.x + (it / kblocks) * gridDim.x;
         const int kb = it % kblocks;
-        mbar_arrive_expect_tx(cfull + s, MMA_N * rrow);
-        tma_load_2d(sRaw + s * MMA_N * rr, &codes_map, kb * RAWB, t * MMA_N, cfull + s);
+        mbar_arrive_expect_tx(cfull + s, NT * rrow);
+        tma_load_2d(sRaw + s * NT * rr, &codes_map, kb * RAWB, t * NT, cfull + s);
         issued = ld + 1;
       }
       // never leave with copies in flight: wait (bounded) for the last one of each stage
@@ -460,10 +485,10 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
         const uint32_t b0 = smem_u32(sB + bs * B_BYTES);
         for (int j = 0; j < qts; ++j) {
           const uint32_t a0 = smem_u32(sA + (as * QT + j) * A_BYTES);
-          const uint32_t dt = tmem + (uint32_t)((set * QT + j) * MMA_N);
+          const uint32_t dt = tmem + (uint32_t)((set * QT + j) * NT);
 #pragma unroll
           for (int kk = 0; kk < KB / 16; ++kk)
-            mma_f16(dt, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), (kb | kk) != 0);
+            mma_f16<NT>(dt, sw128_desc(a0 + kk * 32), sw128_desc(b0 + kk * 32), (kb | kk) != 0);
         }
         mma_commit(bempty + bs);
         mma_commit(aempty + as);
@@ -488,7 +513,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       mma_commit(fin);
       mbar_wait_drain(fin, 0);
     }
-  } else if (warp < DEC_WARPS) {
+  } else if (dec_group<QT>(warp) >= 0) {
     // ---------------------------------------------------------- decoders
     constexpr int PARTS = RAWB / 16;                 // 16-byte parts per row per K-block
     constexpr int CODES = 16 * 8 / BITS;             // codes per part
@@ -503,13 +528,19 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
         th[e >> 2] |= (bitsv >> 8) << (8 * (e & 3));
       }
     }
-    int sb = 0, cs = 0, cpar = 0, bs = 0, bpar = 0;  // sub-block, code stage + parity, B stage + parity
-    for (int it = 0; it < total_it; ++it) {
-      if (!warp_wait(cfull + cs, cpar, abort_flag, err, 4)) break;
-      if (it >= BST && !warp_wait(bempty + bs, bpar ^ 1, abort_flag, err, 8)) break;
-      const unsigned char* raw = sRaw + cs * MMA_N * rr;
+    // G groups of four warps take turns on K-blocks (group g: it = g, g + G,
+    // ...), so one group's fence and barrier round trip overlap the others'
+    // decoding.  K-block it goes to decoded stage it % BST = the group's own.
+    const int grp = dec_group<QT>(warp);
+    const int gtid = (warp & 3) * 32 + lane;
+    for (int it = grp < G ? grp : total_it; it < total_it; it += G) {  // groups >= gact stay idle
+      const int ld = it / sub, sb = it % sub;           // code tile and its K-block
+      const int cs = ld % cst, bs = it % BST;
+      if (!warp_wait(cfull + cs, (ld / cst) & 1, abort_flag, err, 4)) break;
+      if (it >= BST && !warp_wait(bempty + bs, ((it / BST) - 1) & 1, abort_flag, err, 8)) break;
+      const unsigned char* raw = sRaw + cs * NT * rr;
       unsigned char* bdst = sB + bs * B_BYTES;
-      for (int item = tid; item < MMA_N * PARTS; item += DEC_THREADS) {
+      for (int item = gtid; item < NT * PARTS; item += 128) {
         const int r = item / PARTS, p = item % PARTS;
         const int chunk = sb * PARTS + p;  // 16-byte chunk of the row in this code tile
         const uint4 w4 = *reinterpret_cast<const uint4*>(
@@ -543,19 +574,8 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       fence_proxy_async();  // make this thread's writes visible to the tensor core
       __syncwarp();
       if (lane == 0) {
-        if (sb == sub - 1) mbar_arrive(cempty + cs);  // the whole code tile is decoded
+        if (sb + G >= sub) mbar_arrive(cempty + cs);  // this group's last K-block of the code tile
         mbar_arrive(dec + bs);
-      }
-      if (++sb == sub) {
-        sb = 0;
-        if (++cs == cst) {
-          cs = 0;
-          cpar ^= 1;
-        }
-      }
-      if (++bs == BST) {
-        bs = 0;
-        bpar ^= 1;
       }
     }
   } else {
@@ -582,11 +602,11 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     int th_i = INT_MAX;
     for (int tile_i = 0; tile_i < my_tiles; ++tile_i) {
       const int t = blockIdx.x + tile_i * gridDim.x;
-      const int v0 = t * MMA_N;
+      const int v0 = t * NT;
       const int set = tile_i % NSETS;
       // scales of this tile's vectors (the previous tile's readers are done:
       // they passed the named barrier below)
-      for (int j = etid; j < MMA_N; j += EPI_THREADS) {
+      for (int j = etid; j < NT; j += EPI_THREADS) {
         const int v = v0 + j;
         sScale[j] = v < n ? (scale ? scale[v] : 1.0f) : 0.0f;
       }
@@ -603,7 +623,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       if (!all_ok) break;
       tc_fence_after();
       if (mine) {
-        const uint32_t tb = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + jsel) * MMA_N);
+        const uint32_t tb = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + jsel) * NT);
         // one 16-column chunk: scale, flag the scores that may enter the list
         // (branch-free), then insert the flagged ones (rare after the first tiles)
         auto chunk = [&](uint32_t (&r)[16], int c0) {
@@ -664,13 +684,13 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
         tmem_ld16_issue(tb, ra);
         tmem_wait16(ra);
 #pragma unroll 1
-        for (int c0 = 0; c0 < MMA_N; c0 += 32) {
+        for (int c0 = 0; c0 < NT; c0 += 32) {
           tmem_ld16_issue(tb + (uint32_t)(c0 + 16), rb);
           chunk(ra, c0);
           tmem_wait16(rb);
-          if (c0 + 32 < MMA_N) tmem_ld16_issue(tb + (uint32_t)(c0 + 32), ra);
+          if (c0 + 32 < NT) tmem_ld16_issue(tb + (uint32_t)(c0 + 32), ra);
           chunk(rb, c0 + 16);
-          if (c0 + 32 < MMA_N) tmem_wait16(ra);
+          if (c0 + 32 < NT) tmem_wait16(ra);
         }
       }
       tc_fence_before();
@@ -732,13 +752,14 @@ template <int BITS, int QT>
 cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half* qpack, const float* centroids,
                          const float* scale, int n, int nq, int d, int k, int sub, int grid_x, float* cs,
                          int* ci, int* err, cudaStream_t s) {
+  const int gact = active_groups(P.ng, sub, P.cst);
   cudaError_t e = cudaFuncSetAttribute(k_scan_mma<BITS, QT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)P.smem);
   if (e != cudaSuccess) return e;
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));
   k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, n, nq, d, k, P.cst, P.ast,
-                                                         P.rr, sub, cs, ci, err);
+                                                         P.rr, sub, P.ng, gact, cs, ci, err);
   return cudaGetLastError();
 }
 
