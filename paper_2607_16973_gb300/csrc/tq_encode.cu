@@ -48,23 +48,24 @@ __device__ __forceinline__ void store_slice(float (*S)[BM + PAD], float4 v) {
 // columns tx*4 + {0..3} (+64): acc[i][j], i < 4 -> first row block.
 __device__ __forceinline__ void gemm_tile(const float* __restrict__ X, int64_t row0, int64_t n_rows,
                                           const float* __restrict__ R, int col0, int d,
-                                          GemmSmem& sm, float acc[8][8]) {
+                                          GemmSmem& sm, float acc[8][8], int k0 = 0, int k1 = -1) {
+  if (k1 < 0) k1 = d;  // the contraction covers coordinates [k0, k1)
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
 #pragma unroll
   for (int i = 0; i < 8; ++i)
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-  const int nk = d / BK;
-  float4 pa = load_slice(X, row0, n_rows, d, 0);
-  float4 pb = load_slice(R, col0, d, d, 0);
+  const int nk = (k1 - k0) / BK;
+  float4 pa = load_slice(X, row0, n_rows, d, k0);
+  float4 pb = load_slice(R, col0, d, d, k0);
   store_slice(sm.A[0], pa);
   store_slice(sm.B[0], pb);
   __syncthreads();
   for (int kt = 0; kt < nk; ++kt) {
     const int buf = kt & 1;
     if (kt + 1 < nk) {
-      pa = load_slice(X, row0, n_rows, d, (kt + 1) * BK);
-      pb = load_slice(R, col0, d, d, (kt + 1) * BK);
+      pa = load_slice(X, row0, n_rows, d, k0 + (kt + 1) * BK);
+      pb = load_slice(R, col0, d, d, k0 + (kt + 1) * BK);
     }
 #pragma unroll
     for (int k = 0; k < BK; ++k) {
@@ -232,11 +233,18 @@ __global__ void __launch_bounds__(NT, 2)
 k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R,
               float* __restrict__ out, int* __restrict__ status) {
   __shared__ GemmSmem sm;
-  if (status && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
+  if (status && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0) *status = 0;
   const int64_t row0 = (int64_t)blockIdx.x * BM;
   const int col0 = blockIdx.y * BN;
+  // gridDim.z = 2 splits the contraction in halves, each added onto the
+  // zeroed output: two fp32 additions onto 0 give the same sum in either
+  // order, so the result does not depend on which half lands first
+  const int half = d / 2;
   float acc[8][8];
-  gemm_tile(Q, row0, nq, R, col0, d, sm, acc);
+  if (gridDim.z == 2)
+    gemm_tile(Q, row0, nq, R, col0, d, sm, acc, blockIdx.z * half, (blockIdx.z + 1) * half);
+  else
+    gemm_tile(Q, row0, nq, R, col0, d, sm, acc);
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     const int64_t r = row0 + tile_row(i);
@@ -244,7 +252,9 @@ k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __res
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int c = col0 + tile_col(j);
-      if (c < d) out[r * d + c] = acc[i][j];
+      if (c >= d) continue;
+      if (gridDim.z == 2) atomicAdd(out + r * d + c, acc[i][j]);
+      else out[r * d + c] = acc[i][j];
     }
   }
 }
@@ -345,7 +355,15 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
     k_rotate_gemv<8><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status);
     return cudaGetLastError();
   }
-  dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN));
+  // split the contraction in two when the tiles alone would leave SMs idle
+  // (each half must be a whole number of BK slices)
+  const int64_t tiles = ((nq + BM - 1) / BM) * ((d + BN - 1) / BN);
+  const bool split = tiles < device_sm_count() && (d / 2) % BK == 0;
+  if (split) {
+    const cudaError_t e = cudaMemsetAsync(out, 0, (size_t)nq * d * sizeof(float), s);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN), split ? 2u : 1u);
   k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out, status);
   return cudaGetLastError();
 }
