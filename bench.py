@@ -50,6 +50,13 @@ CONFIGS = {
     "tiny": dict(n=10_000, d=1536, bits=4, clusters=64, pool=100, k=10, batches=[1, 100]),
     # profiling case: codes (192 MB) larger than L2, a few GB on the device at most
     "prof": dict(n=250_000, d=1536, bits=4, clusters=256, pool=2_048, k=5, batches=[1, 1024]),
+    # filtered search: Zipf(1.1) tenants, allowlist of one tenant (10% of the
+    # queries five), 64-vector filter blocks
+    "filtered": dict(n=100_000, d=1536, bits=4, clusters=256, pool=1_000, k=10, batches=[1],
+                     tenants=[10, 100, 1000], block=64),
+    # bit-width sweep: encode and batch-256 top-10 search at b = 2, 3, 4, 8
+    "sweep": dict(n=999_000, d=1536, bits=4, clusters=1024, pool=2_000, k=10, batches=[256],
+                  sweep_bits=[2, 3, 4, 8]),
 }
 
 RECALL_Q = 200       # queries whose Recall@k against exact kNN the bench reports
@@ -520,6 +527,158 @@ def run_ours(args, cfg, rank, world):
         print(json.dumps(line), flush=True)
 
 
+def _timed(fn, steps, warmup, stream):
+    """Mean ms of fn() over `steps` calls after `warmup`, CUDA events on `stream`."""
+    import torch
+    for i in range(warmup):
+        fn(i)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record(stream)
+    for i in range(steps):
+        fn(warmup + i)
+    b.record(stream)
+    b.synchronize()
+    return a.elapsed_time(b) / steps
+
+
+def run_filtered(args, cfg):
+    """Filtered search (allowlists of tenants) at batch 1 for each tenant
+    count: queries/s, the share of code bytes the per-block tenant bitmaps
+    skip, and Recall@k against exact filtered kNN."""
+    import torch
+    import paper_2607_16973_gb300 as tq
+    from paper_2607_16973_gb300 import synth
+    from paper_2607_16973_gb300.build import build
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build()
+    tq.load()
+    n, d, bits, k, blk = cfg["n"], cfg["d"], cfg["bits"], args.k or cfg["k"], cfg["block"]
+    stream = torch.cuda.Stream(device=dev)
+    X = synth.mixture_corpus(n, d, cfg["clusters"], workers=min(16, os.cpu_count() or 4))
+    src = synth.query_sources(n, cfg["pool"])
+    Q = synth.perturb(X[src])
+    cen, bnd, _ = tq.codebook(d, bits)
+    R = tq.rotation(d, synth.SEED_ROTATION)
+    Xd, Qd = torch.from_numpy(X).to(dev), torch.from_numpy(Q).to(dev)
+    Rd, cd, bd = (torch.from_numpy(a).to(dev) for a in (R, cen, bnd))
+    codes, scale = tq.encode(Xd, Rd, cd, bd, bits)
+    torch.cuda.synchronize()
+    torch.backends.cuda.matmul.allow_tf32 = False
+    nrec = min(RECALL_Q, len(Q))
+    exact_scores = Qd[:nrec] @ Xd.T                       # [nrec, n] float32, unquantised
+    variants = {}
+    steps = min(args.steps, len(Q) - args.warmup) if len(Q) > args.warmup else args.steps
+    for T in cfg["tenants"]:
+        tid, values = synth.zipf_tenants(n, T)
+        off, allow = synth.allowlists(src, tid, values)
+        filt = tq.Filter(torch.from_numpy(tid.view(np.int32)).to(dev), block=blk)
+        # per-query CSR slices (offsets rebased to 0), on the device
+        q_off = [torch.tensor([0, off[i + 1] - off[i]], dtype=torch.int64, device=dev) for i in range(len(Q))]
+        q_ten = [torch.from_numpy(allow[off[i]:off[i + 1]].view(np.int32)).to(dev) for i in range(len(Q))]
+        ws = torch.empty(tq.search_workspace(1, n, d, bits, k, filt), dtype=torch.uint8, device=dev)
+        ids = torch.empty((1, k), dtype=torch.int64, device=dev)
+        scs = torch.empty((1, k), dtype=torch.float32, device=dev)
+
+        def step(i):
+            j = i % len(Q)
+            tq.search(Qd[j:j + 1], Rd, cd, bits, codes, scale, k, filter=filt, allow_off=q_off[j],
+                      allow_tenants=q_ten[j], workspace=ws, out_ids=ids, out_scores=scs, stream=stream)
+
+        with torch.cuda.stream(stream):
+            ms = _timed(step, steps, args.warmup, stream)
+        # share of code blocks skipped (no allowed tenant in the block)
+        nblocks = (n + blk - 1) // blk
+        pad = np.full(nblocks * blk - n, np.uint32(0xFFFFFFFF), np.uint32)
+        tb = np.concatenate([tid, pad]).reshape(nblocks, blk)
+        skipped = []
+        for i in range(min(200, len(Q))):
+            ok = np.isin(tb, allow[off[i]:off[i + 1]]).any(axis=1)
+            skipped.append(1.0 - ok.mean())
+        # Recall@k against exact kNN restricted to the allowed vectors
+        hits = 0.0
+        for i in range(nrec):
+            mask = torch.from_numpy(np.isin(tid, allow[off[i]:off[i + 1]])).to(dev)
+            sc = torch.where(mask, exact_scores[i], torch.tensor(float("-inf"), device=dev))
+            ex = torch.topk(sc, min(k, int(mask.sum())))[1]
+            with torch.cuda.stream(stream):
+                got, _ = tq.search(Qd[i:i + 1], Rd, cd, bits, codes, scale, k, filter=filt, allow_off=q_off[i],
+                                   allow_tenants=q_ten[i], stream=stream)
+            stream.synchronize()
+            g = got[0][got[0] >= 0]
+            hits += float(torch.isin(g, ex).float().sum()) / max(1, len(ex))
+        variants[str(T)] = {"value": 1e3 / ms, "ms_per_query": ms, "bytes_skipped_frac": float(np.mean(skipped)),
+                            "recall": hits / nrec}
+        log(f"[bench] filtered T={T}: {1e3 / ms:.4g} q/s, {ms * 1e3:.1f} us/query, "
+            f"{100 * np.mean(skipped):.1f}% of code blocks skipped, R@{k} {hits / nrec:.3f}")
+        filt.close()
+    head = variants[str(cfg["tenants"][0])]
+    line = {"metric": f"filtered queries/sec at {n // 1000}Kx{d} {bits}-bit top-{k} (batch 1)", "value": head["value"],
+            "unit": "queries/s", "n_gpus": 1, "steps": steps, "warmup": args.warmup,
+            "ms_per_step": head["ms_per_query"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic (Gaussian mixture, Zipf(1.1) tenants in interleaved order)",
+            "config": {"workload": f"filtered: N={n} d={d} {bits}-bit top-{k}, Zipf tenants T in {cfg['tenants']}, "
+                                   f"block {blk}, 10% of queries allow 5 tenants", "n": n, "d": d, "bits": bits,
+                       "k": k, "block": blk},
+            "variants": variants, "gpu_launches": 4 * steps}
+    print(json.dumps(line), flush=True)
+
+
+def run_sweep(args, cfg):
+    """Encode throughput and batch-B top-k search at each bit width."""
+    import torch
+    import paper_2607_16973_gb300 as tq
+    from paper_2607_16973_gb300 import synth
+    from paper_2607_16973_gb300.build import build
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build()
+    tq.load()
+    n, d, k = cfg["n"], cfg["d"], args.k or cfg["k"]
+    B = int(args.batches.split(",")[0]) if args.batches else cfg["batches"][0]
+    stream = torch.cuda.Stream(device=dev)
+    X, Qpool = make_corpus(cfg, workers=min(16, os.cpu_count() or 4))
+    R = tq.rotation(d, synth.SEED_ROTATION)
+    Xd, Rd, Qd = torch.from_numpy(X).to(dev), torch.from_numpy(R).to(dev), torch.from_numpy(Qpool).to(dev)
+    del X
+    nb = max(1, len(Qpool) // B)
+    variants = {}
+    for bits in cfg["sweep_bits"]:
+        cen, bnd, _ = tq.codebook(d, bits)
+        cd, bd = torch.from_numpy(cen).to(dev), torch.from_numpy(bnd).to(dev)
+        codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
+        scale = torch.empty(n, dtype=torch.float32, device=dev)
+        with torch.cuda.stream(stream):
+            enc_ms = _timed(lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream), 3, 1,
+                            stream)
+            ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
+            ids = torch.empty((B, k), dtype=torch.int64, device=dev)
+            scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+            steps = max(1, min(args.steps, 10))
+            ms = _timed(lambda i: tq.search(Qd[(i % nb) * B:(i % nb) * B + B], Rd, cd, bits, codes, scale, k,
+                                            workspace=ws, out_ids=ids, out_scores=scs, stream=stream),
+                        steps, min(args.warmup, 3), stream)
+        path = "tensor core" if bits in (2, 4, 8) and k <= 64 else "lookup"
+        variants[str(bits)] = {"encode_vectors_per_s": n / enc_ms * 1e3, "encode_ms": enc_ms,
+                               "value": B / ms * 1e3, "ms_per_step": ms, "path": path,
+                               "codes_mb": n * d * bits / 8 / 1e6}
+        log(f"[bench] sweep b={bits}: encode {n / enc_ms * 1e3:.3g} vec/s, search B={B} {B / ms * 1e3:.4g} q/s "
+            f"({path})")
+        del codes, scale, ws
+        torch.cuda.empty_cache()
+    head = variants[str(cfg["sweep_bits"][0])]
+    line = {"metric": f"queries/sec at {n // 1000}Kx{d} top-{k} batch {B} by bit width; encode vectors/sec",
+            "value": head["value"], "unit": "queries/s", "n_gpus": 1, "steps": max(1, min(args.steps, 10)),
+            "warmup": min(args.warmup, 3), "ms_per_step": head["ms_per_step"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded Gaussian-mixture corpus, perturbed-corpus queries)",
+            "config": {"workload": f"sweep: N={n} d={d} b in {cfg['sweep_bits']}, batch {B}, top-{k}", "n": n, "d": d,
+                       "k": k, "batch": B},
+            "variants": variants}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -537,6 +696,10 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     if args.impl == "reference":
         run_reference(args, cfg, rank, world)
+        return
+    if args.config in ("filtered", "sweep"):
+        if rank == 0:
+            (run_filtered if args.config == "filtered" else run_sweep)(args, cfg)
         return
     if world > 1:
         import torch
