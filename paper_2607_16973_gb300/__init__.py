@@ -131,8 +131,8 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
         out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
     if out_scores is None:
         out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
-    need = search_workspace(nq, n, d, bits, k, filter)
-    if workspace is None:
+    if workspace is None:  # a caller-owned workspace is size-checked by tq_search itself
+        need = search_workspace(nq, n, d, bits, k, filter)
         workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
     f32 = torch.float32
     u32 = (torch.int32, getattr(torch, "uint32", torch.int32))

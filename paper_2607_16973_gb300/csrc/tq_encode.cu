@@ -9,7 +9,9 @@
 // and packs the codes straight to HBM (little-endian bit stream per row).
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
+#include <mutex>
 
 #include "tq_internal.h"
 #include "tq_kernels.h"
@@ -313,11 +315,46 @@ k_rotate_gemv(const float* __restrict__ Q, int64_t nq, int d, const float* __res
 
 }  // namespace
 
+// SM count of the current device, queried once per device.
 int device_sm_count() {
+  constexpr int kMaxDev = 64;
+  static std::atomic<int> cache[kMaxDev];
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 1;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
-  return sms > 0 ? sms : 1;
+  if (dev >= 0 && dev < kMaxDev && (sms = cache[dev].load(std::memory_order_relaxed)) > 0) return sms;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) return 1;
+  if (dev >= 0 && dev < kMaxDev) cache[dev].store(sms, std::memory_order_relaxed);
+  return sms;
+}
+
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per kernel, device
+// and size: the call is not free, and the searches launch on every request.
+cudaError_t set_max_dynamic_smem(const void* func, int bytes) {
+  struct Entry {
+    const void* func;
+    int dev, bytes;
+  };
+  static std::mutex mu;
+  static Entry seen[256];
+  static int nseen = 0;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < nseen; ++i)
+      if (seen[i].func == func && seen[i].dev == dev && seen[i].bytes >= bytes) return cudaSuccess;
+  }
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < nseen; ++i)
+    if (seen[i].func == func && seen[i].dev == dev) {
+      if (bytes > seen[i].bytes) seen[i].bytes = bytes;
+      return cudaSuccess;
+    }
+  if (nseen < 256) seen[nseen++] = Entry{func, dev, bytes};
+  return cudaSuccess;
 }
 
 cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,

@@ -61,6 +61,7 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
                             cudaEvent_t ev0, cudaEvent_t ev1);
 
 int device_sm_count();
+cudaError_t set_max_dynamic_smem(const void* func, int bytes);
 
 // cudaMalloc that fails while the calling thread's tq_debug_fail_allocs
 // count is positive (testing hook for the out-of-memory paths).

@@ -753,8 +753,7 @@ cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half*
                          const float* scale, int n, int nq, int d, int k, int sub, int grid_x, float* cs,
                          int* ci, int* err, cudaStream_t s) {
   const int gact = active_groups(P.ng, sub, P.cst);
-  cudaError_t e = cudaFuncSetAttribute(k_scan_mma<BITS, QT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)P.smem);
+  cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_mma<BITS, QT>), (int)P.smem);
   if (e != cudaSuccess) return e;
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));

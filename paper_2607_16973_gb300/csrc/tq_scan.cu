@@ -646,21 +646,20 @@ k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t 
 // Merge of per-CTA candidate lists that are each sorted best first and hold
 // exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
 // any one list is beaten or matched by that list's k entries, so the global
-// k-th best is at least as good as the best such T, and only candidates at
-// least as good as it can be in the global top-k.  Those survivors (at least
-// k of them, usually few more) are compacted; each then finds its rank by
-// counting the survivors ahead of it (equal pairs, which only padding can
-// form, are ordered by slot) and the first k ranks are written out.  If more
-// survive than the P slots hold, the block sorts everything in chunks.
+// k-th best is at least as good as the best such T and worse candidates are
+// skipped at once.  Each warp keeps a sorted top-k of its share of the rest
+// (ballot, then one warp-wide insertion per candidate that still beats the
+// warp's k-th); warp 0 then folds the sorted warp lists into the result,
+// leaving each list at its first entry that no longer qualifies.
 __global__ void __launch_bounds__(1024)
-k_merge_sorted_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k, int P,
-                     int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+k_merge_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k,
+              int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  int* id = reinterpret_cast<int*>(smem_raw);
-  float* s = reinterpret_cast<float*>(id + P);
+  const int nwarps = blockDim.x >> 5;
+  float* ws = reinterpret_cast<float*>(smem_raw);  // [nwarps][k]
+  int* wi = reinterpret_cast<int*>(ws + nwarps * k);
   __shared__ float red_s[32];
   __shared__ int red_i[32];
-  __shared__ int count;
   const int64_t q = blockIdx.x;
   const int total = nlists * k;
   const float* cs = cand_s + q * total;
@@ -690,67 +689,70 @@ k_merge_sorted_lists(const float* __restrict__ cand_s, const int* __restrict__ c
     red_s[warp] = ts;
     red_i[warp] = ti;
   }
-  if (tid == 0) count = 0;
+  for (int i = lane; i < k; i += 32) {
+    ws[warp * k + i] = -INFINITY;
+    wi[warp * k + i] = INT_MAX;
+  }
   __syncthreads();
   ts = red_s[0];
   ti = red_i[0];
-  for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+  for (int w = 1; w < nwarps; ++w)
     if (better(red_s[w], red_i[w], ts, ti)) {
       ts = red_s[w];
       ti = red_i[w];
     }
-  // 2. compact the candidates at least as good as T
-  for (int c = tid; c < total; c += blockDim.x) {
-    const float a = cs[c];
-    const int b = ci[c];
-    if (!better(ts, ti, a, b)) {
-      const int pos = atomicAdd(&count, 1);
-      if (pos < P) {
-        s[pos] = a;
-        id[pos] = b;
+  // 2. per-warp sorted top-k of the candidates at least as good as T
+  float* ls = ws + warp * k;
+  int* li = wi + warp * k;
+  int cnt = 0;
+  float th_s = -INFINITY;
+  int th_i = INT_MAX;
+  for (int c0 = warp * 32; c0 < total; c0 += blockDim.x) {
+    const int c = c0 + lane;
+    float a = -INFINITY;
+    int b = INT_MAX;
+    if (c < total) {
+      a = cs[c];
+      b = ci[c];
+    }
+    const bool cand = b != INT_MAX && !better(ts, ti, a, b) && better(a, b, th_s, th_i);
+    unsigned m = __ballot_sync(FULL, cand);
+    while (m) {
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      const float sv = __shfl_sync(FULL, a, src);
+      const int iv = __shfl_sync(FULL, b, src);
+      if (better(sv, iv, th_s, th_i)) {
+        warp_insert(ls, li, k, cnt, sv, iv);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = ls[k - 1];
+          th_i = li[k - 1];
+        }
       }
     }
   }
   __syncthreads();
-  const int m = count;
-  if (m > P) {  // 3a. too many survivors (e.g. mostly padding): sort everything in chunks
-    for (int i = tid; i < k; i += blockDim.x) {
-      s[i] = -INFINITY;
-      id[i] = INT_MAX;
-    }
-    const int chunk = P - k;
-    for (int c0 = 0; c0 < total; c0 += chunk) {
-      __syncthreads();
-      for (int i = tid; i < chunk; i += blockDim.x) {
-        const int c = c0 + i;
-        s[k + i] = c < total ? cs[c] : -INFINITY;
-        id[k + i] = c < total ? ci[c] : INT_MAX;
-      }
-      __syncthreads();
-      block_sort(s, id, P);
-    }
-  } else {  // 3b. rank the survivors
-    for (int i = tid; i < m; i += blockDim.x) {
-      const float a = s[i];
-      const int b = id[i];
-      int r = 0;
-      for (int j = 0; j < m; ++j) {
-        const float sj = s[j];
-        const int ij = id[j];
-        r += better(sj, ij, a, b) || (sj == a && ij == b && j < i);
-      }
-      if (r < k) {
-        const bool empty = b == INT_MAX;
-        out_ids[q * k + r] = empty ? -1 : (int64_t)b;
-        out_scores[q * k + r] = empty ? -INFINITY : a;
+  // 3. warp 0 folds the other warps' sorted lists into its own
+  if (warp == 0) {
+    for (int w = 1; w < nwarps; ++w) {
+      for (int i = 0; i < k; ++i) {
+        const float sv = ws[w * k + i];
+        const int iv = wi[w * k + i];
+        if (iv == INT_MAX || !better(sv, iv, th_s, th_i)) break;  // sorted: the rest are worse
+        warp_insert(ls, li, k, cnt, sv, iv);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = ls[k - 1];
+          th_i = li[k - 1];
+        }
       }
     }
-    return;
-  }
-  for (int i = tid; i < k; i += blockDim.x) {
-    const bool empty = id[i] == INT_MAX;
-    out_ids[q * k + i] = empty ? -1 : (int64_t)id[i];
-    out_scores[q * k + i] = empty ? -INFINITY : s[i];
+    for (int i = lane; i < k; i += 32) {
+      const bool empty = li[i] == INT_MAX;
+      out_ids[q * k + i] = empty ? -1 : (int64_t)li[i];
+      out_scores[q * k + i] = empty ? -INFINITY : ls[i];
+    }
   }
 }
 
@@ -802,19 +804,19 @@ cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* 
   cudaError_t e;
   if (BITS == 4 && !allow) {
     const size_t psmem = (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int));
-    e = cudaFuncSetAttribute(k_scan_pair_stream<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+    e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_pair_stream<S>), (int)psmem);
     if (e != cudaSuccess) return e;
     k_scan_pair_stream<S><<<grid, SCAN_NT, psmem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
     return cudaGetLastError();
   }
   if (!allow) {
-    e = cudaFuncSetAttribute(k_scan_lut_stream<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut_stream<BITS, S>), (int)smem);
     if (e != cudaSuccess) return e;
     k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
     return cudaGetLastError();
   }
   const size_t fsmem = BITS == 4 ? (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int)) : smem;
-  e = cudaFuncSetAttribute(k_scan_lut<BITS, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)fsmem);
+  e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut<BITS, S>), (int)fsmem);
   if (e != cudaSuccess) return e;
   k_scan_lut<BITS, S><<<grid, SCAN_NT, fsmem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
                                                    words, fblock, allow, k, P, cs, ci);
@@ -881,9 +883,12 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
                          int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   // per_query = grid_x * k: one sorted list of k per scan CTA
-  const int P = std::min(MERGE_P, next_pow2(std::max(per_query + k, 64)));
-  const size_t smem = (size_t)P * (sizeof(float) + sizeof(int32_t));
-  k_merge_sorted_lists<<<(unsigned)nq, 1024, smem, s>>>(cand_s, cand_i, per_query / k, k, P, out_ids, out_scores);
+  // up to 32 warps, fewer for long lists (each warp keeps k entries in shared memory)
+  const int nlists = per_query / k;
+  int warps = std::max(1, std::min(32, (nlists + 31) / 32));
+  while (warps > 1 && (size_t)warps * k * 8 > 48 * 1024) warps >>= 1;
+  const size_t smem = (size_t)warps * k * (sizeof(float) + sizeof(int32_t));
+  k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, out_ids, out_scores);
   return cudaGetLastError();
 }
 
