@@ -600,6 +600,33 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     }
     float th_s = -INFINITY;
     int th_i = INT_MAX;
+    float ps0 = 0.f, ps1 = 0.f, ps2 = 0.f, ps3 = 0.f;  // parked candidates of the current tile
+    int pi0 = 0, pi1 = 0, pi2 = 0, pi3 = 0, npark = 0;
+    // Inserts (sc, v) into this thread's sorted list if it beats entry
+    // k-1: walk up while the entry above is worse, shifting it down; the
+    // new entry k-1 is the first one shifted, or (sc, v) if nothing moves.
+    auto insert = [&](float sc, int v) {
+      if (!better(sc, v, th_s, th_i)) return;
+      float nts = sc;
+      int nti = v;
+      int pos = k - 1;
+      while (pos > 0) {
+        const float as = ls[(pos - 1) * MMA_M + row];
+        const int ai = li[(pos - 1) * MMA_M + row];
+        if (!better(sc, v, as, ai)) break;
+        ls[pos * MMA_M + row] = as;
+        li[pos * MMA_M + row] = ai;
+        if (pos == k - 1) {
+          nts = as;
+          nti = ai;
+        }
+        --pos;
+      }
+      ls[pos * MMA_M + row] = sc;
+      li[pos * MMA_M + row] = v;
+      th_s = nts;
+      th_i = nti;
+    };
     for (int tile_i = 0; tile_i < my_tiles; ++tile_i) {
       const int t = blockIdx.x + tile_i * gridDim.x;
       const int v0 = t * NT;
@@ -625,7 +652,9 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       if (mine) {
         const uint32_t tb = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)((set * QT + jsel) * NT);
         // one 16-column chunk: scale, flag the scores that may enter the list
-        // (branch-free), then insert the flagged ones (rare after the first tiles)
+        // (branch-free); flagged ones (rare after the first tiles) are parked
+        // in registers and inserted after the accumulator is released, so the
+        // insertions overlap the next tile's MMAs; a full park inserts at once
         auto chunk = [&](uint32_t (&r)[16], int c0) {
           if (q >= nq) return;
           const int valid = min(16, n - (v0 + c0));
@@ -647,7 +676,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
             m |= (y.y >= th_s ? 1u : 0u) << (jj + 3);
           }
           if (valid < 16) m &= valid > 0 ? (1u << valid) - 1u : 0u;
-          while (m) {  // rare after the first tiles; every step stays in registers but one load
+          while (m) {
             const int jj = __ffs(m) - 1;
             m &= m - 1;
             float sc = 0.f;
@@ -655,28 +684,19 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
             for (int t = 0; t < 16; ++t) sc = t == jj ? __uint_as_float(r[t]) : sc;
             const int v = v0 + c0 + jj;
             if (!better(sc, v, th_s, th_i)) continue;
-            // (sc, v) beats entry k-1: walk up while the entry above is worse,
-            // shifting it down; the new entry k-1 is the first one shifted, or
-            // (sc, v) itself if nothing moves
-            float nts = sc;
-            int nti = v;
-            int pos = k - 1;
-            while (pos > 0) {
-              const float as = ls[(pos - 1) * MMA_M + row];
-              const int ai = li[(pos - 1) * MMA_M + row];
-              if (!better(sc, v, as, ai)) break;
-              ls[pos * MMA_M + row] = as;
-              li[pos * MMA_M + row] = ai;
-              if (pos == k - 1) {
-                nts = as;
-                nti = ai;
-              }
-              --pos;
+            if (npark < 4) {
+              ps0 = npark == 0 ? sc : ps0;
+              pi0 = npark == 0 ? v : pi0;
+              ps1 = npark == 1 ? sc : ps1;
+              pi1 = npark == 1 ? v : pi1;
+              ps2 = npark == 2 ? sc : ps2;
+              pi2 = npark == 2 ? v : pi2;
+              ps3 = npark == 3 ? sc : ps3;
+              pi3 = npark == 3 ? v : pi3;
+              ++npark;
+            } else {
+              insert(sc, v);
             }
-            ls[pos * MMA_M + row] = sc;
-            li[pos * MMA_M + row] = v;
-            th_s = nts;
-            th_i = nti;
           }
         };
         // two chunks in flight: the next chunk's TMEM load overlaps this one's work
@@ -696,6 +716,13 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty + set);
+      // the accumulator is free: insert the parked candidates while the next
+      // tile's MMAs run
+      if (npark > 0) insert(ps0, pi0);
+      if (npark > 1) insert(ps1, pi1);
+      if (npark > 2) insert(ps2, pi2);
+      if (npark > 3) insert(ps3, pi3);
+      npark = 0;
       asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
     }
     if (mine && q < nq) {
