@@ -2,7 +2,7 @@
 """Benchmark of the TurboQuant search path on GB300 (one JSON line on stdout).
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--config scale|c2|tiny] [--batches 1,1024] [--k 5]
+                    [--config scale|c2|tiny|filtered|sweep|idmap|prof] [--batches 1,1024] [--k 5]
 
 Workload (default "scale"): N = 999,000 synthetic L2-normalised d = 1536
 vectors (1,024-cluster Gaussian mixture, seed 42), rotated by a seeded Haar R
@@ -54,6 +54,10 @@ CONFIGS = {
     # queries five), 64-vector filter blocks
     "filtered": dict(n=100_000, d=1536, bits=4, clusters=256, pool=1_000, k=10, batches=[1],
                      tenants=[10, 100, 1000], block=64),
+    # id-mapped index: external ids, 1% of the rows deleted; same searches
+    # with and without the id map
+    "idmap": dict(n=999_000, d=1536, bits=4, clusters=1024, pool=2_048, k=5, batches=[1, 1024],
+                  deleted_frac=0.01),
     # bit-width sweep: encode and batch-256 top-10 search at b = 2, 3, 4, 8
     "sweep": dict(n=999_000, d=1536, bits=4, clusters=1024, pool=2_000, k=10, batches=[256],
                   sweep_bits=[2, 3, 4, 8]),
@@ -679,6 +683,71 @@ def run_sweep(args, cfg):
     print(json.dumps(line), flush=True)
 
 
+def run_idmap(args, cfg):
+    """Search over an id-mapped index (external uint64 ids, a share of the
+    rows deleted) against the same search without the id map: the cost of
+    the tombstone checks and the id mapping."""
+    import torch
+    import paper_2607_16973_gb300 as tq
+    from paper_2607_16973_gb300 import synth
+    from paper_2607_16973_gb300.build import build
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    build()
+    tq.load()
+    n, d, bits, k = cfg["n"], cfg["d"], cfg["bits"], args.k or cfg["k"]
+    batches = [int(b) for b in args.batches.split(",")] if args.batches else cfg["batches"]
+    stream = torch.cuda.Stream(device=dev)
+    X, Qpool = make_corpus(cfg, workers=min(16, os.cpu_count() or 4))
+    cen, bnd, _ = tq.codebook(d, bits)
+    R = tq.rotation(d, synth.SEED_ROTATION)
+    Xd = torch.from_numpy(X).to(dev)
+    Rd, cd, bd, Qd = (torch.from_numpy(a).to(dev) for a in (R, cen, bnd, Qpool))
+    codes, scale = tq.encode(Xd, Rd, cd, bd, bits)
+    del Xd, X
+    rng = np.random.default_rng(synth.SEED_QUERIES)
+    ext = rng.choice(1 << 62, size=n, replace=False).astype(np.uint64)
+    gone = rng.choice(n, int(cfg["deleted_frac"] * n), replace=False)
+    m = tq.IdMap(n)
+    m.add(ext, stream=stream)
+    m.remove(ext[gone], stream=stream)
+    torch.cuda.synchronize()
+    variants = {}
+    for B in batches:
+        nb = max(1, len(Qpool) // B)
+        ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
+        ids = torch.empty((B, k), dtype=torch.int64, device=dev)
+        scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+        res = {}
+        for name, im in (("plain", None), ("idmap", m)):
+            with torch.cuda.stream(stream):
+                res[name] = _timed(lambda i: tq.search(Qd[(i % nb) * B:(i % nb) * B + B], Rd, cd, bits, codes, scale,
+                                                       k, workspace=ws, out_ids=ids, out_scores=scs, stream=stream,
+                                                       idmap=im), args.steps, args.warmup, stream)
+        # every returned id is a live external id
+        with torch.cuda.stream(stream):
+            got, _ = tq.search(Qd[:B], Rd, cd, bits, codes, scale, k, stream=stream, idmap=m)
+        stream.synchronize()
+        live = set(np.delete(ext, gone).view(np.int64).tolist())
+        ok = all(v in live for v in got.cpu().numpy().reshape(-1).tolist() if v != -1)
+        variants[str(B)] = {"value": B / res["idmap"] * 1e3, "ms_per_step": res["idmap"],
+                            "plain_value": B / res["plain"] * 1e3, "plain_ms_per_step": res["plain"],
+                            "overhead_frac": res["idmap"] / res["plain"] - 1.0, "results_live": ok}
+        log(f"[bench] idmap B={B}: {B / res['idmap'] * 1e3:.4g} q/s with the id map, "
+            f"{B / res['plain'] * 1e3:.4g} without ({100 * (res['idmap'] / res['plain'] - 1):+.1f}%), "
+            f"results live: {ok}")
+    m.close()
+    head = variants[str(batches[0])]
+    line = {"metric": f"queries/sec at {n // 1000}Kx{d} {bits}-bit top-{k} over an id-mapped index",
+            "value": head["value"], "unit": "queries/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": head["ms_per_step"], "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f32", "data": "synthetic (seeded Gaussian-mixture corpus, random external ids)",
+            "config": {"workload": f"idmap: N={n} d={d} {bits}-bit top-{k}, {cfg['deleted_frac']:.0%} of the rows "
+                                   f"deleted, batches {batches}", "n": n, "d": d, "bits": bits, "k": k},
+            "variants": variants}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -697,9 +766,9 @@ def main():
     if args.impl == "reference":
         run_reference(args, cfg, rank, world)
         return
-    if args.config in ("filtered", "sweep"):
+    if args.config in ("filtered", "sweep", "idmap"):
         if rank == 0:
-            (run_filtered if args.config == "filtered" else run_sweep)(args, cfg)
+            {"filtered": run_filtered, "sweep": run_sweep, "idmap": run_idmap}[args.config](args, cfg)
         return
     if world > 1:
         import torch

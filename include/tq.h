@@ -192,6 +192,71 @@ tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
                     size_t ws_bytes, void* stream);
 
 /*
+ * tq_search_ex - tq_search over an id-mapped index (Sec. III-A: external
+ * uint64 ids, O(1) deletion).  Same arguments and results as tq_search, plus:
+ *   deleted   device [ceil(n/32)] uint32 tombstone bitmap, or NULL: bit i % 32
+ *             of word i / 32 set means row i is deleted and is never returned
+ *             (like a vector whose tenant is not allowed)
+ *   ext_ids   device [n] uint64 external id of each row, or NULL: results are
+ *             written as ext_ids[row] (bit pattern in the int64 out_ids);
+ *             the ranking tie-break stays on the row (insertion order), and
+ *             -1 (all ones) still marks an empty slot, so it must not be used
+ *             as an external id
+ * tq_search(...) is tq_search_ex(..., NULL, NULL, ...).  A tq_idmap handle
+ * (below) keeps both arrays and the id -> row map.
+ */
+tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
+                       const float* centroids, int bits, const uint8_t* codes,
+                       const float* scale, int64_t n, const tq_filter* filter,
+                       const int64_t* allow_off, const uint32_t* allow_tenants,
+                       const uint32_t* deleted, const uint64_t* ext_ids,
+                       int k, int64_t* out_ids, float* out_scores, void* workspace,
+                       size_t ws_bytes, void* stream);
+
+/*
+ * tq_idmap - the id map of an id-mapped index (Sec. III-A): external uint64
+ * ids for rows 0, 1, 2, ... in insertion order, O(1) lookup and deletion.
+ * Library-owned: a host hash map id -> row plus two device arrays sized for
+ * `capacity` rows, the external ids [capacity] uint64 and the tombstone
+ * bitmap [ceil(capacity/32)] uint32 (zero = live), which tq_idmap_device
+ * returns for tq_search_ex.  Rows are never reused: a deleted row stays
+ * tombstoned, and its id may be added again as a new row.  A handle is not
+ * thread-safe: calls on one handle must be serialised by the caller and
+ * queue their copies on one stream (or be synchronised between streams), and
+ * a search that reads the device arrays must be ordered (same stream, or
+ * synchronised) after the add or remove whose effect it should see.  Removal
+ * is O(1) per id on the host plus one copy of the touched bitmap words.
+ *
+ * tq_idmap_create  capacity rows (1..2^31-1) on the current device; device
+ *                  arrays zero-initialised (synchronously).  TQ_ENOMEM if the
+ *                  allocation fails.
+ * tq_idmap_destroy frees everything (NULL is a no-op); the caller makes sure
+ *                  no queued work still reads the device arrays.
+ * tq_idmap_add     appends n_new rows with the given external ids (host array,
+ *                  copied before the call returns); *first_row receives the
+ *                  first new row.  TQ_EINVAL, with nothing changed, if the
+ *                  capacity would be exceeded, an id is -1, or an id is already
+ *                  live (in the map or twice in the batch).
+ * tq_idmap_remove  deletes the rows of the given external ids (host array):
+ *                  each live id leaves the map and its row's tombstone bit is
+ *                  set on the device (stream-ordered); ids that are not live
+ *                  are ignored.  *n_removed (nullable) receives how many were.
+ * tq_idmap_lookup  row of a live external id, or -1.
+ * tq_idmap_info    rows used, capacity, live ids (any pointer may be NULL).
+ * tq_idmap_device  the device arrays (valid until tq_idmap_destroy).
+ */
+typedef struct tq_idmap tq_idmap;
+tq_status tq_idmap_create(int64_t capacity, tq_idmap** out);
+tq_status tq_idmap_destroy(tq_idmap* m);
+tq_status tq_idmap_add(tq_idmap* m, const uint64_t* ext_ids, int64_t n_new, int64_t* first_row,
+                       void* stream);
+tq_status tq_idmap_remove(tq_idmap* m, const uint64_t* ext_ids, int64_t n, int64_t* n_removed,
+                          void* stream);
+tq_status tq_idmap_lookup(const tq_idmap* m, uint64_t ext_id, int64_t* row);
+tq_status tq_idmap_info(const tq_idmap* m, int64_t* rows, int64_t* capacity, int64_t* live);
+tq_status tq_idmap_device(const tq_idmap* m, const uint32_t** deleted, const uint64_t** ext_ids);
+
+/*
  * tq_search_static - tq_search without a workspace, for callers that cannot
  * allocate device memory (for example a C host program or plugin that is
  * handed device pointers for its inputs and outputs but owns no allocator, or

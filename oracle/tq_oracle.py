@@ -12,6 +12,8 @@ numpy/scipy in float64, written step by step from the paper:
   renormalisation scalar;
 * Sec. III-B: allowlist filtering (a vector whose tenant is not allowed never
   enters the top-k);
+* Sec. III-A: the id-mapped index (a deleted row never enters the top-k; rows
+  are reported by their external uint64 ids);
 * Sec. IV-A: exact brute-force inner-product ground truth and Recall@k.
 
 Readings where the paper is silent (each is also listed in the design doc):
@@ -33,7 +35,10 @@ Readings where the paper is silent (each is also listed in the design doc):
   default), "none" = ||x||, "unbiased" = ||x|| / <y, c[code]>;  a zero row has
   y = 0 and scale 0;
 * ranking: score descending, ties by id ascending, taken on float32 scores;
-  fewer than k allowed vectors pad with id -1 and score -inf.
+  fewer than k allowed vectors pad with id -1 and score -inf;
+* id map: deletion excludes a row as a disallowed tenant does; the tie-break
+  stays on the row (insertion order), which is then reported as its external
+  id; the all-ones id (-1) is reserved for empty slots.
 """
 from __future__ import annotations
 
@@ -372,16 +377,27 @@ def quantized_scores(Q, R, centroids, bits, packed, scale, d, row_chunk=16384) -
 
 
 def search(Q, R, centroids, bits, packed, scale, k, d,
-           tenant_ids=None, allow_off=None, allow_ids=None) -> SearchResult:
-    """Top-k inner-product search over the quantised corpus."""
+           tenant_ids=None, allow_off=None, allow_ids=None, deleted=None, ext_ids=None) -> SearchResult:
+    """Top-k inner-product search over the quantised corpus.
+
+    Id-mapped index (Sec. III-A: external uint64 ids, O(1) deletion): a row
+    with deleted[i] True is never returned, exactly like a row whose tenant
+    is not allowed; with ext_ids the k rows, ranked as usual (ties by row,
+    i.e. insertion order), are reported as ext_ids[row] (their int64 bit
+    pattern; empty slots stay -1)."""
     S = quantized_scores(Q, R, centroids, bits, packed, scale, d)
     nq, n = S.shape
     allowed = allowed_mask(tenant_ids, allow_off, allow_ids, nq, n)
+    if deleted is not None:
+        allowed = allowed & ~np.asarray(deleted, dtype=bool)[None, :]
     ids = np.empty((nq, k), dtype=np.int64)
     sc = np.empty((nq, k), dtype=np.float32)
     S32 = S.astype(np.float32)
     for q in range(nq):
         ids[q], sc[q] = rank_topk(S32[q], allowed[q], k)
+    if ext_ids is not None:
+        ext = np.asarray(ext_ids, dtype=np.uint64).view(np.int64)
+        ids = np.where(ids >= 0, ext[np.maximum(ids, 0)], -1)
     return SearchResult(ids=ids, scores=sc, scores64=S)
 
 

@@ -13,7 +13,7 @@ import numpy as np
 
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
-__all__ = ["codebook", "rotation", "encode", "Filter", "search", "search_workspace",
+__all__ = ["codebook", "rotation", "encode", "Filter", "IdMap", "search", "search_workspace",
            "search_from_host", "search_check", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
            "TQError"]
 
@@ -113,6 +113,71 @@ class Filter:
             pass
 
 
+class IdMap:
+    """tq_idmap handle: external uint64 ids of rows 0, 1, ... in insertion
+    order, O(1) lookup and deletion (Sec. III-A).  Pass it to search() as
+    `idmap`: deleted rows are never returned and results come back as
+    external ids (int64 bit patterns; -1 marks an empty slot)."""
+
+    def __init__(self, capacity: int):
+        self._h = C.c_void_p()
+        check(load().tq_idmap_create(int(capacity), C.byref(self._h)))
+
+    @property
+    def handle(self) -> int:
+        return self._h.value or 0
+
+    @staticmethod
+    def _ids(ext_ids) -> np.ndarray:
+        a = np.ascontiguousarray(np.asarray(ext_ids).reshape(-1))
+        if a.dtype == np.int64:
+            a = a.view(np.uint64)
+        return np.ascontiguousarray(a, dtype=np.uint64)
+
+    def add(self, ext_ids, stream=None) -> int:
+        """Appends rows with these external ids; returns the first new row."""
+        a = self._ids(ext_ids)
+        first = C.c_int64()
+        check(load().tq_idmap_add(self._h, a.ctypes.data, a.size, C.byref(first), _stream_handle(stream)))
+        return first.value
+
+    def remove(self, ext_ids, stream=None) -> int:
+        """Deletes the rows of these ids (ids that are not live are ignored);
+        returns how many were removed."""
+        a = self._ids(ext_ids)
+        n = C.c_int64()
+        check(load().tq_idmap_remove(self._h, a.ctypes.data, a.size, C.byref(n), _stream_handle(stream)))
+        return n.value
+
+    def lookup(self, ext_id: int) -> int:
+        """Row of a live external id, or -1."""
+        row = C.c_int64()
+        check(load().tq_idmap_lookup(self._h, C.c_uint64(int(ext_id) & 0xFFFFFFFFFFFFFFFF), C.byref(row)))
+        return row.value
+
+    def info(self):
+        r, c, l = C.c_int64(), C.c_int64(), C.c_int64()
+        check(load().tq_idmap_info(self._h, C.byref(r), C.byref(c), C.byref(l)))
+        return {"rows": r.value, "capacity": c.value, "live": l.value}
+
+    def device(self):
+        """(tombstone bitmap, external ids) device addresses for tq_search_ex."""
+        dd, de = C.c_void_p(), C.c_void_p()
+        check(load().tq_idmap_device(self._h, C.byref(dd), C.byref(de)))
+        return dd.value or 0, de.value or 0
+
+    def close(self) -> None:
+        if self._h and self._h.value:
+            load().tq_idmap_destroy(self._h)
+            self._h = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 def search_workspace(nq: int, n: int, d: int, bits: int, k: int, filter: Filter | None = None) -> int:
     out = C.c_size_t()
     check(load().tq_search_workspace(nq, n, d, bits, k, filter.handle if filter else None, C.byref(out)))
@@ -121,11 +186,18 @@ def search_workspace(nq: int, n: int, d: int, bits: int, k: int, filter: Filter 
 
 def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | None = None,
            allow_off=None, allow_tenants=None, workspace=None, out_ids=None, out_scores=None,
-           stream=None):
-    """tq_search on CUDA tensors: returns (ids int64 [nq, k], scores f32 [nq, k])."""
+           stream=None, idmap: IdMap | None = None):
+    """tq_search (tq_search_ex with an IdMap) on CUDA tensors: returns
+    (ids int64 [nq, k], scores f32 [nq, k]); with an IdMap the ids are
+    external ids and deleted rows are skipped."""
     torch = _torch()
     nq, d = Q.shape
     n = codes.shape[0]
+    deleted = ext = 0
+    if idmap is not None:
+        if idmap.info()["rows"] < n:
+            raise ValueError(f"the id map holds {idmap.info()['rows']} rows, the corpus {n}")
+        deleted, ext = idmap.device()
     dev = Q.device
     if out_ids is None:
         out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
@@ -136,11 +208,12 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
         workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
     f32 = torch.float32
     u32 = (torch.int32, getattr(torch, "uint32", torch.int32))
-    check(load().tq_search(
+    check(load().tq_search_ex(
         _dev_ptr(Q, "Q", f32), nq, d, _dev_ptr(R, "R", f32), _dev_ptr(centroids, "centroids", f32), bits,
         _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), n,
         filter.handle if filter else None, _dev_ptr(allow_off, "allow_off", torch.int64),
-        _dev_ptr(allow_tenants, "allow_tenants", u32), k, _dev_ptr(out_ids, "out_ids", torch.int64),
+        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None, k,
+        _dev_ptr(out_ids, "out_ids", torch.int64),
         _dev_ptr(out_scores, "out_scores", f32), _dev_ptr(workspace, "workspace", contiguous=True),
         workspace.numel() * workspace.element_size(), _stream_handle(stream)))
     return out_ids, out_scores
@@ -148,13 +221,13 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
 
 def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, q_dev, ids_host,
                      scores_host, filter: Filter | None = None, allow_off=None, allow_tenants=None,
-                     workspace=None, out_ids=None, out_scores=None, stream=None):
+                     workspace=None, out_ids=None, out_scores=None, stream=None, idmap: IdMap | None = None):
     """search() for queries in (pinned) host memory: copies Q to q_dev, runs
     tq_search and copies ids/scores back into the host tensors, all queued on
     `stream`."""
     q_dev.copy_(Q_host, non_blocking=True)
     ids, scores = search(q_dev, R, centroids, bits, codes, scale, k, filter, allow_off, allow_tenants,
-                         workspace, out_ids, out_scores, stream)
+                         workspace, out_ids, out_scores, stream, idmap)
     ids_host.copy_(ids, non_blocking=True)
     scores_host.copy_(scores, non_blocking=True)
     return ids_host, scores_host

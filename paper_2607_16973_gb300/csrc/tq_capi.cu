@@ -1,5 +1,5 @@
 // C ABI entry points that queue device work: tq_encode, tq_filter_*,
-// tq_search_workspace, tq_search.  Every argument is validated before any
+// tq_search_workspace, tq_search / tq_search_ex.  Every argument is validated before any
 // work is queued; CUDA errors come back as TQ_ECUDA with the runtime's text.
 #include <cuda_runtime.h>
 
@@ -170,12 +170,13 @@ extern "C" tq_status tq_search_workspace(int64_t nq, int64_t n, int d, int bits,
   return tq::ok();
 }
 
-extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
-                               const float* centroids, int bits, const uint8_t* codes,
-                               const float* scale, int64_t n, const tq_filter* filter,
-                               const int64_t* allow_off, const uint32_t* allow_tenants, int k,
-                               int64_t* out_ids, float* out_scores, void* workspace,
-                               size_t ws_bytes, void* stream) {
+extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
+                                  const float* centroids, int bits, const uint8_t* codes,
+                                  const float* scale, int64_t n, const tq_filter* filter,
+                                  const int64_t* allow_off, const uint32_t* allow_tenants,
+                                  const uint32_t* deleted, const uint64_t* ext_ids, int k,
+                                  int64_t* out_ids, float* out_scores, void* workspace,
+                                  size_t ws_bytes, void* stream) {
   tq_status st = check_search(nq, n, d, bits, k);
   if (st != TQ_OK) return st;
   if (nq == 0) return tq::ok();
@@ -184,8 +185,8 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
   if (!tq::aligned16(Q) || !tq::aligned16(R) || !tq::aligned16(codes) || !tq::aligned16(workspace))
     return fail(TQ_EINVAL, "tq_search: Q, R, codes and workspace must be 16-byte aligned");
   if (((uintptr_t)centroids & 3u) || ((uintptr_t)scale & 3u) || ((uintptr_t)out_scores & 3u) ||
-      ((uintptr_t)out_ids & 7u))
-    return fail(TQ_EINVAL, "tq_search: misaligned centroids/scale/out pointers");
+      ((uintptr_t)out_ids & 7u) || ((uintptr_t)deleted & 3u) || ((uintptr_t)ext_ids & 7u))
+    return fail(TQ_EINVAL, "tq_search: misaligned centroids/scale/out/deleted/ext_ids pointers");
   if (filter) {
     if (filter->f.n != n)
       return fail(TQ_EINVAL, "tq_search: filter built for n=%lld, search has n=%lld",
@@ -214,19 +215,31 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
   cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, s);  // also zeroes the status word
   if (use_mma) {
     if (e == cudaSuccess)
-      e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, k, p.grid_mma, ws + p.off_qpack, cs, ci,
+      e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, deleted, k, p.grid_mma,
+                              ws + p.off_qpack, cs, ci,
                               status, s, (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
-    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, out_ids, out_scores, s);
+    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, ext_ids, out_ids, out_scores, s);
   } else {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
     if (e == cudaSuccess)
-      e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, filter ? &filter->f : nullptr, allow,
+      e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
+                              filter ? &filter->f : nullptr, allow,
                               k, p.grid_lut, cs, ci, s, (cudaEvent_t)tq::profile_start(),
                               (cudaEvent_t)tq::profile_stop());
-    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_lut * k, k, out_ids, out_scores, s);
+    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_lut * k, k, ext_ids, out_ids, out_scores, s);
   }
   if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
   return tq::ok();
+}
+
+extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
+                               const float* centroids, int bits, const uint8_t* codes,
+                               const float* scale, int64_t n, const tq_filter* filter,
+                               const int64_t* allow_off, const uint32_t* allow_tenants, int k,
+                               int64_t* out_ids, float* out_scores, void* workspace,
+                               size_t ws_bytes, void* stream) {
+  return tq_search_ex(Q, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, nullptr,
+                      nullptr, k, out_ids, out_scores, workspace, ws_bytes, stream);
 }
 
 extern "C" tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_scores, int64_t n_src, int64_t nq,

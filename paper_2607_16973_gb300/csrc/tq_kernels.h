@@ -35,16 +35,18 @@ cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
 // Filter build: dense index per vector and per-block tenant bitmaps.
 cudaError_t launch_filter_build(const uint32_t* tenant_ids, FilterDev& f, cudaStream_t s);
 
-// LUT scan: per-CTA top-k candidates [nq][grid_x][k] (score, id).
+// LUT scan: per-CTA top-k candidates [nq][grid_x][k] (score, id).  `del`
+// (nullable) is the tombstone bitmap: rows whose bit is set are skipped.
 int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d);
 cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, const FilterDev* f,
-                            const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
+                            const FilterDev* f, const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
                             int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1);
 
-// Final merge of per-CTA candidates into sorted top-k.
+// Final merge of per-CTA candidates into sorted top-k; with `ext` (nullable)
+// the rows are written as ext[row].
 cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
-                         int k, int64_t* out_ids, float* out_scores, cudaStream_t s);
+                         int k, const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s);
 
 // Merge of S sources x m candidates per query ([S][nq][m]) with global int64
 // ids (-1 = padding).
@@ -56,8 +58,8 @@ bool mma_supported(int bits, int d, int k);
 int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits);
 size_t mma_qpack_bytes(int64_t nq, int d);
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, int k, int grid_x,
-                            void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del, int k,
+                            int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1);
 
 int device_sm_count();

@@ -5,15 +5,17 @@
 // memory (TMEM).  A CTA owns QT (1 or 2) query tiles and a strided set of
 // vector tiles.  With one query tile TMEM holds two accumulator sets, so the
 // epilogue of one vector tile overlaps the MMAs of the next; with two, the
-// next tile's MMAs wait for the epilogue.  Roles (warp-specialised, 19 warps):
-//   warps 0-7   decoders, two groups of four on alternate K-blocks: expand
-//               one K-block (64 coordinates) of packed codes, brought to
-//               shared memory by TMA, into fp16 centroid values laid out as
-//               the K-major, 128-byte-swizzled B operand;
+// next tile's MMAs wait for the epilogue.  Roles (warp-specialised, 23 warps):
+//   warps 0-7, 19-22  decoders, in groups of four warps that take turns on
+//               K-blocks (with one query tile, warps 12-15 are a fourth
+//               group): expand one K-block (64 coordinates) of packed codes,
+//               brought to shared memory by TMA, into fp16 centroid values
+//               laid out as the K-major, 128-byte-swizzled B operand;
 //   warps 8-15  epilogue: read the 128 x 256 fp32 accumulators from TMEM (one
 //               query per thread; warps 8-11 the first query tile, 12-15 the
 //               second), apply the per-vector scale and keep each query's
-//               top-k in a thread-private sorted list;
+//               top-k in a thread-private sorted list (rows marked in the
+//               optional tombstone bitmap never enter it);
 //   warp 16     code producer: TMA of the code tiles; allocates TMEM;
 //   warp 17     MMA issuer: one thread issues tcgen05.mma (M=128, N=256,
 //               K=16) and commits completion to mbarriers;
@@ -347,7 +349,8 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
 template <int BITS, int QT>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,
-           const float* __restrict__ centroids, const float* __restrict__ scale, int n, int nq, int d,
+           const float* __restrict__ centroids, const float* __restrict__ scale,
+           const uint32_t* __restrict__ del, int n, int nq, int d,
            int k, int cst, int ast, int rr, int sub, int ng, int gact, float* __restrict__ cand_s,
            int* __restrict__ cand_i, int* __restrict__ err) {
   constexpr int RAWB = raw_bytes_per_row<BITS>();
@@ -684,6 +687,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
             for (int t = 0; t < 16; ++t) sc = t == jj ? __uint_as_float(r[t]) : sc;
             const int v = v0 + c0 + jj;
             if (!better(sc, v, th_s, th_i)) continue;
+            if (del && ((__ldg(del + (v >> 5)) >> (v & 31)) & 1u)) continue;  // deleted row
             if (npark < 4) {
               ps0 = npark == 0 ? sc : ps0;
               pi0 = npark == 0 ? v : pi0;
@@ -777,14 +781,14 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
 
 template <int BITS, int QT>
 cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half* qpack, const float* centroids,
-                         const float* scale, int n, int nq, int d, int k, int sub, int grid_x, float* cs,
-                         int* ci, int* err, cudaStream_t s) {
+                         const float* scale, const uint32_t* del, int n, int nq, int d, int k, int sub,
+                         int grid_x, float* cs, int* ci, int* err, cudaStream_t s) {
   const int gact = active_groups(P.ng, sub, P.cst);
   cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_mma<BITS, QT>), (int)P.smem);
   if (e != cudaSuccess) return e;
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));
-  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, n, nq, d, k, P.cst, P.ast,
+  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, del, n, nq, d, k, P.cst, P.ast,
                                                          P.rr, sub, P.ng, gact, cs, ci, err);
   return cudaGetLastError();
 }
@@ -816,8 +820,8 @@ size_t mma_qpack_bytes(int64_t nq, int d) {
 }
 
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, int k, int grid_x,
-                            void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del, int k,
+                            int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
   PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
@@ -845,12 +849,12 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   if (e != cudaSuccess) return e;
   if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;
   const __half* qp = static_cast<const __half*>(qpack);
-#define TQ_MMA_CASE(B)                                                                                        \
-  case B:                                                                                                     \
-    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, (int)n, (int)nq, d, k, sub, grid_x,      \
-                                       cand_s, cand_i, err, s)                                                \
-                  : launch_typed<B, 1>(P, map, qp, centroids, scale, (int)n, (int)nq, d, k, sub, grid_x,      \
-                                       cand_s, cand_i, err, s);                                               \
+#define TQ_MMA_CASE(B)                                                                                \
+  case B:                                                                                             \
+    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, del, (int)n, (int)nq, d, k, sub, \
+                                       grid_x, cand_s, cand_i, err, s)                                \
+                  : launch_typed<B, 1>(P, map, qp, centroids, scale, del, (int)n, (int)nq, d, k, sub, \
+                                       grid_x, cand_s, cand_i, err, s);                               \
     break;
   switch (bits) {
     TQ_MMA_CASE(2)

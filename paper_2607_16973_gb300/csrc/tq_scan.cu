@@ -12,7 +12,9 @@
 //
 // Top-k: each warp keeps a sorted list of its k best (score desc, id asc) in
 // shared memory, entered only when a score beats the list's k-th entry; a
-// disallowed vector never enters (Sec. III-B: dropped at heap insert).  Blocks
+// disallowed vector never enters (Sec. III-B: dropped at heap insert), and
+// neither does a deleted one (its bit set in the caller's tombstone bitmap,
+// the O(1) deletion of the id-mapped index of Sec. III-A).  Blocks
 // of `block` vectors whose tenant bitmap shares no bit with the query's allow
 // bitmap are skipped before any code byte is read (Sec. III-B).
 #include <cuda_runtime.h>
@@ -29,6 +31,13 @@ namespace tq {
 namespace {
 
 constexpr unsigned FULL = 0xffffffffu;
+
+// Bit v % 32 of word v / 32 of the tombstone bitmap marks row v deleted.  It
+// is read only for a vector that would enter a list, so a scan with few
+// candidates per step pays almost nothing for it.
+__device__ __forceinline__ bool tombstoned(const uint32_t* __restrict__ del, int v) {
+  return del && ((__ldg(del + (v >> 5)) >> (v & 31)) & 1u);
+}
 constexpr int SCAN_NT = 256;
 constexpr int SCAN_WARPS = SCAN_NT / 32;
 constexpr int MERGE_P = 2048;
@@ -236,6 +245,7 @@ template <int BITS, int S>
 __global__ void __launch_bounds__(SCAN_NT, 2)
 k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
            const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+           const uint32_t* __restrict__ del,
            const uint32_t* __restrict__ dense, const uint32_t* __restrict__ block_bits, int words,
            int fblock, const uint32_t* __restrict__ allow_bits, int k, int P,
            float* __restrict__ cand_s, int* __restrict__ cand_i) {
@@ -335,7 +345,7 @@ k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ cent
     if ((lane & 3) == 0 && vm < n) {
       score = total * sc_my;
       const bool allowed = !ab || ((__ldg(ab + (ten_my >> 5)) >> (ten_my & 31)) & 1u);
-      cand = allowed && better(score, vm, th_s, th_i);
+      cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
     unsigned m = __ballot_sync(FULL, cand);
     while (m) {  // in vector order; re-checked against the moving threshold
@@ -387,7 +397,8 @@ __device__ __forceinline__ float warp_sum4(float (&p)[4]) {
 template <int BITS, int S>
 __global__ void __launch_bounds__(SCAN_NT, 2)
 k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
-                  const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n, int k, int P,
+                  const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+                  const uint32_t* __restrict__ del, int k, int P,
                   float* __restrict__ cand_s, int* __restrict__ cand_i) {
   constexpr int L = 1 << BITS;
   constexpr int CB = 2 * BITS;
@@ -466,7 +477,7 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
       score = total * sc_cur;
-      cand = better(score, vm, th_s, th_i);
+      cand = better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
     unsigned m = __ballot_sync(FULL, cand);
     while (m) {  // in vector order; re-checked against the moving threshold
@@ -503,7 +514,8 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
 template <int S>
 __global__ void __launch_bounds__(SCAN_NT, 2)
 k_scan_pair_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
-                   const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n, int k, int P,
+                   const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+                   const uint32_t* __restrict__ del, int k, int P,
                    float* __restrict__ cand_s, int* __restrict__ cand_i) {
   constexpr int V = 4;
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -566,7 +578,7 @@ k_scan_pair_stream(const float* __restrict__ qrot, int d, const float* __restric
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
       score = total * sc_cur;
-      cand = better(score, vm, th_s, th_i);
+      cand = better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
     unsigned m = __ballot_sync(FULL, cand);
     while (m) {
@@ -650,10 +662,11 @@ k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t 
 // skipped at once.  Each warp keeps a sorted top-k of its share of the rest
 // (ballot, then one warp-wide insertion per candidate that still beats the
 // warp's k-th); warp 0 then folds the sorted warp lists into the result,
-// leaving each list at its first entry that no longer qualifies.
+// leaving each list at its first entry that no longer qualifies.  With an
+// id map the result rows are written as their external ids.
 __global__ void __launch_bounds__(1024)
 k_merge_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k,
-              int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+              const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int nwarps = blockDim.x >> 5;
   float* ws = reinterpret_cast<float*>(smem_raw);  // [nwarps][k]
@@ -750,7 +763,7 @@ k_merge_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, 
     }
     for (int i = lane; i < k; i += 32) {
       const bool empty = li[i] == INT_MAX;
-      out_ids[q * k + i] = empty ? -1 : (int64_t)li[i];
+      out_ids[q * k + i] = empty ? -1 : ext ? (int64_t)__ldg(ext + li[i]) : (int64_t)li[i];
       out_scores[q * k + i] = empty ? -INFINITY : ls[i];
     }
   }
@@ -799,26 +812,26 @@ int next_pow2(int x) {
 template <int BITS, int S>
 cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
                            const float* centroids, const uint8_t* codes, const float* scale, int n,
-                           const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
+                           const uint32_t* del, const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
                            const uint32_t* allow, int k, int P, float* cs, int* ci) {
   cudaError_t e;
   if (BITS == 4 && !allow) {
     const size_t psmem = (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int));
     e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_pair_stream<S>), (int)psmem);
     if (e != cudaSuccess) return e;
-    k_scan_pair_stream<S><<<grid, SCAN_NT, psmem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
+    k_scan_pair_stream<S><<<grid, SCAN_NT, psmem, s>>>(qrot, d, centroids, codes, scale, n, del, k, P, cs, ci);
     return cudaGetLastError();
   }
   if (!allow) {
     e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut_stream<BITS, S>), (int)smem);
     if (e != cudaSuccess) return e;
-    k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, k, P, cs, ci);
+    k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, del, k, P, cs, ci);
     return cudaGetLastError();
   }
   const size_t fsmem = BITS == 4 ? (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int)) : smem;
   e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut<BITS, S>), (int)fsmem);
   if (e != cudaSuccess) return e;
-  k_scan_lut<BITS, S><<<grid, SCAN_NT, fsmem, s>>>(qrot, d, centroids, codes, scale, n, dense, block_bits,
+  k_scan_lut<BITS, S><<<grid, SCAN_NT, fsmem, s>>>(qrot, d, centroids, codes, scale, n, del, dense, block_bits,
                                                    words, fblock, allow, k, P, cs, ci);
   return cudaGetLastError();
 }
@@ -826,13 +839,13 @@ cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* 
 template <int BITS>
 cudaError_t scan_lut_bits(int S, dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
                           const float* centroids, const uint8_t* codes, const float* scale, int n,
-                          const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
+                          const uint32_t* del, const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
                           const uint32_t* allow, int k, int P, float* cs, int* ci) {
   switch (S) {
-    case 1: return scan_lut_typed<BITS, 1>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 2: return scan_lut_typed<BITS, 2>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 3: return scan_lut_typed<BITS, 3>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 4: return scan_lut_typed<BITS, 4>(grid, smem, s, qrot, d, centroids, codes, scale, n, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 1: return scan_lut_typed<BITS, 1>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 2: return scan_lut_typed<BITS, 2>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 3: return scan_lut_typed<BITS, 3>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 4: return scan_lut_typed<BITS, 4>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -853,8 +866,8 @@ int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d) {
 }
 
 cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, const FilterDev* f,
-                            const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
+                            const FilterDev* f, const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
                             int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
   const int S = (d + 511) / 512;
@@ -868,10 +881,10 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
   cudaError_t e;
   if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;
   switch (bits) {
-    case 2: e = scan_lut_bits<2>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 3: e = scan_lut_bits<3>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 4: e = scan_lut_bits<4>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 8: e = scan_lut_bits<8>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 2: e = scan_lut_bits<2>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 3: e = scan_lut_bits<3>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 4: e = scan_lut_bits<4>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 8: e = scan_lut_bits<8>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
     default: e = cudaErrorInvalidValue;
   }
   if (e != cudaSuccess) return e;
@@ -880,7 +893,7 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
 }
 
 cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq, int per_query,
-                         int k, int64_t* out_ids, float* out_scores, cudaStream_t s) {
+                         int k, const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   // per_query = grid_x * k: one sorted list of k per scan CTA
   // up to 32 warps, fewer for long lists (each warp keeps k entries in shared memory)
@@ -888,7 +901,7 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
   int warps = std::max(1, std::min(32, (nlists + 31) / 32));
   while (warps > 1 && (size_t)warps * k * 8 > 48 * 1024) warps >>= 1;
   const size_t smem = (size_t)warps * k * (sizeof(float) + sizeof(int32_t));
-  k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, out_ids, out_scores);
+  k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, ext, out_ids, out_scores);
   return cudaGetLastError();
 }
 

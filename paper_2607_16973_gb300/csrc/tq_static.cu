@@ -113,9 +113,9 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
   e = tq::launch_rotate(Q, nq, d, R, qrot, nullptr, s);
   if (e == cudaSuccess && f) e = tq::launch_allow_bits(*f, allow_off, allow_tenants, nq, allow_bits, s);
   if (e == cudaSuccess)
-    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, f, allow_bits, k, gx, cand_s, cand_i, s,
-                            nullptr, nullptr);
-  if (e == cudaSuccess) e = tq::launch_merge(cand_s, cand_i, nq, gx * k, k, out_ids, out_scores, s);
+    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, nullptr, f, allow_bits, k, gx, cand_s,
+                            cand_i, s, nullptr, nullptr);
+  if (e == cudaSuccess) e = tq::launch_merge(cand_s, cand_i, nq, gx * k, k, nullptr, out_ids, out_scores, s);
   if (e != cudaSuccess) return fail(TQ_ECUDA, "tq_search_static: %s", cudaGetErrorString(e));
   return tq::ok();
 }

@@ -121,6 +121,25 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert search(codes=p + 8) == _lib.TQ_EINVAL
     assert search(ws=null) == _lib.TQ_EINVAL
     assert search(nq=0) == _lib.TQ_OK
+    # search over an id map: misaligned tombstone bitmap / external ids
+    ex = list(args[:12]) + [p + 2, null] + list(args[12:])
+    assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
+    ex[12], ex[13] = null, p + 4
+    assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
+    ex[13], ex[14] = null, 0
+    assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
+    # id map: capacity, NULL handle / ids (no device memory is touched)
+    m = C.c_void_p()
+    assert lib.tq_idmap_create(0, C.byref(m)) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_create(1 << 31, C.byref(m)) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_create(10, null) == _lib.TQ_EINVAL
+    r = C.c_int64()
+    assert lib.tq_idmap_add(null, p, 1, C.byref(r), null) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_remove(null, p, 1, C.byref(r), null) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_lookup(null, 5, C.byref(r)) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_info(null, null, null, null) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_device(null, null, null) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_destroy(null) == _lib.TQ_OK
     # filter
     h = C.c_void_p()
     assert lib.tq_filter_build(p, 10, 48, C.byref(h), null) == _lib.TQ_EINVAL

@@ -456,3 +456,59 @@ def test_exact_knn_and_recall_definitions():
     wrong = ids.copy()
     wrong[:, -1] = -1
     assert O.recall_at_k(wrong, ids) == pytest.approx(4 / 5)
+
+
+# ------------------------------------------------------- id-mapped index -----
+def test_deleted_rows_brute_force_tiny():
+    """Sec. III-A: a deleted row is never returned; results carry the rows'
+    external ids.  Checked against the pure-Python definition with the
+    deleted rows left out and a dict from row to external id."""
+    d, n, k, bits = 32, 50, 6, 2
+    X = synth.mixture_corpus(n, d, 4, seed=31)
+    R = O.rotation(d, 5).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    Q = synth.perturb(X[[2, 17, 40]], seed=8)
+    rng = np.random.default_rng(3)
+    deleted = rng.random(n) < 0.3
+    deleted[[2, 17]] = True  # the queries' own sources
+    ext = rng.choice(1 << 40, size=n, replace=False).astype(np.uint64) | np.uint64(1 << 63)
+    res = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, k, d, deleted=deleted, ext_ids=ext)
+    want = _brute_force_topk(Q, R, cb.centroids32, bits, enc.packed, enc.scale, d, k, allowed=~deleted)
+    to_ext = {v: int(ext[v]) - (1 << 64) for v in range(n)}  # the int64 bit pattern (high bit set)
+    assert res.ids.tolist() == [[to_ext[v] for v in row] for row in want]
+    assert np.all(res.ids < 0)  # every external id here has the high bit set
+
+
+def test_deleted_rows_equal_subset_search(tenant_index):
+    """Deleting rows returns what searching only the live rows returns, with
+    ids mapped back; combined with a tenant filter too."""
+    X, R, cb, enc, tid, values, src, Q, d, bits = tenant_index
+    n = len(X)
+    deleted = np.zeros(n, dtype=bool)
+    deleted[np.random.default_rng(9).choice(n, n // 4, replace=False)] = True
+    deleted[src[:6]] = True
+    off, ids = synth.allowlists(src, tid, values, frac_multi=0.0)
+    for filt in (False, True):
+        kw = dict(tenant_ids=tid, allow_off=off, allow_ids=ids) if filt else {}
+        got = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d, deleted=deleted, **kw)
+        for q in range(len(Q)):
+            keep = np.nonzero(~deleted & (tid == ids[off[q]] if filt else True))[0]
+            sub = O.search(Q[q:q + 1], R, cb.centroids32, bits, enc.packed[keep], enc.scale[keep], 10, d)
+            g = sub.ids[0]
+            assert np.array_equal(np.where(g >= 0, keep[np.maximum(g, 0)], -1), got.ids[q])
+
+
+def test_delete_all_pads_and_ext_ties_follow_rows():
+    d, bits = 32, 2
+    X = synth.mixture_corpus(10, d, 2, seed=1)
+    X = np.concatenate([X, X[[3, 3]]])  # rows 3, 10, 11 tie
+    R = O.rotation(d, 2).astype(np.float32)
+    cb = O.codebook(d, bits)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits)
+    ext = np.arange(100, 88, -1, dtype=np.uint64)  # external ids decrease with the row
+    res = O.search(X[[3]], R, cb.centroids32, bits, enc.packed, enc.scale, 3, d, ext_ids=ext)
+    assert res.ids[0].tolist() == [97, 90, 89]  # rows 3, 10, 11: the tie keeps row order
+    gone = O.search(X[[3]], R, cb.centroids32, bits, enc.packed, enc.scale, 3, d,
+                    deleted=np.ones(12, bool), ext_ids=ext)
+    assert np.all(gone.ids == -1) and np.all(np.isneginf(gone.scores))
