@@ -143,6 +143,21 @@ tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
 tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int block,
                           tq_filter** out, void* stream);
 
+/*
+ * tq_filter_append - online ingest for the filter (Sec. III-A: indexes take
+ * new vectors without a rebuild): rows n .. n+n_new-1 of the corpus get the
+ * tenants tenant_ids[0 .. n_new-1] (device uint32 [n_new]).  When every
+ * tenant is already known the new rows' dense indices and block bits are
+ * written in place (a block shared with earlier rows keeps their bits), the
+ * arrays doubling when full; a tenant the filter has not seen changes the
+ * sorted tenant list, so the filter is rebuilt from all rows.  Either way the
+ * result equals tq_filter_build over all n+n_new rows.  Synchronises
+ * `stream`; on failure the filter is unchanged.  The caller ensures no queued
+ * search still uses the handle.
+ */
+tq_status tq_filter_append(tq_filter* filter, const uint32_t* tenant_ids, int64_t n_new,
+                           void* stream);
+
 /* Frees a handle from tq_filter_build (NULL is a no-op).  The caller ensures
  * no queued search still uses it. */
 tq_status tq_filter_destroy(tq_filter* filter);
@@ -244,6 +259,13 @@ tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
  * tq_idmap_lookup  row of a live external id, or -1.
  * tq_idmap_info    rows used, capacity, live ids (any pointer may be NULL).
  * tq_idmap_device  the device arrays (valid until tq_idmap_destroy).
+ * tq_idmap_export  host copies of the rows' external ids (host [rows] uint64)
+ *                  and the tombstone bitmap (host [ceil(rows/32)] uint32), for
+ *                  persistence; reads only host state.
+ * tq_idmap_import  fills an empty map with n rows from such copies (host
+ *                  arrays; the live ids must be distinct and not -1; no bit
+ *                  past row n may be set); the device copies are queued on
+ *                  `stream`.  TQ_EINVAL, with the map left empty, otherwise.
  */
 typedef struct tq_idmap tq_idmap;
 tq_status tq_idmap_create(int64_t capacity, tq_idmap** out);
@@ -255,6 +277,9 @@ tq_status tq_idmap_remove(tq_idmap* m, const uint64_t* ext_ids, int64_t n, int64
 tq_status tq_idmap_lookup(const tq_idmap* m, uint64_t ext_id, int64_t* row);
 tq_status tq_idmap_info(const tq_idmap* m, int64_t* rows, int64_t* capacity, int64_t* live);
 tq_status tq_idmap_device(const tq_idmap* m, const uint32_t** deleted, const uint64_t** ext_ids);
+tq_status tq_idmap_export(const tq_idmap* m, uint64_t* ext_ids, uint32_t* deleted);
+tq_status tq_idmap_import(tq_idmap* m, const uint64_t* ext_ids, const uint32_t* deleted, int64_t n,
+                          void* stream);
 
 /*
  * tq_search_static - tq_search without a workspace, for callers that cannot

@@ -13,7 +13,7 @@ import numpy as np
 
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
-__all__ = ["codebook", "rotation", "encode", "Filter", "IdMap", "search", "search_workspace",
+__all__ = ["codebook", "rotation", "encode", "Filter", "IdMap", "Index", "search", "search_workspace",
            "search_from_host", "search_check", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
            "TQError"]
 
@@ -96,6 +96,12 @@ class Filter:
     def handle(self) -> int:
         return self._h.value or 0
 
+    def append(self, tenant_ids, stream=None) -> None:
+        """tq_filter_append: tenants of the rows added after the current ones."""
+        torch = _torch()
+        ptr = _dev_ptr(tenant_ids, "tenant_ids", (torch.int32, getattr(torch, "uint32", torch.int32)))
+        check(load().tq_filter_append(self._h, ptr, tenant_ids.numel(), _stream_handle(stream)))
+
     def info(self):
         n, b, t = C.c_int64(), C.c_int(), C.c_int64()
         check(load().tq_filter_info(self._h, C.byref(n), C.byref(b), C.byref(t)))
@@ -165,6 +171,23 @@ class IdMap:
         dd, de = C.c_void_p(), C.c_void_p()
         check(load().tq_idmap_device(self._h, C.byref(dd), C.byref(de)))
         return dd.value or 0, de.value or 0
+
+    def export(self):
+        """(external ids uint64 [rows], tombstone bitmap uint32 [ceil(rows/32)])
+        as host arrays."""
+        rows = self.info()["rows"]
+        ext = np.zeros(rows, np.uint64)
+        dead = np.zeros((rows + 31) // 32, np.uint32)
+        check(load().tq_idmap_export(self._h, ext.ctypes.data, dead.ctypes.data))
+        return ext, dead
+
+    def import_(self, ext_ids, deleted, stream=None) -> None:
+        """Fills this (empty) map from export()'s arrays."""
+        ext = self._ids(ext_ids)
+        dead = np.ascontiguousarray(deleted, dtype=np.uint32)
+        if dead.size != (ext.size + 31) // 32:
+            raise ValueError("the tombstone bitmap needs ceil(rows/32) words")
+        check(load().tq_idmap_import(self._h, ext.ctypes.data, dead.ctypes.data, ext.size, _stream_handle(stream)))
 
     def close(self) -> None:
         if self._h and self._h.value:
@@ -278,3 +301,6 @@ def profile_events(start=None, stop=None) -> None:
             ev.record()
         handles.append(int(ev.cuda_event))
     check(load().tq_profile_events(*handles))
+
+
+from .index import Index  # noqa: E402  (index.py builds on the calls above)

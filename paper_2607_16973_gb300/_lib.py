@@ -23,6 +23,7 @@ SIGNATURES = {
     "tq_encode": (C.c_int, [C.c_void_p, C.c_int64, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p,
                             C.c_int, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]),
     "tq_filter_build": (C.c_int, [C.c_void_p, C.c_int64, C.c_int, C.POINTER(C.c_void_p), C.c_void_p]),
+    "tq_filter_append": (C.c_int, [C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p]),
     "tq_filter_destroy": (C.c_int, [C.c_void_p]),
     "tq_filter_info": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int),
                                  C.POINTER(C.c_int64)]),
@@ -42,6 +43,8 @@ SIGNATURES = {
     "tq_idmap_lookup": (C.c_int, [C.c_void_p, C.c_uint64, C.POINTER(C.c_int64)]),
     "tq_idmap_info": (C.c_int, [C.c_void_p, C.POINTER(C.c_int64), C.POINTER(C.c_int64), C.POINTER(C.c_int64)]),
     "tq_idmap_device": (C.c_int, [C.c_void_p, C.POINTER(C.c_void_p), C.POINTER(C.c_void_p)]),
+    "tq_idmap_export": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "tq_idmap_import": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p]),
     "tq_search_static": (C.c_int, [C.c_void_p, C.c_int64, C.c_int, C.c_void_p, C.c_void_p, C.c_int,
                                    C.c_void_p, C.c_void_p, C.c_int64, C.c_void_p, C.c_void_p,
                                    C.c_void_p, C.c_int, C.c_void_p, C.c_void_p, C.c_void_p]),

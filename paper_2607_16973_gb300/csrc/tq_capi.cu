@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <iterator>
 #include <cstring>
 #include <new>
 #include <vector>
@@ -102,6 +103,7 @@ extern "C" tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int 
     ids.erase(std::unique(ids.begin(), ids.end()), ids.end());
     h = new tq_filter();
     cudaGetDevice(&h->device);
+    h->cap = n;
     tq::FilterDev& f = h->f;
     f.n = n;
     f.block = block;
@@ -124,11 +126,114 @@ extern "C" tq_status tq_filter_build(const uint32_t* tenant_ids, int64_t n, int 
       tq_filter_destroy(h);
       return tq::cuda_fail("tq_filter_build", e);
     }
+    h->tenants_host = std::move(ids);
     *out = h;
     return tq::ok();
   } catch (const std::bad_alloc&) {
     if (h) tq_filter_destroy(h);
     return fail(TQ_ENOMEM, "tq_filter_build: out of host memory");
+  }
+}
+
+// Appends rows to a filter.  Rows whose tenants the filter already knows are
+// added in place: their dense indices and block bits are written, and the
+// arrays grow (doubling) when they are full.  A new tenant changes the sorted
+// tenant list and with it every dense index and the bitmap width, so then the
+// filter is rebuilt from all rows' raw ids.  The old arrays stay in place
+// until the new ones are complete, so a failure leaves the filter unchanged.
+extern "C" tq_status tq_filter_append(tq_filter* h, const uint32_t* tenant_ids, int64_t n_new, void* stream) {
+  if (!h) return fail(TQ_EINVAL, "tq_filter_append: NULL filter");
+  if (n_new < 0 || n_new > INT32_MAX - h->f.n)
+    return fail(TQ_EINVAL, "tq_filter_append: %lld rows + %lld new outside [0, 2^31-1]", (long long)h->f.n,
+                (long long)n_new);
+  if (n_new == 0) return tq::ok();
+  if (!tenant_ids) return fail(TQ_EINVAL, "tq_filter_append: NULL tenant_ids");
+  cudaStream_t s = (cudaStream_t)stream;
+  tq::FilterDev& f = h->f;
+  const int64_t n_total = f.n + n_new;
+  uint32_t *dense = nullptr, *bits = nullptr, *tenants = nullptr, *raw = nullptr;
+  auto release = [&] {
+    cudaFree(dense);
+    cudaFree(bits);
+    cudaFree(tenants);
+    cudaFree(raw);
+  };
+  try {
+    std::vector<uint32_t> ids((size_t)n_new);
+    cudaError_t e = cudaMemcpyAsync(ids.data(), tenant_ids, (size_t)n_new * sizeof(uint32_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return tq::cuda_fail("tq_filter_append: reading tenant ids", e);
+    std::sort(ids.begin(), ids.end());
+    ids.erase(std::unique(ids.begin(), ids.end()), ids.end());
+    std::vector<uint32_t> merged;
+    std::set_union(h->tenants_host.begin(), h->tenants_host.end(), ids.begin(), ids.end(),
+                   std::back_inserter(merged));
+    const bool same_tenants = merged.size() == h->tenants_host.size();
+    const int64_t cap = n_total <= h->cap ? h->cap : std::min<int64_t>(INT32_MAX, std::max(n_total, 2 * h->cap));
+    const int words = same_tenants ? f.words : (int)((merged.size() + 31) / 32);
+    const int64_t cap_blocks = (cap + f.block - 1) / f.block;
+    if (same_tenants && cap == h->cap) {  // room left: write the new rows in place
+      e = tq::launch_filter_extend(tenant_ids, n_new, f, s);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+      if (e != cudaSuccess) return tq::cuda_fail("tq_filter_append", e);
+      f.n = n_total;
+      return tq::ok();
+    }
+    e = tq::dev_malloc(reinterpret_cast<void**>(&dense), (size_t)cap * sizeof(uint32_t));
+    if (e == cudaSuccess) e = tq::dev_malloc(reinterpret_cast<void**>(&bits), (size_t)cap_blocks * words * 4);
+    if (e == cudaSuccess && !same_tenants)
+      e = tq::dev_malloc(reinterpret_cast<void**>(&tenants), merged.size() * sizeof(uint32_t));
+    if (e == cudaSuccess && !same_tenants)
+      e = tq::dev_malloc(reinterpret_cast<void**>(&raw), (size_t)n_total * sizeof(uint32_t));
+    if (e != cudaSuccess) {
+      release();
+      cudaGetLastError();
+      return fail(TQ_ENOMEM, "tq_filter_append: device allocation failed: %s", cudaGetErrorString(e));
+    }
+    e = cudaMemsetAsync(bits, 0, (size_t)cap_blocks * words * 4, s);
+    tq::FilterDev g = f;  // the grown (or rebuilt) filter
+    g.dense = dense;
+    g.block_bits = bits;
+    if (same_tenants) {  // grow: copy the old rows' arrays, then add the new rows
+      const int64_t old_blocks = (f.n + f.block - 1) / f.block;
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(dense, f.dense, (size_t)f.n * sizeof(uint32_t), cudaMemcpyDeviceToDevice, s);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(bits, f.block_bits, (size_t)old_blocks * words * 4, cudaMemcpyDeviceToDevice, s);
+      if (e == cudaSuccess) e = tq::launch_filter_extend(tenant_ids, n_new, g, s);
+    } else {  // rebuild from every row's raw id
+      g.tenants = tenants;
+      g.n_tenants = (int64_t)merged.size();
+      g.words = words;
+      g.n = n_total;
+      if (e == cudaSuccess) e = tq::launch_filter_raw_ids(f, raw, s);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(raw + f.n, tenant_ids, (size_t)n_new * sizeof(uint32_t), cudaMemcpyDeviceToDevice, s);
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(tenants, merged.data(), merged.size() * sizeof(uint32_t), cudaMemcpyHostToDevice, s);
+      if (e == cudaSuccess) e = tq::launch_filter_build(raw, g, s);
+    }
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);  // `merged` is freed on return
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(s);
+      release();
+      return tq::cuda_fail("tq_filter_append", e);
+    }
+    cudaFree(raw);
+    cudaFree(f.dense);
+    cudaFree(f.block_bits);
+    if (!same_tenants) {
+      cudaFree(f.tenants);
+      h->tenants_host = std::move(merged);
+    }
+    g.n = n_total;
+    f = g;
+    h->cap = cap;
+    return tq::ok();
+  } catch (const std::bad_alloc&) {
+    cudaStreamSynchronize(s);
+    release();
+    return fail(TQ_ENOMEM, "tq_filter_append: out of host memory");
   }
 }
 

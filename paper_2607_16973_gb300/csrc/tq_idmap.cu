@@ -6,6 +6,7 @@
 // order and never reused.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdint>
 #include <new>
 #include <unordered_map>
@@ -19,7 +20,7 @@ struct tq_idmap {
   int64_t capacity = 0, rows = 0;
   std::unordered_map<uint64_t, int64_t> live;  // external id -> row, live rows only
   std::vector<uint32_t> dead;                  // host copy of the tombstone bitmap
-  std::vector<uint64_t> staging;               // pageable copy of the ids being added
+  std::vector<uint64_t> ext;                   // host copy of the external ids, [rows]
   uint64_t* d_ext = nullptr;                   // [capacity]
   uint32_t* d_dead = nullptr;                  // [ceil(capacity / 32)]
 };
@@ -100,9 +101,9 @@ extern "C" tq_status tq_idmap_add(tq_idmap* m, const uint64_t* ext_ids, int64_t 
                     (unsigned long long)id);
       }
     }
-    // a pageable copy: cudaMemcpyAsync has read it when it returns, so the
-    // caller's array (pinned or not) is free as soon as this call returns
-    m->staging.assign(ext_ids, ext_ids + n_new);
+    // the host copy is pageable: cudaMemcpyAsync has read it when it returns,
+    // so the caller's array (pinned or not) is free as soon as this call returns
+    m->ext.insert(m->ext.end(), ext_ids, ext_ids + n_new);
   } catch (const std::bad_alloc&) {
     for (int64_t j = 0; j < n_new; ++j) {
       auto it = m->live.find(ext_ids[j]);
@@ -110,10 +111,11 @@ extern "C" tq_status tq_idmap_add(tq_idmap* m, const uint64_t* ext_ids, int64_t 
     }
     return fail(TQ_ENOMEM, "tq_idmap_add: out of host memory");
   }
-  const cudaError_t e = cudaMemcpyAsync(m->d_ext + m->rows, m->staging.data(), (size_t)n_new * sizeof(uint64_t),
+  const cudaError_t e = cudaMemcpyAsync(m->d_ext + m->rows, m->ext.data() + m->rows, (size_t)n_new * sizeof(uint64_t),
                                         cudaMemcpyHostToDevice, (cudaStream_t)stream);
   if (e != cudaSuccess) {
     for (int64_t j = 0; j < n_new; ++j) m->live.erase(ext_ids[j]);
+    m->ext.resize((size_t)m->rows);
     return cuda_fail("tq_idmap_add", e);
   }
   m->rows += n_new;
@@ -165,5 +167,55 @@ extern "C" tq_status tq_idmap_device(const tq_idmap* m, const uint32_t** deleted
   if (!m) return fail(TQ_EINVAL, "tq_idmap_device: NULL map");
   if (deleted) *deleted = m->d_dead;
   if (ext_ids) *ext_ids = m->d_ext;
+  return tq::ok();
+}
+
+extern "C" tq_status tq_idmap_export(const tq_idmap* m, uint64_t* ext_ids, uint32_t* deleted) {
+  if (!m) return fail(TQ_EINVAL, "tq_idmap_export: NULL map");
+  if (m->rows > 0 && (!ext_ids || !deleted)) return fail(TQ_EINVAL, "tq_idmap_export: NULL output array");
+  std::copy(m->ext.begin(), m->ext.begin() + m->rows, ext_ids);
+  std::copy(m->dead.begin(), m->dead.begin() + (m->rows + 31) / 32, deleted);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_idmap_import(tq_idmap* m, const uint64_t* ext_ids, const uint32_t* deleted, int64_t n,
+                                     void* stream) {
+  if (!m) return fail(TQ_EINVAL, "tq_idmap_import: NULL map");
+  if (m->rows != 0) return fail(TQ_EINVAL, "tq_idmap_import: the map already holds %lld rows", (long long)m->rows);
+  if (n < 0 || n > m->capacity)
+    return fail(TQ_EINVAL, "tq_idmap_import: n=%lld outside [0, capacity %lld]", (long long)n,
+                (long long)m->capacity);
+  if (n == 0) return tq::ok();
+  if (!ext_ids || !deleted) return fail(TQ_EINVAL, "tq_idmap_import: NULL ext_ids or deleted");
+  const size_t words = (size_t)((n + 31) / 32);
+  if (n % 32 != 0 && (deleted[words - 1] >> (n % 32)) != 0u)
+    return fail(TQ_EINVAL, "tq_idmap_import: tombstone bits set past row %lld", (long long)n);
+  try {
+    for (int64_t r = 0; r < n; ++r) {
+      if ((deleted[r >> 5] >> (r & 31)) & 1u) continue;
+      const uint64_t id = ext_ids[r];
+      if (id == kEmptyId || !m->live.emplace(id, r).second) {
+        m->live.clear();
+        return fail(TQ_EINVAL, "tq_idmap_import: live id %llu at row %lld is -1 or repeated",
+                    (unsigned long long)id, (long long)r);
+      }
+    }
+    m->ext.assign(ext_ids, ext_ids + n);
+    std::copy(deleted, deleted + words, m->dead.begin());
+  } catch (const std::bad_alloc&) {
+    m->live.clear();
+    m->ext.clear();
+    return fail(TQ_ENOMEM, "tq_idmap_import: out of host memory");
+  }
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(m->d_ext, m->ext.data(), (size_t)n * sizeof(uint64_t), cudaMemcpyHostToDevice, s);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(m->d_dead, m->dead.data(), words * 4, cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) {
+    m->live.clear();
+    m->ext.clear();
+    std::fill(m->dead.begin(), m->dead.end(), 0u);
+    return cuda_fail("tq_idmap_import", e);
+  }
+  m->rows = n;
   return tq::ok();
 }

@@ -5,6 +5,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <vector>
 
 namespace tq {
 
@@ -34,6 +35,11 @@ cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
 
 // Filter build: dense index per vector and per-block tenant bitmaps.
 cudaError_t launch_filter_build(const uint32_t* tenant_ids, FilterDev& f, cudaStream_t s);
+// Rows f.n .. f.n+n_new-1 (ids tenant_ids[0 .. n_new-1], every one already in
+// f.tenants) into dense and block_bits, which must have room for them.
+cudaError_t launch_filter_extend(const uint32_t* tenant_ids, int64_t n_new, const FilterDev& f, cudaStream_t s);
+// The raw tenant id of each of f's n rows into raw [f.n].
+cudaError_t launch_filter_raw_ids(const FilterDev& f, uint32_t* raw, cudaStream_t s);
 
 // LUT scan: per-CTA top-k candidates [nq][grid_x][k] (score, id).  `del`
 // (nullable) is the tombstone bitmap: rows whose bit is set are skipped.
@@ -80,4 +86,6 @@ cudaError_t launch_debug_wait(long long budget, int* status, cudaStream_t s);
 struct tq_filter {
   tq::FilterDev f;
   int device = 0;
+  int64_t cap = 0;                     // rows dense / block_bits have room for
+  std::vector<uint32_t> tenants_host;  // host copy of f.tenants
 };

@@ -792,15 +792,25 @@ __global__ void k_allow_bits(const uint32_t* __restrict__ tenants, int64_t T, in
   }
 }
 
-__global__ void k_filter_build(const uint32_t* __restrict__ tenant_ids, int64_t n,
+// Rows v0 .. v0+n-1 get their dense tenant index and set their bit in their
+// block's bitmap (bits already set by earlier rows of a shared block stay).
+__global__ void k_filter_build(const uint32_t* __restrict__ tenant_ids, int64_t n, int64_t v0,
                                const uint32_t* __restrict__ tenants, int64_t T, int words, int block,
                                uint32_t* __restrict__ dense, uint32_t* __restrict__ block_bits) {
   for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n; v += (int64_t)gridDim.x * blockDim.x) {
     const int64_t pos = find_tenant(tenants, T, tenant_ids[v]);  // always found: tenants holds every id
     const uint32_t p = (uint32_t)(pos < 0 ? 0 : pos);
-    dense[v] = p;
-    atomicOr(block_bits + (v / block) * words + (p >> 5), 1u << (p & 31));
+    const int64_t r = v0 + v;
+    dense[r] = p;
+    atomicOr(block_bits + (r / block) * words + (p >> 5), 1u << (p & 31));
   }
+}
+
+// raw[v] = tenants[dense[v]]: the tenant ids of rows 0 .. n-1 back from a filter.
+__global__ void k_filter_raw_ids(const uint32_t* __restrict__ dense, const uint32_t* __restrict__ tenants, int64_t n,
+                                 uint32_t* __restrict__ raw) {
+  for (int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; v < n; v += (int64_t)gridDim.x * blockDim.x)
+    raw[v] = __ldg(tenants + __ldg(dense + v));
 }
 
 int next_pow2(int x) {
@@ -930,8 +940,23 @@ cudaError_t launch_filter_build(const uint32_t* tenant_ids, FilterDev& f, cudaSt
   cudaError_t e = cudaMemsetAsync(f.block_bits, 0, (size_t)nblocks * f.words * sizeof(uint32_t), s);
   if (e != cudaSuccess) return e;
   const int grid = (int)std::min<int64_t>((f.n + 255) / 256, (int64_t)device_sm_count() * 8);
-  k_filter_build<<<grid, 256, 0, s>>>(tenant_ids, f.n, f.tenants, f.n_tenants, f.words, f.block, f.dense,
+  k_filter_build<<<grid, 256, 0, s>>>(tenant_ids, f.n, 0, f.tenants, f.n_tenants, f.words, f.block, f.dense,
                                       f.block_bits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_filter_extend(const uint32_t* tenant_ids, int64_t n_new, const FilterDev& f, cudaStream_t s) {
+  if (n_new == 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>((n_new + 255) / 256, (int64_t)device_sm_count() * 8);
+  k_filter_build<<<grid, 256, 0, s>>>(tenant_ids, n_new, f.n, f.tenants, f.n_tenants, f.words, f.block, f.dense,
+                                      f.block_bits);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_filter_raw_ids(const FilterDev& f, uint32_t* raw, cudaStream_t s) {
+  if (f.n == 0) return cudaSuccess;
+  const int grid = (int)std::min<int64_t>((f.n + 255) / 256, (int64_t)device_sm_count() * 8);
+  k_filter_raw_ids<<<grid, 256, 0, s>>>(f.dense, f.tenants, f.n, raw);
   return cudaGetLastError();
 }
 

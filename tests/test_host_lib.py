@@ -140,6 +140,9 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert lib.tq_idmap_info(null, null, null, null) == _lib.TQ_EINVAL
     assert lib.tq_idmap_device(null, null, null) == _lib.TQ_EINVAL
     assert lib.tq_idmap_destroy(null) == _lib.TQ_OK
+    assert lib.tq_idmap_export(null, p, p) == _lib.TQ_EINVAL
+    assert lib.tq_idmap_import(null, p, p, 1, null) == _lib.TQ_EINVAL
+    assert lib.tq_filter_append(null, p, 1, null) == _lib.TQ_EINVAL
     # filter
     h = C.c_void_p()
     assert lib.tq_filter_build(p, 10, 48, C.byref(h), null) == _lib.TQ_EINVAL
