@@ -14,7 +14,9 @@ numpy/scipy in float64, written step by step from the paper:
   enters the top-k);
 * Sec. III-A: the id-mapped index (a deleted row never enters the top-k; rows
   are reported by their external uint64 ids);
-* Sec. IV-A: exact brute-force inner-product ground truth and Recall@k.
+* Sec. IV-A: exact brute-force inner-product ground truth and Recall@k;
+  Sec. IV-E: Hit@k and MRR@20 against the exact top-1;
+* Sec. V-C: the over-fetch post-filter baseline that filtering is compared with.
 
 Readings where the paper is silent (each is also listed in the design doc):
 * marginal: the exact coordinate density of a uniformly random unit vector,
@@ -420,6 +422,39 @@ def exact_knn(X, Q, k, tenant_ids=None, allow_off=None, allow_ids=None):
         ids[q, : len(top)] = top
         sc[q, : len(top)] = S[q, top]
     return ids, sc
+
+
+def hit_at_k(approx_ids: np.ndarray, exact_ids: np.ndarray, k: int) -> float:
+    """Hit@k (Sec. IV-E, Table III): the share of queries whose exact top-1
+    result is among the first k approximate results.  Queries without an
+    exact result are skipped."""
+    vals = [int(e[0]) in set(int(v) for v in a[:k]) for a, e in zip(approx_ids, exact_ids) if e[0] >= 0]
+    return float(np.mean(vals)) if vals else 1.0
+
+
+def mrr_at(approx_ids: np.ndarray, exact_ids: np.ndarray, depth: int = 20) -> float:
+    """MRR@depth (Sec. IV-E, Table III): the mean over queries of 1 / rank of
+    the exact top-1 result in the approximate list (rank 1 = first), counted
+    as 0 when it is not among the first `depth`."""
+    vals = []
+    for a, e in zip(approx_ids, exact_ids):
+        if e[0] < 0:
+            continue
+        ranks = [r for r, v in enumerate(a[:depth], start=1) if v == e[0]]
+        vals.append(1.0 / ranks[0] if ranks else 0.0)
+    return float(np.mean(vals)) if vals else 1.0
+
+
+def postfilter_topk(cand_ids: np.ndarray, allowed: np.ndarray, k: int) -> np.ndarray:
+    """The over-fetch post-filter baseline (Sec. V-C, Table V): from each
+    query's unfiltered candidate list (best first, -1 = empty), keep the
+    candidates whose vector is allowed, in order, and return the first k,
+    padded with -1.  allowed: bool [nq, n]."""
+    out = np.full((len(cand_ids), k), -1, dtype=np.int64)
+    for q, row in enumerate(cand_ids):
+        keep = [int(v) for v in row if v >= 0 and allowed[q, v]][:k]
+        out[q, :len(keep)] = keep
+    return out
 
 
 def recall_at_k(approx_ids: np.ndarray, exact_ids: np.ndarray) -> float:

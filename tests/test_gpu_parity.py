@@ -124,6 +124,29 @@ def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
     assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
 
 
+@pytest.mark.parametrize("path", ["lut", "mma"])
+def test_rag_metrics_tiny_config(cuda_lib, torch_dev, tiny_config, path):
+    """Hit@1/3/5/10 and MRR@20 against the exact top-1 (Sec. IV-E, Table III)
+    from the CUDA path's top-20 equal the oracle's, up to one query of the
+    100 (a near-tie at the exact top-1 may rank differently)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = tiny_config
+    tq.set_search_path(path)
+    try:
+        ids, _ = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                             c["enc"].scale, 20)
+    finally:
+        tq.set_search_path("auto")
+    ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, 20, c["d"])
+    exact, _ = O.exact_knn(c["X"], c["Q"], 1)
+    one = 1.0 / len(c["Q"]) + 1e-9
+    for kk in (1, 3, 5, 10):
+        assert abs(O.hit_at_k(ids, exact, kk) - O.hit_at_k(ref.ids, exact, kk)) <= one
+    assert abs(O.mrr_at(ids, exact, 20) - O.mrr_at(ref.ids, exact, 20)) <= one
+    assert O.hit_at_k(ref.ids, exact, 10) > 0.9  # the workload is retrievable at 4 bits
+
+
 @pytest.mark.parametrize("bits,path", [(2, "lut"), (3, "lut"), (8, "lut"), (2, "mma"), (8, "mma")])
 def test_search_bit_widths(cuda_lib, torch_dev, bits, path):
     torch, dev = torch_dev

@@ -512,3 +512,45 @@ def test_delete_all_pads_and_ext_ties_follow_rows():
     gone = O.search(X[[3]], R, cb.centroids32, bits, enc.packed, enc.scale, 3, d,
                     deleted=np.ones(12, bool), ext_ids=ext)
     assert np.all(gone.ids == -1) and np.all(np.isneginf(gone.scores))
+
+
+# ------------------------------------------------ RAG metrics, post-filter ---
+def test_hit_and_mrr_by_hand():
+    """Hit@k and MRR@20 (Sec. IV-E) on lists checked by hand."""
+    approx = np.array([[3, 1, 2], [5, 6, 7], [9, 8, 4], [1, 2, 3]])
+    exact = np.array([[3, 0], [7, 1], [0, 2], [-1, -1]])  # the last query has no exact result
+    assert O.hit_at_k(approx, exact, 1) == pytest.approx(1 / 3)
+    assert O.hit_at_k(approx, exact, 2) == pytest.approx(1 / 3)
+    assert O.hit_at_k(approx, exact, 3) == pytest.approx(2 / 3)
+    assert O.mrr_at(approx, exact, 20) == pytest.approx((1 + 1 / 3 + 0) / 3)
+    assert O.mrr_at(approx, exact, 2) == pytest.approx(1 / 3)  # rank 3 is past the depth
+
+
+def test_exact_search_has_perfect_rag_metrics():
+    X = synth.mixture_corpus(300, 32, 4, seed=2)
+    Q = synth.perturb(X[:15], seed=5)
+    ex, _ = O.exact_knn(X, Q, 20)
+    assert O.hit_at_k(ex, ex, 1) == 1.0 and O.mrr_at(ex, ex) == 1.0
+    shifted = np.concatenate([ex[:, 1:2], ex[:, :1], ex[:, 2:]], axis=1)  # top-1 moved to rank 2
+    assert O.hit_at_k(shifted, ex, 1) == 0.0 and O.hit_at_k(shifted, ex, 2) == 1.0
+    assert O.mrr_at(shifted, ex) == pytest.approx(0.5)
+
+
+def test_postfilter_by_hand_and_full_overfetch_equals_filtering(tenant_index):
+    """The over-fetch post-filter (Sec. V-C) keeps allowed candidates in
+    order; over-fetching the whole corpus recovers the filtered search."""
+    allowed = np.zeros((1, 10), bool)
+    allowed[0, [2, 1, 7]] = True
+    assert O.postfilter_topk(np.array([[5, 2, 9, 1, 7, -1]]), allowed, 3).tolist() == [[2, 1, 7]]
+    assert O.postfilter_topk(np.array([[5, 2, 9, 1, 7, -1]]), allowed, 2).tolist() == [[2, 1]]
+    assert O.postfilter_topk(np.array([[5, 2, -1, -1]]), allowed, 3).tolist() == [[2, -1, -1]]
+    X, R, cb, enc, tid, values, src, Q, d, bits = tenant_index
+    n = len(X)
+    off, ids = synth.allowlists(src, tid, values)
+    filt = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d, tid, off, ids)
+    full = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, n, d)
+    mask = O.allowed_mask(tid, off, ids, len(Q), n)
+    assert np.array_equal(O.postfilter_topk(full.ids, mask, 10), filt.ids)
+    small = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d)
+    pf = O.postfilter_topk(small.ids, mask, 10)
+    assert O.recall_at_k(pf, filt.ids) < 1.0  # over-fetch 1 loses results of small tenants
