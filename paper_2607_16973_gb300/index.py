@@ -77,7 +77,12 @@ class Index:
         """Appends the rows of X ([m, d] float32; a CUDA tensor or host array),
         encoded on the GPU into rows n .. n+m-1; returns n.  `ids` (host
         uint64 [m]) is required with an id map, `tenant_ids` ([m] int32/uint32,
-        host or device) with tenants."""
+        host or device) with tenants.
+
+        The rows are encoded first and committed by the id map and the filter
+        after: rejected ids (live, repeated or -1) leave the index unchanged.
+        A filter that cannot grow (device memory) raises after the id map
+        took the rows; the index should then be rebuilt or reloaded."""
         torch = _torch()
         X = torch.as_tensor(X, dtype=torch.float32, device=self.device).contiguous()
         if X.dim() != 2 or X.shape[1] != self.d:
@@ -101,8 +106,6 @@ class Index:
             if ten.numel() != m or ten.dtype not in (torch.int32, getattr(torch, "uint32", torch.int32)):
                 raise ValueError("one int32/uint32 tenant id per row")
         first = self.n
-        if self.id_map is not None:  # validates the ids before anything changes
-            self.id_map.add(ids, stream=stream)
         rows = slice(first, first + m)
         codes, scale = self.codes[rows], self.scale[rows]
         if codes.data_ptr() % 16 == 0:
@@ -113,6 +116,8 @@ class Index:
             with torch.cuda.stream(stream) if stream is not None else _null():
                 codes.copy_(c)
                 scale.copy_(s)
+        if self.id_map is not None:  # validates the ids; a rejection leaves n as it was
+            self.id_map.add(ids, stream=stream)
         if ten is not None:
             with torch.cuda.stream(stream) if stream is not None else _null():
                 self.tenant_ids[rows].copy_(ten.view(torch.int32))

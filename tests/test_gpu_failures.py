@@ -30,6 +30,35 @@ def test_injected_allocation_failure_is_enomem(cuda_lib):
     assert abs(torch.cuda.mem_get_info()[0] - free0) < (8 << 20)
 
 
+def test_allocation_failure_in_idmap_and_filter_growth(cuda_lib):
+    """An id map that cannot allocate either of its device arrays is
+    TQ_ENOMEM; a filter whose growth cannot allocate (in place of doubling, or
+    of a rebuild for a new tenant) is TQ_ENOMEM and left exactly as it was."""
+    import torch
+    tq = cuda_lib
+    dev = torch.device("cuda:0")
+    free0 = torch.cuda.mem_get_info()[0]
+    for count in (1, 2):
+        tq.load().tq_debug_fail_allocs(count)
+        with pytest.raises(tq.TQError, match="TQ_ENOMEM"):
+            tq.IdMap(1000)
+        tq.load().tq_debug_fail_allocs(0)
+    tid = torch.from_numpy((np.arange(2000, dtype=np.uint32) % 7).view(np.int32)).to(dev)
+    f = tq.Filter(tid[:1000])
+    for new in (tid[1000:1500], torch.full((10,), 99, dtype=torch.int32, device=dev)):  # grow, rebuild
+        for count in (1, 2):
+            tq.load().tq_debug_fail_allocs(count)
+            with pytest.raises(tq.TQError, match="TQ_ENOMEM"):
+                f.append(new)
+            tq.load().tq_debug_fail_allocs(0)
+            assert f.info() == {"n": 1000, "block": 64, "n_tenants": 7}
+    f.append(tid[1000:2000])
+    assert f.info()["n"] == 2000
+    f.close()
+    torch.cuda.synchronize()
+    assert abs(torch.cuda.mem_get_info()[0] - free0) < (8 << 20)
+
+
 def test_bounded_wait_timeout_is_reported_and_context_survives(cuda_lib):
     import torch
     tq = cuda_lib

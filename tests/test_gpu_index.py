@@ -158,3 +158,19 @@ def test_index_search_delete_filter_and_persist(cuda_lib, torch_dev, tmp_path):
     assert ids3.cpu().numpy()[:, 0].tolist() == [(1 << 62) + i for i in range(3)]
     for x in (idx, back):
         x.close()
+
+
+def test_index_rejected_ids_leave_it_unchanged(cuda_lib, torch_dev):
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d = 64
+    X = synth.mixture_corpus(20, d, 2, seed=6)
+    idx = tq.Index(d, 4, capacity=100, id_map=True)
+    idx.add(X[:10], ids=np.arange(10, dtype=np.uint64))
+    with pytest.raises(tq.TQError, match="already live"):
+        idx.add(X[10:15], ids=np.array([10, 11, 3, 12, 13], np.uint64))
+    assert len(idx) == 10 and idx.live == 10 and idx.id_map.info()["rows"] == 10
+    assert idx.add(X[10:15], ids=np.arange(10, 15, dtype=np.uint64)) == 10
+    ids, _ = idx.search(X[[12]], 1)
+    assert ids.cpu().numpy().tolist() == [[12]]
+    idx.close()
