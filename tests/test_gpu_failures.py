@@ -37,15 +37,24 @@ def test_allocation_failure_in_idmap_and_filter_growth(cuda_lib):
     import torch
     tq = cuda_lib
     dev = torch.device("cuda:0")
+    tid = torch.from_numpy((np.arange(2000, dtype=np.uint32) % 7).view(np.int32)).to(dev)
+    extra = torch.full((10,), 99, dtype=torch.int32, device=dev)
+    # run every path once first: a first launch of a kernel or a copy can
+    # reserve device memory for good, which is not a leak
+    warm = tq.Filter(tid[:1000])
+    warm.append(tid[1000:1500])
+    warm.append(extra)
+    warm.close()
+    tq.IdMap(1000).close()
+    torch.cuda.synchronize()
     free0 = torch.cuda.mem_get_info()[0]
     for count in (1, 2):
         tq.load().tq_debug_fail_allocs(count)
         with pytest.raises(tq.TQError, match="TQ_ENOMEM"):
             tq.IdMap(1000)
         tq.load().tq_debug_fail_allocs(0)
-    tid = torch.from_numpy((np.arange(2000, dtype=np.uint32) % 7).view(np.int32)).to(dev)
     f = tq.Filter(tid[:1000])
-    for new in (tid[1000:1500], torch.full((10,), 99, dtype=torch.int32, device=dev)):  # grow, rebuild
+    for new in (tid[1000:1500], extra):  # grow, rebuild
         for count in (1, 2):
             tq.load().tq_debug_fail_allocs(count)
             with pytest.raises(tq.TQError, match="TQ_ENOMEM"):
