@@ -53,9 +53,15 @@ def gather_topk(ids, scores, offset: int, group=None):
 
 def sharded_search(Q, R, centroids, bits: int, codes, scale, k: int, offset: int, group=None, **search_kw):
     """tq_search over this rank's rows, the all-gather of every rank's top-k,
-    and tq_merge_topk: (ids [nq, k] global, scores [nq, k]) on every rank."""
+    and tq_merge_topk: (ids [nq, k] global, scores [nq, k]) on every rank.
+
+    An id map is refused: its search reports external ids, which the merge
+    would take for local rows (shifting them by the offset and breaking ties
+    by them), and each rank knows only its own rows' external ids."""
     import torch
     from . import merge_topk, search
+    if search_kw.get("idmap") is not None:
+        raise ValueError("sharded_search takes no id map: results are global rows")
     if codes.shape[0] == 0:  # an empty shard contributes only empty slots
         ids = torch.full((Q.shape[0], k), -1, dtype=torch.int64, device=Q.device)
         scores = torch.full((Q.shape[0], k), float("-inf"), dtype=torch.float32, device=Q.device)

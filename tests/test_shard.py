@@ -29,6 +29,12 @@ def test_shard_rows_partition(n, world, align):
     assert max(sizes) - min(sizes) <= align
 
 
+def test_sharded_search_refuses_an_id_map():
+    from paper_2607_16973_gb300 import shard
+    with pytest.raises(ValueError, match="no id map"):
+        shard.sharded_search(None, None, None, 4, None, None, 5, 0, idmap=object())
+
+
 def test_shard_rows_rejects_bad_rank():
     with pytest.raises(ValueError):
         shard_rows(10, 2, 2)
