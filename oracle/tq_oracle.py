@@ -18,7 +18,7 @@ numpy/scipy in float64, written step by step from the paper:
   Sec. IV-E: Hit@k and MRR@20 against the exact top-1;
 * Sec. V-C: the over-fetch post-filter baseline that filtering is compared with.
 
-Readings where the paper is silent (each is also listed in the design doc):
+Readings where the paper is silent:
 * marginal: the exact coordinate density of a uniformly random unit vector,
   f_d(x) proportional to (1-x^2)^((d-3)/2) on [-1, 1]; N(0, 1/d) is an option;
 * Lloyd-Max: centroids start at the (i+1/2)/L quantiles of the marginal and the
@@ -252,20 +252,48 @@ def row_bytes(d: int, bits: int) -> int:
 
 def pack(codes: np.ndarray, bits: int) -> np.ndarray:
     """codes uint [n, d] (< 2^bits) -> uint8 [n, d*bits/8]: little-endian bit
-    stream, code j in bits [bits*j, bits*j + bits) of its row."""
+    stream, code j in bits [bits*j, bits*j + bits) of its row.
+
+    Written group by group: g = lcm(bits, 8) / 8 bytes hold 8g/bits whole
+    codes, code r of a group adding code << bits*r to the group's
+    little-endian integer value."""
     codes = np.asarray(codes)
     n, d = codes.shape
-    bitplanes = (codes[:, :, None].astype(np.uint16) >> np.arange(bits, dtype=np.uint16)) & 1
-    return np.packbits(bitplanes.reshape(n, d * bits).astype(np.uint8), axis=1, bitorder="little")
+    g = int(np.lcm(bits, 8)) // 8
+    per = 8 * g // bits
+    nb = (d * bits + 7) // 8
+    groups = -(-nb // g)
+    c = np.zeros((n, groups * per), dtype=np.uint64)
+    c[:, :d] = codes
+    v = np.zeros((n, groups), dtype=np.uint64)
+    for r in range(per):
+        v |= c[:, r::per] << np.uint64(bits * r)
+    out = np.empty((n, groups * g), dtype=np.uint8)
+    for i in range(g):
+        out[:, i::g] = ((v >> np.uint64(8 * i)) & np.uint64(255)).astype(np.uint8)
+    return out[:, :nb]
 
 
 def unpack(packed: np.ndarray, d: int, bits: int) -> np.ndarray:
-    """Inverse of `pack`: uint8 [n, d*bits/8] -> codes uint16 [n, d]."""
+    """Inverse of `pack`: uint8 [n, d*bits/8] -> codes uint16 [n, d].
+
+    The row is read in groups of g = lcm(bits, 8) / 8 bytes, each holding
+    8g/bits whole codes: the group's little-endian integer value v gives code
+    r of the group as (v >> bits*r) & (2^bits - 1)."""
     packed = np.asarray(packed, dtype=np.uint8)
     n = packed.shape[0]
-    b = np.unpackbits(packed, axis=1, bitorder="little")[:, : d * bits]
-    b = b.reshape(n, d, bits).astype(np.uint16)
-    return (b << np.arange(bits, dtype=np.uint16)).sum(axis=2).astype(np.uint16)
+    g = int(np.lcm(bits, 8)) // 8
+    per = 8 * g // bits
+    nb = (d * bits + 7) // 8
+    groups = -(-nb // g)
+    rows = np.zeros((n, groups * g), dtype=np.uint8)
+    rows[:, :nb] = packed[:, :nb]
+    v = np.zeros((n, groups), dtype=np.uint64)
+    for i in range(g):
+        v |= rows[:, i::g].astype(np.uint64) << np.uint64(8 * i)
+    shifts = (np.arange(per, dtype=np.uint64) * np.uint64(bits))
+    codes = (v[:, :, None] >> shifts) & np.uint64((1 << bits) - 1)
+    return codes.reshape(n, groups * per)[:, :d].astype(np.uint16)
 
 
 # ---------------------------------------------------------------------------
@@ -280,6 +308,20 @@ class Encoded:
     norm: np.ndarray     # float64 [n]
 
 
+def rotate_normalize(X: np.ndarray, R: np.ndarray):
+    """Steps 1-2 of the encoder: n = ||x|| and y = R x / n (y = 0 when n = 0),
+    float64.  R is the float32 array the GPU path also gets, promoted.
+    Returns (y [rows, d], n [rows])."""
+    X64 = np.asarray(X, dtype=np.float64)
+    R64 = np.asarray(R, dtype=np.float32).astype(np.float64)
+    n = np.sqrt(np.sum(X64 * X64, axis=1))
+    y = X64 @ R64.T
+    nz = n > 0
+    y[nz] /= n[nz, None]
+    y[~nz] = 0.0
+    return y, n
+
+
 def encode(X: np.ndarray, R: np.ndarray, centroids: np.ndarray, boundaries: np.ndarray,
            bits: int, scale_mode: str = "norm") -> Encoded:
     """Encode rows of X.
@@ -290,18 +332,20 @@ def encode(X: np.ndarray, R: np.ndarray, centroids: np.ndarray, boundaries: np.n
     R, centroids and boundaries are the float32 arrays the GPU path also gets;
     they are promoted to float64 here.
     """
+    y, n = rotate_normalize(X, R)
+    return quantize(y, n, centroids, boundaries, bits, scale_mode)
+
+
+def quantize(y: np.ndarray, n: np.ndarray, centroids: np.ndarray, boundaries: np.ndarray,
+             bits: int, scale_mode: str = "norm") -> Encoded:
+    """Steps 3-5 of the encoder on rotated, normalised rows y (float64) with
+    norms n: nearest-centroid codes, packing and the per-vector scalar."""
     if scale_mode not in SCALE_MODES:
         raise ValueError(scale_mode)
-    X64 = np.asarray(X, dtype=np.float64)
-    R64 = np.asarray(R, dtype=np.float32).astype(np.float64)
     c64 = np.asarray(centroids, dtype=np.float32).astype(np.float64)
     t32 = np.asarray(boundaries, dtype=np.float32)
     assert len(c64) == 1 << bits and len(t32) == len(c64) - 1
-    n = np.sqrt(np.sum(X64 * X64, axis=1))
-    y = X64 @ R64.T
     nz = n > 0
-    y[nz] /= n[nz, None]
-    y[~nz] = 0.0
     code = np.searchsorted(t32, y.astype(np.float32), side="left").astype(np.uint16)
     c = c64[code]
     if scale_mode == "norm":
@@ -346,6 +390,12 @@ def rank_topk(scores32: np.ndarray, allowed: np.ndarray, k: int):
     with (-1, -inf)."""
     idx = np.nonzero(allowed)[0]
     s = scores32[idx]
+    if len(idx) > k:
+        # a vector scoring below the k-th largest score has k better ones and
+        # cannot be in the top k; every vector tied with that score stays
+        kth = np.partition(s, len(s) - k)[len(s) - k]
+        keep = s >= kth
+        idx, s = idx[keep], s[keep]
     order = np.lexsort((idx, -s.astype(np.float64)))
     top = idx[order[:k]]
     ids = np.full(k, -1, dtype=np.int64)
@@ -403,19 +453,27 @@ def search(Q, R, centroids, bits, packed, scale, k, d,
     return SearchResult(ids=ids, scores=sc, scores64=S)
 
 
-def exact_knn(X, Q, k, tenant_ids=None, allow_off=None, allow_ids=None):
+def exact_knn(X, Q, k, tenant_ids=None, allow_off=None, allow_ids=None, row_chunk=65536):
     """Ground truth: brute-force float64 inner product on the unquantised rows
-    (Sec. IV-A), same tie rule and allowlist.  Returns (ids, scores64)."""
-    X64 = np.asarray(X, dtype=np.float64)
+    (Sec. IV-A), same tie rule and allowlist.  Returns (ids, scores64).  The
+    corpus is converted to float64 `row_chunk` rows at a time."""
     Q64 = np.asarray(Q, dtype=np.float64)
-    S = Q64 @ X64.T
-    nq, n = S.shape
+    n = X.shape[0]
+    S = np.empty((Q64.shape[0], n), dtype=np.float64)
+    for r0 in range(0, n, row_chunk):
+        S[:, r0:r0 + row_chunk] = Q64 @ np.asarray(X[r0:r0 + row_chunk], dtype=np.float64).T
+    nq = S.shape[0]
     allowed = allowed_mask(tenant_ids, allow_off, allow_ids, nq, n)
     ids = np.empty((nq, k), dtype=np.int64)
     sc = np.empty((nq, k), dtype=np.float64)
     for q in range(nq):
         idx = np.nonzero(allowed[q])[0]
-        order = np.lexsort((idx, -S[q, idx]))
+        s = S[q, idx]
+        if len(idx) > k:  # only scores >= the k-th largest can be in the top k
+            kth = np.partition(s, len(s) - k)[len(s) - k]
+            keep = s >= kth
+            idx, s = idx[keep], s[keep]
+        order = np.lexsort((idx, -s))
         top = idx[order[:k]]
         ids[q] = -1
         sc[q] = -np.inf

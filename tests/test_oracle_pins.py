@@ -166,6 +166,60 @@ def test_golden_codebooks_are_oracle_output():
         assert np.allclose(cb.boundaries, e["boundaries"], rtol=1e-12, atol=1e-300)
 
 
+def _golden(bits, marginal="beta"):
+    with open(os.path.join(GOLDEN, "codebooks.json")) as f:
+        return [e for e in json.load(f)["entries"] if e["bits"] == bits and e["marginal"] == marginal][0]
+
+
+def test_golden_8bit_is_lloyd_max_fixed_point_by_quadrature():
+    """Every one of the 256 cells of the stored 8-bit codebook (d = 1536): the
+    centroid is the cell's conditional mean and the boundaries are midpoints,
+    by adaptive quadrature of the textbook density (independent of the
+    oracle's incomplete-beta moments).  For a log-concave density that fixed
+    point is unique, so this pins the codebook itself.  The distortion is
+    re-integrated cell by cell as well."""
+    d = 1536
+    e = _golden(8)
+    c, t = np.asarray(e["centroids"]), np.asarray(e["boundaries"])
+    assert len(c) == 256 and np.array_equal(t, (c[:-1] + c[1:]) / 2)
+    f = _coord_density(d)
+    edges = np.concatenate([[-12 / math.sqrt(d)], t, [12 / math.sqrt(d)]])
+    dist = 0.0
+    for i, ci in enumerate(c):
+        a, b = edges[i], edges[i + 1]
+        m0 = integrate.quad(f, a, b, epsabs=0, epsrel=1e-12, limit=200)[0]
+        m1 = integrate.quad(lambda x: x * f(x), a, b, epsabs=0, epsrel=1e-12, limit=200)[0]
+        assert ci == pytest.approx(m1 / m0, rel=1e-9, abs=1e-15), f"cell {i}"
+        dist += integrate.quad(lambda x: (x - ci) ** 2 * f(x), a, b, epsabs=0, epsrel=1e-12, limit=200)[0]
+    assert e["distortion"] == pytest.approx(dist, rel=1e-9)
+
+
+@pytest.mark.parametrize("bits,dD,digits", [(2, 0.11736, 5), (3, 0.03450, 4), (4, 0.009485, 4)])
+def test_beta_distortion_at_1536_matches_independent_values(bits, dD, digits):
+    """d * D at d = 1536 from an independent Lloyd-Max computation on the same
+    Beta marginal, to the digits it was given with (half a unit in the last
+    digit)."""
+    e = _golden(bits)
+    got = 1536 * e["distortion"]
+    half_ulp = 0.5 * 10.0 ** (math.floor(math.log10(dD)) - (digits - 1))
+    assert abs(got - dD) <= half_ulp
+    cb = O.codebook(1536, bits, "beta")
+    assert 1536 * cb.distortion == pytest.approx(got, rel=1e-12)
+
+
+def test_beta_8bit_distortion_below_unconverged_value():
+    """The 8-bit value given alongside the ones above (d * D = 4.12e-5) lies
+    0.2% above the stored codebook's 4.1106e-5.  The stored codebook is the
+    Lloyd-Max fixed point (pinned cell by cell by quadrature), which has the
+    least distortion of any codebook satisfying the two Lloyd conditions, so
+    the larger value is read as an iteration stopped before convergence: the
+    fixed point must lie at or below it, and within 1% (the high-resolution
+    limit (sqrt(3) pi / 2) / L^2 = 4.15e-5 bounds it from above too)."""
+    got = 1536 * _golden(8)["distortion"]
+    assert got <= 4.12e-5 and got == pytest.approx(4.12e-5, rel=0.01)
+    assert got <= math.sqrt(3) * math.pi / 2 / 256 ** 2
+
+
 def test_golden_8bit_distortion_matches_monte_carlo():
     with open(os.path.join(GOLDEN, "codebooks.json")) as f:
         g = json.load(f)
