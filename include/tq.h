@@ -289,14 +289,18 @@ tq_status tq_idmap_import(tq_idmap* m, const uint64_t* ext_ids, const uint32_t* 
  * the device or fail under memory pressure mid-request).  The paper has no
  * counterpart: it is an interface convenience of this library.
  * Same arguments and results as tq_search (always the lookup scan), minus
- * workspace/ws_bytes.  Its scratch is one 8 MiB device array per GPU,
- * reserved when the library is loaded and held until the process exits; the
+ * workspace/ws_bytes.  Its scratch is one 8 MiB device array per GPU; the
  * call allocates nothing.  Sizes whose scratch (about nq*d*4 bytes of rotated
  * queries plus nq*k*8 bytes per scan CTA of candidates) exceeds 8 MiB return
  * TQ_EINVAL with the byte counts.  The first call on each device looks the
- * array's device address up (make it before any stream capture).  All calls on
- * a device share the array: calls whose work overlaps on the GPU (two streams
- * or two threads) race and must be serialised by the caller.  Limit on d: 2048.
+ * array's device address up (make it before any stream capture); under CUDA's
+ * lazy module loading (the default) that first call is also the one that
+ * reserves the array on the device, which then holds it until the process
+ * exits, so make one warm-up call per device before serving (TQ_ENOMEM if the
+ * device has no room for it).  All calls on a device share the array: calls
+ * whose work overlaps on the GPU (two streams or two threads) race and must be
+ * serialised by the caller.  The status for d > 2048 is TQ_EUNSUPPORTED, as
+ * for tq_search.
  */
 tq_status tq_search_static(const float* Q, int64_t nq, int d, const float* R,
                            const float* centroids, int bits, const uint8_t* codes,

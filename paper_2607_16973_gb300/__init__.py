@@ -29,6 +29,36 @@ def _stream_handle(stream) -> int:
     return int(s.cuda_stream)
 
 
+class _on_stream:
+    """Allocations made inside belong to `stream` (None: the current stream).
+
+    Tensors a call creates for work it queues on a side stream must come from
+    that stream's pool: the caching allocator recycles a freed block for the
+    next allocation on the block's own stream without waiting, so a temporary
+    taken from the current stream and freed on return could be handed out
+    again while the side stream's kernels still read or write it."""
+
+    def __init__(self, stream):
+        self._ctx = _torch().cuda.stream(stream) if stream is not None else None
+
+    def __enter__(self):
+        if self._ctx is not None:
+            self._ctx.__enter__()
+        return self
+
+    def __exit__(self, *exc):
+        if self._ctx is not None:
+            return self._ctx.__exit__(*exc)
+        return False
+
+
+def _used_on(t, stream) -> None:
+    """Marks a tensor allocated elsewhere as used by work queued on `stream`,
+    so that its memory is not reused before that work has finished."""
+    if stream is not None and t is not None and t.is_cuda:
+        t.record_stream(stream)
+
+
 def _dev_ptr(t, name: str, dtype=None, contiguous: bool = True) -> int:
     if t is None:
         return 0
@@ -70,10 +100,11 @@ def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
     """tq_encode on CUDA tensors: returns (codes uint8 [n, d*bits/8], scale f32 [n])."""
     torch = _torch()
     n, d = X.shape
-    if codes is None:
-        codes = torch.empty((n, row_bytes(d, bits)), dtype=torch.uint8, device=X.device)
-    if scale is None:
-        scale = torch.empty(n, dtype=torch.float32, device=X.device)
+    with _on_stream(stream):
+        if codes is None:
+            codes = torch.empty((n, row_bytes(d, bits)), dtype=torch.uint8, device=X.device)
+        if scale is None:
+            scale = torch.empty(n, dtype=torch.float32, device=X.device)
     f32 = torch.float32
     check(load().tq_encode(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32),
                            _dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32),
@@ -222,13 +253,14 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
             raise ValueError(f"the id map holds {idmap.info()['rows']} rows, the corpus {n}")
         deleted, ext = idmap.device()
     dev = Q.device
-    if out_ids is None:
-        out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
-    if out_scores is None:
-        out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
-    if workspace is None:  # a caller-owned workspace is size-checked by tq_search itself
-        need = search_workspace(nq, n, d, bits, k, filter)
-        workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
+    with _on_stream(stream):  # freed temporaries must not be recycled before the search ends
+        if out_ids is None:
+            out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+        if out_scores is None:
+            out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+        if workspace is None:  # a caller-owned workspace is size-checked by tq_search itself
+            need = search_workspace(nq, n, d, bits, k, filter)
+            workspace = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
     f32 = torch.float32
     u32 = (torch.int32, getattr(torch, "uint32", torch.int32))
     check(load().tq_search_ex(
@@ -266,10 +298,11 @@ def merge_topk(cand_ids, cand_scores, k: int, out_ids=None, out_scores=None, str
         raise ValueError("cand_ids and cand_scores must both be [n_src, nq, m]")
     n_src, nq, m = cand_ids.shape
     dev = cand_ids.device
-    if out_ids is None:
-        out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
-    if out_scores is None:
-        out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    with _on_stream(stream):
+        if out_ids is None:
+            out_ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+        if out_scores is None:
+            out_scores = torch.empty((nq, k), dtype=torch.float32, device=dev)
     check(load().tq_merge_topk(
         _dev_ptr(cand_ids, "cand_ids", torch.int64), _dev_ptr(cand_scores, "cand_scores", torch.float32),
         n_src, nq, m, k, _dev_ptr(out_ids, "out_ids", torch.int64),

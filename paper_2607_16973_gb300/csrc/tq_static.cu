@@ -7,17 +7,22 @@
 // not call cudaMalloc/cudaFree (an allocation can block, synchronise the
 // device or fail under memory pressure in the middle of a request).  For them
 // this entry point keeps its scratch (rotated queries, allow bitmaps, per-CTA
-// top-k candidates) in one file-scope device array of kStaticScratchBytes,
-// which every GPU that loads the library holds until the process exits.  It
+// top-k candidates) in one file-scope device array of kStaticScratchBytes.  It
 // allocates nothing and calls no allocating routine.
 //
 // The array's name in host code is only a host-side stand-in, never a device
 // address, so the device address is looked up with cudaGetSymbolAddress, once
 // per device, with that device current: the first call on a device does this
-// set-up (make that first call before any stream capture).  Every call on a
-// device shares the one array and the array keeps the last call's contents;
-// nothing in it needs to start at zero because each kernel writes every word
-// it later reads.  Calls whose work overlaps on the GPU (two streams, or two
+// set-up (make that first call before any stream capture).  With CUDA's lazy
+// module loading (the default) that lookup is also what loads the array's
+// module on the device, so the first call on each device is the one that
+// reserves the 8 MiB, which the device then holds until the process exits: a
+// server makes one warm-up call per device before it starts serving.  If the
+// device has no room for the array, that first call returns TQ_ENOMEM.
+//
+// Every call on a device shares the one array and the array keeps the last
+// call's contents; nothing in it needs to start at zero because each kernel
+// writes every word it later reads.  Calls whose work overlaps on the GPU (two streams, or two
 // host threads) race on the array: serialise them.
 #include <cuda_runtime.h>
 
@@ -48,12 +53,15 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
                                       const int64_t* allow_off, const uint32_t* allow_tenants, int k,
                                       int64_t* out_ids, float* out_scores, void* stream) {
   using tq::fail;
-  if (d < 32 || d > 2048 || d % 32 != 0)
-    return fail(TQ_EINVAL, "tq_search_static: d=%d must be a multiple of 32 in [32, 2048]", d);
+  // the same checks, in the same order, as tq_search: the two report the same
+  // status for the same arguments
+  if (d < 32 || d > tq::kMaxD || d % 32 != 0)
+    return fail(TQ_EINVAL, "tq_search_static: d=%d must be a multiple of 32 in [32, %d]", d, tq::kMaxD);
   if (!tq::valid_bits(bits)) return fail(TQ_EINVAL, "tq_search_static: bits=%d must be 2, 3, 4 or 8", bits);
   if (nq < 0 || nq > (1 << 24)) return fail(TQ_EINVAL, "tq_search_static: nq=%lld outside [0, 2^24]", (long long)nq);
   if (n < 1 || n > INT32_MAX - 1) return fail(TQ_EINVAL, "tq_search_static: n=%lld outside [1, 2^31-2]", (long long)n);
   if (k < 1 || k > tq::kMaxK) return fail(TQ_EINVAL, "tq_search_static: k=%d outside [1, %d]", k, tq::kMaxK);
+  if (d > 2048) return fail(TQ_EUNSUPPORTED, "tq_search_static: d=%d > 2048 is not supported by this build", d);
   if (nq == 0) return tq::ok();
   if (!Q || !R || !centroids || !codes || !out_ids || !out_scores)
     return fail(TQ_EINVAL, "tq_search_static: NULL device pointer");
@@ -98,6 +106,11 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
       e = cudaGetSymbolAddress(&tq::g_static_ptr[dev], tq::g_static_scratch);
       if (e != cudaSuccess) {
         tq::g_static_ptr[dev] = nullptr;
+        if (e == cudaErrorMemoryAllocation) {
+          cudaGetLastError();  // not sticky: clear it so later calls start clean
+          return fail(TQ_ENOMEM, "tq_search_static: no device memory for the %zu-byte static scratch: %s",
+                      tq::kStaticScratchBytes, cudaGetErrorString(e));
+        }
         return fail(TQ_ECUDA, "tq_search_static: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
       }
     }

@@ -18,7 +18,7 @@ from __future__ import annotations
 import numpy as np
 
 from . import Filter, IdMap, codebook, encode, rotation, row_bytes, search
-from . import flatfile
+from . import _used_on, flatfile
 
 FORMAT_VERSION = 1
 
@@ -105,6 +105,12 @@ class Index:
             ten = tenant_ids.to(self.device).reshape(-1)
             if ten.numel() != m or ten.dtype not in (torch.int32, getattr(torch, "uint32", torch.int32)):
                 raise ValueError("one int32/uint32 tenant id per row")
+        if stream is not None:
+            # X and ten were made on the current stream: the work queued on
+            # `stream` waits for them, and their memory stays theirs until it ends
+            stream.wait_stream(torch.cuda.current_stream(self.device))
+            _used_on(X, stream)
+            _used_on(ten, stream)
         first = self.n
         rows = slice(first, first + m)
         codes, scale = self.codes[rows], self.scale[rows]
@@ -162,6 +168,10 @@ class Index:
                          if off_h[-1] else np.zeros(1, np.uint32))
                 off = torch.from_numpy(off_h).to(self.device)
                 ten = torch.from_numpy(ten_h.view(np.int32)).to(self.device)
+        if stream is not None:  # inputs made on the current stream, used on `stream`
+            stream.wait_stream(torch.cuda.current_stream(self.device))
+            for t in (Q, off, ten):
+                _used_on(t, stream)
         return search(Q, self.R, self.centroids, self.bits, self.codes[: self.n], self.scale[: self.n], k,
                       filter=self.filter if allow is not None else None, allow_off=off, allow_tenants=ten,
                       workspace=workspace, stream=stream, idmap=self.id_map)

@@ -337,3 +337,37 @@ def test_search_mma_unsupported(cuda_lib, torch_dev):
                 tq.search(Q, R, c, bits, codes, None, k)
     finally:
         tq.set_search_path("auto")
+
+
+def test_search_on_side_stream_keeps_its_temporaries(cuda_lib, torch_dev):
+    """search() on a side stream with library-made workspace and outputs: the
+    caller then allocates and fills blocks of the same sizes on its current
+    stream while the scan is still running.  The temporaries belong to the
+    side stream's pool, so the results equal a search run alone."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, n, bits, k, nq = 1536, 300_000, 4, 10, 48
+    packed = synth.random_codes(n, d * bits // 8, seed=31)
+    scale = synth.random_scales(n, seed=31)
+    R = O.rotation(d, 5).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    Q = synth.gaussian_rows(nq, d, seed=31)
+    Qd, Rd, cd, pd, sd = (_t(torch, dev, a) for a in (Q, R, c32, packed, scale))
+    tq.set_search_path("lut")  # one full corpus pass per query: milliseconds of work
+    try:
+        want_i, want_s = tq.search(Qd, Rd, cd, bits, pd, sd, k)
+        torch.cuda.synchronize()
+        want_i, want_s = want_i.cpu(), want_s.cpu()
+        ws_bytes = tq.search_workspace(nq, n, d, bits, k)
+        side = torch.cuda.Stream(device=dev)
+        side.wait_stream(torch.cuda.current_stream())
+        for _ in range(3):
+            got_i, got_s = tq.search(Qd, Rd, cd, bits, pd, sd, k, stream=side)
+            junk = [torch.full((ws_bytes,), 255, dtype=torch.uint8, device=dev),
+                    torch.full((nq, k), -5, dtype=torch.int64, device=dev),
+                    torch.full((nq, k), 9.0, dtype=torch.float32, device=dev)]
+            side.synchronize()
+            assert torch.equal(got_i.cpu(), want_i) and torch.equal(got_s.cpu(), want_s)
+            del junk
+    finally:
+        tq.set_search_path("auto")

@@ -6,10 +6,15 @@ cudaMalloc in the middle of a request) get a search entry point whose scratch
 is a fixed device array inside the library.  This test calls it through the C
 ABI twice in a row, with different query batches (the second call must not see
 the first call's leftovers in the shared array), and checks each result
-against tq_search with a caller-provided workspace.  It lives in a file that
-pytest collects last and runs alone in a fresh process as well.
+against tq_search with a caller-provided workspace and against the oracle.
+It checks that a call after the first one on the device takes no device
+memory, and runs the comparison once more alone in a fresh process.  It
+lives in a file that pytest collects last.
 """
 import ctypes as C
+import os
+import subprocess
+import sys
 
 import numpy as np
 import pytest
@@ -17,7 +22,7 @@ import pytest
 import oracle as O
 from paper_2607_16973_gb300 import synth
 from paper_2607_16973_gb300.build import build
-from parity import TOL_LUT
+from parity import TOL_LUT, check_topk
 
 pytestmark = pytest.mark.gpu
 
@@ -76,6 +81,15 @@ def test_static_scratch_search_matches_workspace_search(env):
             ok = ids_w >= 0
             assert np.all(np.abs(sc_s[ok] - sc_w[ok]) <= TOL_LUT)
             assert np.array_equal(np.isneginf(sc_s), np.isneginf(sc_w))
+            # and against the oracle's search of the same codes
+            Qh = Qall[:20] if first else Qall[20:]
+            if first:
+                ref = O.search(Qh, R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
+                allowed = np.ones((20, n), bool)
+            else:
+                ref = O.search(Qh, R, cb.centroids32, bits, enc.packed, enc.scale, k, d, tid, off, allow)
+                allowed = O.allowed_mask(tid, off, allow, 20, n)
+            check_topk(ids_s, sc_s, ref.ids, ref.scores64, allowed, k, TOL_LUT)
     finally:
         tq.set_search_path("auto")
         filt.close()
@@ -96,3 +110,43 @@ def test_static_scratch_rejects_oversize(env):
                               scale.data_ptr(), 1000, None, None, None, k, ids.data_ptr(), sc.data_ptr(),
                               torch.cuda.current_stream().cuda_stream)
     assert st == 1 and b"static scratch holds" in lib.tq_last_error()
+
+
+def test_static_scratch_call_takes_no_device_memory(env):
+    """After the first call on the device (which may reserve the array), a
+    call leaves the device's free memory exactly as it was."""
+    tq, lib, torch = env
+    dev = torch.device("cuda:0")
+    d, n, bits, k, nq = 256, 5000, 4, 8, 12
+    T = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    packed = T(synth.random_codes(n, d * bits // 8, seed=12))
+    scale = T(synth.random_scales(n, seed=12))
+    R = T(O.rotation(d, 3).astype(np.float32))
+    c = T(O.codebook(d, bits).centroids32)
+    Q = T(synth.gaussian_rows(nq, d, seed=12))
+    first = _static_search(lib, torch, Q, R, c, bits, packed, scale, k)
+    ids = torch.empty((nq, k), dtype=torch.int64, device=dev)
+    sc = torch.empty((nq, k), dtype=torch.float32, device=dev)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    st = lib.tq_search_static(Q.data_ptr(), nq, d, R.data_ptr(), c.data_ptr(), bits, packed.data_ptr(),
+                              scale.data_ptr(), n, None, None, None, k, ids.data_ptr(), sc.data_ptr(),
+                              torch.cuda.current_stream().cuda_stream)
+    assert st == 0, lib.tq_last_error()
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert np.array_equal(ids.cpu().numpy(), first[0])
+
+
+def test_static_scratch_fresh_process(env):
+    """The comparison above, alone in a new process: the first call there is
+    also the first on the device."""
+    if os.environ.get("TQ_NO_ALLOC_CHILD"):
+        pytest.skip("already the child process")
+    here = os.path.dirname(os.path.abspath(__file__))
+    envv = dict(os.environ, TQ_NO_ALLOC_CHILD="1")
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-p", "no:cacheprovider", "-m", "gpu",
+                        os.path.join(here, "test_zz_no_alloc.py"), "-k", "matches_workspace_search"],
+                       cwd=os.path.dirname(here), env=envv, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-3000:]
+    assert "1 passed" in r.stdout
