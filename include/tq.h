@@ -66,8 +66,15 @@ enum { TQ_MARGINAL_BETA = 0, TQ_MARGINAL_GAUSS = 1 };
 enum { TQ_SCALE_NORM = 0, TQ_SCALE_NONE = 1, TQ_SCALE_UNBIASED = 2 };
 
 /* Search kernels: AUTO picks by batch size; LUT forces the per-query lookup
- * scan, MMA forces the tensor-core decode-GEMM scan (used by tests). */
-enum { TQ_PATH_AUTO = 0, TQ_PATH_LUT = 1, TQ_PATH_MMA = 2 };
+ * scan, MMA forces the tensor-core decode-GEMM scan (used by tests).
+ * LUT_FIXED is the lookup scan with, for 4-bit codes at d >= 512, a table of
+ * 15-bit fixed-point centroid values (each centroid rounded to a step near
+ * max|c| / 16383, chosen to make the largest rounding error small: about
+ * 6e-7 for the d = 1536 codebook; the score error is that rounding error
+ * weighted by the rotated query, about 2.5e-7 rms for unit queries).  It
+ * moves half the shared-memory bytes of the exact fp32 table per code but
+ * needs more instructions per code. */
+enum { TQ_PATH_AUTO = 0, TQ_PATH_LUT = 1, TQ_PATH_MMA = 2, TQ_PATH_LUT_FIXED = 3 };
 
 typedef struct tq_filter tq_filter; /* opaque, library-owned */
 

@@ -31,11 +31,13 @@ inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct SearchPlan {
   int grid_lut = 1, grid_mma = 0;
-  size_t off_status = 0, off_rot = 0, off_allow = 0, off_qpack = 0, off_cs = 0, off_ci = 0, total = 0;
+  size_t off_status = 0, off_cnt = 0, off_rot = 0, off_allow = 0, off_mask = 0, off_qpack = 0, off_cs = 0,
+         off_ci = 0, total = 0;
 };
 
-// Workspace layout (both scan paths): status word | rotated queries | allow
-// bitmaps | fp16 query tiles (tensor-core path) | candidate scores | ids.
+// Workspace layout (both scan paths): status word | merge counters (one per
+// query) | rotated queries | allow bitmaps | block masks | fp16 query tiles
+// (tensor-core path) | candidate scores | ids.
 SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
   SearchPlan p;
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
@@ -45,10 +47,14 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   size_t off = 0;
   p.off_status = off;
   off = align_up(off + sizeof(int));
+  p.off_cnt = off;
+  off = align_up(off + (size_t)nq * sizeof(int));
   p.off_rot = off;
   off = align_up(off + (size_t)nq * d * sizeof(float));
   p.off_allow = off;
   if (filter) off = align_up(off + (size_t)nq * filter->f.words * sizeof(uint32_t));
+  p.off_mask = off;
+  if (filter) off = align_up(off + (size_t)nq * filter_mask_words(filter->f) * sizeof(uint32_t));
   p.off_qpack = off;
   if (mma) off = align_up(off + mma_qpack_bytes(nq, d));
   p.off_cs = off;
@@ -313,11 +319,13 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
   cudaStream_t s = (cudaStream_t)stream;
   char* ws = static_cast<char*>(workspace);
   int* status = reinterpret_cast<int*>(ws + p.off_status);
+  int* counters = reinterpret_cast<int*>(ws + p.off_cnt);
   float* qrot = reinterpret_cast<float*>(ws + p.off_rot);
   uint32_t* allow = filter ? reinterpret_cast<uint32_t*>(ws + p.off_allow) : nullptr;
+  uint32_t* bmask = filter ? reinterpret_cast<uint32_t*>(ws + p.off_mask) : nullptr;
   float* cs = reinterpret_cast<float*>(ws + p.off_cs);
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
-  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, s);  // also zeroes the status word
+  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);  // also zeroes both
   if (use_mma) {
     if (e == cudaSuccess)
       e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, deleted, k, p.grid_mma,
@@ -326,12 +334,13 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
     if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, ext_ids, out_ids, out_scores, s);
   } else {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
+    if (e == cudaSuccess && filter) e = tq::launch_block_mask(filter->f, allow, nq, bmask, s);
     if (e == cudaSuccess)
       e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
-                              filter ? &filter->f : nullptr, allow,
-                              k, p.grid_lut, cs, ci, s, (cudaEvent_t)tq::profile_start(),
-                              (cudaEvent_t)tq::profile_stop());
-    if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_lut * k, k, ext_ids, out_ids, out_scores, s);
+                              filter ? &filter->f : nullptr, allow, bmask,
+                              path == TQ_PATH_LUT_FIXED && d >= tq::kFixMinD,
+                              k, p.grid_lut, cs, ci, status, counters, ext_ids, out_ids, out_scores, s,
+                              (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
   }
   if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
   return tq::ok();

@@ -230,12 +230,24 @@ k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict_
   }
 }
 
-// Q' = Q R^T, plain store epilogue (nq > 8).
+// Every search starts with the query rotation, which clears the search's
+// status word and merge counters, and lets the kernel after it (launched as a
+// programmatic dependent) start its prologue while the rotation runs.
+__device__ __forceinline__ void search_start(int* status, int* counters, int64_t n_counters) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int64_t nb = (int64_t)gridDim.x * gridDim.y * gridDim.z;
+  const int64_t b = blockIdx.x + (int64_t)gridDim.x * (blockIdx.y + (int64_t)gridDim.y * blockIdx.z);
+  if (status && b == 0 && threadIdx.x == 0) *status = 0;
+  if (counters)
+    for (int64_t i = b * blockDim.x + threadIdx.x; i < n_counters; i += nb * blockDim.x) counters[i] = 0;
+}
+
+// Q' = Q R^T, plain store epilogue (nq > 256).
 __global__ void __launch_bounds__(NT, 2)
 k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R,
-              float* __restrict__ out, int* __restrict__ status) {
+              float* __restrict__ out, int* __restrict__ status, int* __restrict__ counters, int64_t n_counters) {
   __shared__ GemmSmem sm;
-  if (status && blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0 && threadIdx.x == 0) *status = 0;
+  search_start(status, counters, n_counters);
   const int64_t row0 = (int64_t)blockIdx.x * BM;
   const int col0 = blockIdx.y * BN;
   // gridDim.z = 2 splits the contraction in halves, each added onto the
@@ -261,12 +273,13 @@ k_rotate_gemm(const float* __restrict__ Q, int64_t nq, int d, const float* __res
   }
 }
 
-// Q' = Q R^T for nq <= 8: one warp per output coordinate, R read once.
+// Q' = Q R^T for groups of NQ <= 8 queries: one warp per output coordinate,
+// R read once per group.
 template <int NQ>
 __global__ void __launch_bounds__(256)
 k_rotate_gemv(const float* __restrict__ Q, int64_t nq, int d, const float* __restrict__ R, float* __restrict__ out,
-              int* __restrict__ status) {
-  if (status && blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0) *status = 0;  // a new search starts
+              int* __restrict__ status, int* __restrict__ counters, int64_t n_counters) {
+  search_start(status, counters, n_counters);
   const int lane = threadIdx.x & 31;
   const int i = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (i >= d) return;
@@ -281,16 +294,18 @@ k_rotate_gemv(const float* __restrict__ Q, int64_t nq, int d, const float* __res
   const float4* r4 = reinterpret_cast<const float4*>(R + (int64_t)i * d);
   const int d4 = d / 4;
   // R (d*d*4 bytes) is usually evicted from L2 by the corpus stream between
-  // searches, so issue 8 row loads per lane before using any of them
-  for (int j0 = lane; j0 < d4; j0 += 32 * 8) {
-    float4 rv[8];
+  // searches, so a lane issues all its row loads (16 for d = 2048) before
+  // using any of them
+  constexpr int RL = 16;
+  for (int j0 = lane; j0 < d4; j0 += 32 * RL) {
+    float4 rv[RL];
 #pragma unroll
-    for (int t = 0; t < 8; ++t) {
+    for (int t = 0; t < RL; ++t) {
       const int j = j0 + 32 * t;
       rv[t] = j < d4 ? __ldg(r4 + j) : make_float4(0.f, 0.f, 0.f, 0.f);
     }
 #pragma unroll
-    for (int t = 0; t < 8; ++t) {
+    for (int t = 0; t < RL; ++t) {
       const int j = j0 + 32 * t;
       if (j >= d4) break;
 #pragma unroll
@@ -374,13 +389,13 @@ cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, cons
 }
 
 cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out, int* status,
-                          cudaStream_t s) {
+                          int* counters, int64_t n_counters, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   if (nq <= 8) {
     const dim3 grid((unsigned)((d + 7) / 8), 1);
     switch (nq) {
 #define TQ_GEMV_CASE(N) \
-  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status); break;
+  case N: k_rotate_gemv<N><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status, counters, n_counters); break;
       TQ_GEMV_CASE(1) TQ_GEMV_CASE(2) TQ_GEMV_CASE(3) TQ_GEMV_CASE(4)
       TQ_GEMV_CASE(5) TQ_GEMV_CASE(6) TQ_GEMV_CASE(7) TQ_GEMV_CASE(8)
 #undef TQ_GEMV_CASE
@@ -389,7 +404,7 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
   }
   if (nq <= 256) {  // groups of 8 queries: R stays in L2 across the groups; the GEMM would use few CTAs
     const dim3 grid((unsigned)((d + 7) / 8), (unsigned)((nq + 7) / 8));
-    k_rotate_gemv<8><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status);
+    k_rotate_gemv<8><<<grid, 256, 0, s>>>(Q, nq, d, R, out, status, counters, n_counters);
     return cudaGetLastError();
   }
   // split the contraction in two when the tiles alone would leave SMs idle
@@ -401,7 +416,7 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
     if (e != cudaSuccess) return e;
   }
   dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN), split ? 2u : 1u);
-  k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out, status);
+  k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out, status, counters, n_counters);
   return cudaGetLastError();
 }
 

@@ -24,9 +24,10 @@ cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, cons
                           const float* boundaries, int bits, int scale_mode, uint8_t* codes,
                           float* scale, cudaStream_t s);
 
-// q' = R q for nq queries: out [nq * d] float32.
+// q' = R q for nq queries: out [nq * d] float32.  Also zeroes the status word
+// and `n_counters` merge counters (each nullable) for the search it starts.
 cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, float* out, int* status,
-                          cudaStream_t s);
+                          int* counters, int64_t n_counters, cudaStream_t s);
 
 // Per-query allow bitmaps over the dense tenant index: out [nq * words].
 cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
@@ -43,11 +44,26 @@ cudaError_t launch_filter_raw_ids(const FilterDev& f, uint32_t* raw, cudaStream_
 
 // LUT scan: per-CTA top-k candidates [nq][grid_x][k] (score, id).  `del`
 // (nullable) is the tombstone bitmap: rows whose bit is set are skipped.
+// With a filter, `allow_bits` [nq * f->words] are the queries' allow bitmaps
+// and `bmask` [nq * filter_mask_words(*f)] their block masks.  `fix` selects
+// the fixed-point byte-pair table for 4-bit codes (else the exact fp32 one).
+// `err` is the search status word the scan's bounded waits report to.  The
+// last CTA of each query merges the CTA lists into out_ids/out_scores
+// (written as ext[row] with an id map); `counters` [nq] must be zero (the
+// query rotation zeroes them).
 int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d);
 cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
-                            const FilterDev* f, const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
-                            int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1);
+                            const FilterDev* f, const uint32_t* allow_bits, const uint32_t* bmask, bool fix,
+                            int k, int grid_x, float* cand_s, int32_t* cand_i, int* err, int* counters,
+                            const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s,
+                            cudaEvent_t ev0, cudaEvent_t ev1);
+
+// Per-query bitmap over the filter's blocks: bit b set when block b holds a
+// tenant the query allows.  out [nq * filter_mask_words(f)].
+int filter_mask_words(const FilterDev& f);
+cudaError_t launch_block_mask(const FilterDev& f, const uint32_t* allow, int64_t nq, uint32_t* mask,
+                              cudaStream_t s);
 
 // Final merge of per-CTA candidates into sorted top-k; with `ext` (nullable)
 // the rows are written as ext[row].

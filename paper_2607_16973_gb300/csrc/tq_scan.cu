@@ -1,7 +1,7 @@
 // Search-side kernels: the lookup scan with fused top-k (Sec. II-B step 5,
 // Sec. III-B), per-query allow bitmaps, the filter build and the final merge.
 //
-// Lookup scan layout.  One warp scores 8 consecutive vectors per step.  Each
+// Lookup scan layout.  One warp scores 4 consecutive vectors per step.  Each
 // packed row is cut into chunks of 16 codes (2*bits bytes); lane l owns chunks
 // l, l+32, l+64, ... of every row, so each load instruction of a warp reads a
 // contiguous run of one row and every lane always handles the same
@@ -16,7 +16,8 @@
 // neither does a deleted one (its bit set in the caller's tombstone bitmap,
 // the O(1) deletion of the id-mapped index of Sec. III-A).  Blocks
 // of `block` vectors whose tenant bitmap shares no bit with the query's allow
-// bitmap are skipped before any code byte is read (Sec. III-B).
+// bitmap are skipped before any code byte is read (Sec. III-B): a small kernel
+// turns the two bitmaps into one bit per block and query first.
 #include <cuda_runtime.h>
 
 #include <climits>
@@ -26,6 +27,7 @@
 
 #include "tq_internal.h"
 #include "tq_kernels.h"
+#include "tq_wait.cuh"
 
 namespace tq {
 namespace {
@@ -38,6 +40,16 @@ constexpr unsigned FULL = 0xffffffffu;
 __device__ __forceinline__ bool tombstoned(const uint32_t* __restrict__ del, int v) {
   return del && ((__ldg(del + (v >> 5)) >> (v & 31)) & 1u);
 }
+// Programmatic dependent launch: a kernel launched with the
+// programmatic-serialization attribute may start while the kernel before it
+// in the stream still runs; it must wait here before reading anything that
+// kernel (or any earlier one) wrote.  Without the attribute both are no-ops
+// in effect.  The kernel before it lets it start early with launch_dependents.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 constexpr int SCAN_NT = 256;
 constexpr int SCAN_WARPS = SCAN_NT / 32;
 constexpr int MERGE_P = 2048;
@@ -214,162 +226,136 @@ __device__ __forceinline__ void load_q2(float2 (&q2)[S][8], const float* qq, int
   }
 }
 
-// Sums p[0..7] across the warp: afterwards lanes 4i..4i+3 hold the total of
-// p[i] (a transposed butterfly: 4 + 2 + 1 + 1 + 1 shuffles for 8 values).
-__device__ __forceinline__ float warp_sum8(float (&p)[8]) {
-  const int lane = threadIdx.x & 31;
-  const bool h16 = lane & 16, h8 = lane & 8, h4 = lane & 4;
-  float a[4], b[2];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float send = h16 ? p[i] : p[i + 4];
-    const float keep = h16 ? p[i + 4] : p[i];
-    a[i] = keep + __shfl_xor_sync(FULL, send, 16);
-  }
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {
-    const float send = h8 ? a[i] : a[i + 2];
-    const float keep = h8 ? a[i + 2] : a[i];
-    b[i] = keep + __shfl_xor_sync(FULL, send, 8);
-  }
-  float c = (h4 ? b[1] : b[0]) + __shfl_xor_sync(FULL, h4 ? b[0] : b[1], 4);
-  c += __shfl_xor_sync(FULL, c, 2);
-  c += __shfl_xor_sync(FULL, c, 1);
-  return c;
-}
-
-// Each warp scores 8 consecutive vectors per step: all their code loads (and
-// their scales and tenants) are issued before any arithmetic, so a warp keeps
-// 8 x d*bits/8 bytes in flight.
-template <int BITS, int S>
-__global__ void __launch_bounds__(SCAN_NT, 2)
-k_scan_lut(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
-           const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
-           const uint32_t* __restrict__ del,
-           const uint32_t* __restrict__ dense, const uint32_t* __restrict__ block_bits, int words,
-           int fblock, const uint32_t* __restrict__ allow_bits, int k, int P,
-           float* __restrict__ cand_s, int* __restrict__ cand_i) {
-  constexpr int L = 1 << BITS;
-  constexpr int CB = 2 * BITS;
-  constexpr int V = 8;  // vectors per warp step; a CTA step covers 64
-  // 4-bit codes use the byte-pair table (pair_dot), other widths the
-  // per-code table [L][32] with entry (c, lane) in bank lane
-  constexpr int TAB_BYTES = BITS == 4 ? PAIR_TAB_BYTES : L * 32 * 4;
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* ctab = reinterpret_cast<float*>(smem_raw);
-  float* ls = reinterpret_cast<float*>(smem_raw + TAB_BYTES);  // [P] scores; warp w's list at [w*k, w*k+k)
-  int* li = reinterpret_cast<int*>(ls + P);                     // [P] ids
+// Merge of per-CTA candidate lists that are each sorted best first and hold
+// exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
+// any one list is beaten or matched by that list's k entries, so the global
+// k-th best is at least as good as the best such T and worse candidates are
+// skipped at once.  Each warp keeps a sorted top-k of its share of the rest
+// (ballot, then one warp-wide insertion per candidate that still beats the
+// warp's k-th); warp 0 then folds the sorted warp lists into the result,
+// leaving each list at its first entry that no longer qualifies.  With an
+// id map the result rows are written as their external ids.  Every thread of
+// the block calls it; cs/ci hold one query's lists [nlists][k] (read through
+// L2: in the scans' tail other CTAs of the same grid wrote them); ws/wi are
+// shared scratch of (blockDim.x / 32) * k entries; out_* point at the query's
+// k results.
+__device__ void merge_lists_block(const float* cs, const int* ci, int nlists, int k, const uint64_t* __restrict__ ext,
+                                  int64_t* out_ids, float* out_scores, float* ws, int* wi) {
+  __shared__ float red_s[32];
+  __shared__ int red_i[32];
+  const int nwarps = blockDim.x >> 5;
+  const int total = nlists * k;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int q = blockIdx.y;
-  if constexpr (BITS == 4) pair_table_init(reinterpret_cast<float2*>(smem_raw), centroids, tid, SCAN_NT);
-  else
-    for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
-  for (int i = tid; i < P; i += SCAN_NT) {
-    ls[i] = -INFINITY;
-    li[i] = INT_MAX;
-  }
-  const int nchunks = d >> 4;
-  const float* qq = qrot + (size_t)q * d;
-  float qr[BITS == 4 ? 1 : S][16];
-  float2 q2[BITS == 4 ? S : 1][8];
-  if constexpr (BITS == 4) {
-    load_q2(q2, qq, nchunks, lane);
-  } else {
-#pragma unroll
-    for (int s = 0; s < S; ++s) {
-      const int chunk = lane + 32 * s;
-#pragma unroll
-      for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+  // 1. T = best k-th entry over the lists
+  float ts = -INFINITY;
+  int ti = INT_MAX;
+  for (int l = tid; l < nlists; l += blockDim.x) {
+    const float a = __ldcg(cs + l * k + k - 1);
+    const int b = __ldcg(ci + l * k + k - 1);
+    if (better(a, b, ts, ti)) {
+      ts = a;
+      ti = b;
     }
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float a = __shfl_xor_sync(FULL, ts, o);
+    const int b = __shfl_xor_sync(FULL, ti, o);
+    if (better(a, b, ts, ti)) {
+      ts = a;
+      ti = b;
+    }
+  }
+  if (lane == 0) {
+    red_s[warp] = ts;
+    red_i[warp] = ti;
+  }
+  for (int i = lane; i < k; i += 32) {
+    ws[warp * k + i] = -INFINITY;
+    wi[warp * k + i] = INT_MAX;
+  }
   __syncthreads();
-
-  const int64_t row_bytes = (int64_t)d * BITS / 8;
-  const uint32_t* ab = allow_bits ? allow_bits + (size_t)q * words : nullptr;
-  float* wl_s = ls + warp * k;
-  int* wl_i = li + warp * k;
+  ts = red_s[0];
+  ti = red_i[0];
+  for (int w = 1; w < nwarps; ++w)
+    if (better(red_s[w], red_i[w], ts, ti)) {
+      ts = red_s[w];
+      ti = red_i[w];
+    }
+  // 2. per-warp sorted top-k of the candidates at least as good as T
+  float* ls = ws + warp * k;
+  int* li = wi + warp * k;
   int cnt = 0;
   float th_s = -INFINITY;
   int th_i = INT_MAX;
-  const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
-  const int my = (lane >> 2) & 7;  // the vector whose total this lane ends up holding
-  const uint32_t lane4 = (uint32_t)lane * 4u;
-  for (int st = blockIdx.x; st < nsteps; st += gridDim.x) {
-    const int v0 = st * (SCAN_WARPS * V) + warp * V;
-    if (v0 >= n) continue;
-    if (ab) {  // the warp's 8 vectors lie in one filter block (block is 32 or 64)
-      const int fb = v0 / fblock;
-      uint32_t any = 0;
-      for (int w = lane; w < words; w += 32) any |= __ldg(block_bits + (size_t)fb * words + w) & __ldg(ab + w);
-      if (!__any_sync(FULL, any != 0u)) continue;  // no allowed vector: skip before reading codes
+  for (int c0 = warp * 32; c0 < total; c0 += blockDim.x) {
+    const int c = c0 + lane;
+    float a = -INFINITY;
+    int b = INT_MAX;
+    if (c < total) {
+      a = __ldcg(cs + c);
+      b = __ldcg(ci + c);
     }
-    const int vm = v0 + my;
-    float sc_my = 0.f;
-    uint32_t ten_my = 0;
-    if ((lane & 3) == 0 && vm < n) {
-      sc_my = scale ? __ldg(scale + vm) : 1.0f;
-      if (ab) ten_my = __ldg(dense + vm);
-    }
-    Chunk<BITS> ch[V][S];
-#pragma unroll
-    for (int i = 0; i < V; ++i) {
-      const uint8_t* row = codes + (size_t)(v0 + i) * row_bytes;
-#pragma unroll
-      for (int s = 0; s < S; ++s) {
-        const int chunk = lane + 32 * s;
-        if (v0 + i < n && chunk < nchunks) ch[i][s].load(row + chunk * CB);
-        else ch[i][s].zero();
-      }
-    }
-    // keep every load above in flight before the first lookup below
-    asm volatile("" ::: "memory");
-    float p[V];
-    const char* tab = reinterpret_cast<const char*>(ctab);
-#pragma unroll
-    for (int i = 0; i < V; ++i) {
-      if constexpr (BITS == 4) {
-        p[i] = pair_dot<S>(ch[i], q2, tab, lane4 * 2u);
-      } else {
-        float acc = 0.f;
-#pragma unroll
-        for (int s = 0; s < S; ++s)
-#pragma unroll
-          for (int t = 0; t < 16; ++t)
-            acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + ch[i][s].off(t, lane4)), acc);
-        p[i] = acc;
-      }
-    }
-    const float total = warp_sum8(p);
-    float score = -INFINITY;
-    bool cand = false;
-    if ((lane & 3) == 0 && vm < n) {
-      score = total * sc_my;
-      const bool allowed = !ab || ((__ldg(ab + (ten_my >> 5)) >> (ten_my & 31)) & 1u);
-      cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
-    }
+    const bool cand = b != INT_MAX && !better(ts, ti, a, b) && better(a, b, th_s, th_i);
     unsigned m = __ballot_sync(FULL, cand);
-    while (m) {  // in vector order; re-checked against the moving threshold
+    while (m) {
       const int src = __ffs(m) - 1;
       m &= m - 1;
-      const float s = __shfl_sync(FULL, score, src);
-      const int vv = v0 + ((src >> 2) & 7);
-      if (better(s, vv, th_s, th_i)) {
-        warp_insert(wl_s, wl_i, k, cnt, s, vv);
+      const float sv = __shfl_sync(FULL, a, src);
+      const int iv = __shfl_sync(FULL, b, src);
+      if (better(sv, iv, th_s, th_i)) {
+        warp_insert(ls, li, k, cnt, sv, iv);
         cnt = min(cnt + 1, k);
         if (cnt == k) {
-          th_s = wl_s[k - 1];
-          th_i = wl_i[k - 1];
+          th_s = ls[k - 1];
+          th_i = li[k - 1];
         }
       }
     }
   }
   __syncthreads();
-  block_sort(ls, li, P);
-  for (int i = tid; i < k; i += SCAN_NT) {
-    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
-    cand_s[o] = ls[i];
-    cand_i[o] = li[i];
+  // 3. warp 0 folds the other warps' sorted lists into its own
+  if (warp == 0) {
+    for (int w = 1; w < nwarps; ++w) {
+      for (int i = 0; i < k; ++i) {
+        const float sv = ws[w * k + i];
+        const int iv = wi[w * k + i];
+        if (iv == INT_MAX || !better(sv, iv, th_s, th_i)) break;  // sorted: the rest are worse
+        warp_insert(ls, li, k, cnt, sv, iv);
+        cnt = min(cnt + 1, k);
+        if (cnt == k) {
+          th_s = ls[k - 1];
+          th_i = li[k - 1];
+        }
+      }
+    }
+    for (int i = lane; i < k; i += 32) {
+      const bool empty = li[i] == INT_MAX;
+      out_ids[i] = empty ? -1 : ext ? (int64_t)__ldg(ext + li[i]) : (int64_t)li[i];
+      out_scores[i] = empty ? -INFINITY : ls[i];
+    }
   }
+}
+
+// Publishes a scan CTA's sorted list of k (already in cand_*) and, in the
+// last CTA of the query to finish (an arrival counter per query, zeroed by
+// the query rotation that starts every search), merges all of the query's
+// lists into its results: no separate merge launch.  ls/li: the CTA's list
+// scratch (at least blockDim.x / 32 * k entries).
+__device__ __forceinline__ void merge_if_last(const float* cand_s, const int* cand_i, int k, int* counters,
+                                              const uint64_t* ext, int64_t* out_ids, float* out_scores, float* ls,
+                                              int* li) {
+  __shared__ int last;
+  const int q = blockIdx.y;
+  __threadfence();  // this thread's part of the list, before the arrival
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(counters + q, 1) == (int)gridDim.x - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();  // every other CTA's list, after seeing all arrivals
+  const size_t base = (size_t)q * gridDim.x * k;
+  merge_lists_block(cand_s + base, cand_i + base, gridDim.x, k, ext, out_ids + (size_t)q * k,
+                    out_scores + (size_t)q * k, ls, li);
 }
 
 // Sums p[0..3] across the warp: afterwards lanes 8i..8i+7 hold the total of
@@ -391,41 +377,192 @@ __device__ __forceinline__ float warp_sum4(float (&p)[4]) {
   return c;
 }
 
-// Unfiltered lookup scan with a register double buffer: each warp scores 4
-// consecutive vectors per step and issues the next step's code loads before
-// it starts on the current ones, so every warp always has loads in flight.
-template <int BITS, int S>
+// Fixed-point byte-pair table for 4-bit codes.  The exact table above moves
+// 8 bytes through shared memory per packed byte (two fp32 centroids), which
+// bounds the scan by the shared-memory datapath (128 B per cycle per SM).
+// Here each centroid is a 15-bit fixed-point value u_v = rint(c_v / step) +
+// 16384, and the entry (x, lane) = u[x & 15] | u[x >> 4] << 16 is 4 bytes: one
+// wavefront per warp lookup instead of two.  A byte permute turns a 16-bit
+// half into a float without any arithmetic: bytes (0, u_lo, u_hi, 0x3F) are
+// the float 0.5 + u * 2^-16 (u < 2^15 keeps bit 23, the exponent's low bit,
+// clear), exact.  With the query pre-scaled, q''_j = q'_j * step * 2^16,
+//   q''_j * (0.5 + u_j 2^-16 - 0.75) = q'_j * (u_j - 16384) * step = q'_j * c^_j,
+// so each lane starts its two accumulators at -0.75 * (its sum of q'') and
+// then needs one fused multiply-add per centroid: per packed byte a byte
+// permute for the address, one 4-byte load, two byte permutes and one paired
+// FMA.  c^_v differs from c_v by the rounding to the step; the step is the
+// one, among FIX_CANDIDATES values in [d0, 1.25 d0) (d0 = max|c| / 16383),
+// whose largest rounding error over the 16 centroids is least, chosen the
+// same way by every CTA.
+constexpr int FIX_CANDIDATES = 2048;
+constexpr uint32_t FIX_HALF = 0x3F000000u;  // byte 3 of 0.5f, byte 0 zero
+
+// Fills the fixed-point table (uint32 entry (x, lane) at index x * 64 + lane;
+// the other half of each 256-byte row is unused) and returns the step * 2^16
+// the rotated query is multiplied by.  All threads of the CTA call it; `red`
+// is shared scratch of 2 * 32 words.
+__device__ float fix_table_init(uint32_t* tab, const float* __restrict__ centroids, float* red, int tid, int nt) {
+  float c[16];
+  float m = 0.f;
+#pragma unroll
+  for (int v = 0; v < 16; ++v) {
+    c[v] = __ldg(centroids + v);
+    m = fmaxf(m, fabsf(c[v]));
+  }
+  const float d0 = m > 0.f ? m / 16383.0f * (1.0f + 0x1p-20f) : 1.0f;
+  float best_e = INFINITY;
+  int best_i = 0;
+  for (int i = tid; i < FIX_CANDIDATES; i += nt) {
+    const float st = d0 * (1.0f + (float)i * (0.25f / FIX_CANDIDATES));
+    const float inv = 1.0f / st;
+    float e = 0.f;
+#pragma unroll
+    for (int v = 0; v < 16; ++v) {
+      const float r = c[v] * inv;
+      e = fmaxf(e, fabsf(r - rintf(r)));
+    }
+    e *= st;
+    if (e < best_e) {  // candidates are visited in increasing i: ties keep the smaller
+      best_e = e;
+      best_i = i;
+    }
+  }
+  const int lane = tid & 31, warp = tid >> 5;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float oe = __shfl_xor_sync(FULL, best_e, o);
+    const int oi = __shfl_xor_sync(FULL, best_i, o);
+    if (oe < best_e || (oe == best_e && oi < best_i)) {
+      best_e = oe;
+      best_i = oi;
+    }
+  }
+  if (lane == 0) {
+    red[warp] = best_e;
+    reinterpret_cast<int*>(red)[32 + warp] = best_i;
+  }
+  __syncthreads();
+  best_e = red[0];
+  best_i = reinterpret_cast<int*>(red)[32];
+  for (int w = 1; w < nt / 32; ++w) {
+    const float oe = red[w];
+    const int oi = reinterpret_cast<int*>(red)[32 + w];
+    if (oe < best_e || (oe == best_e && oi < best_i)) {
+      best_e = oe;
+      best_i = oi;
+    }
+  }
+  const float step = d0 * (1.0f + (float)best_i * (0.25f / FIX_CANDIDATES));
+  __shared__ uint32_t su[16];
+  if (tid < 16) su[tid] = (uint32_t)min(32767, max(0, (int)rintf(c[tid] / step) + 16384));
+  __syncthreads();
+  for (int i = tid; i < 256 * 32; i += nt) {
+    const int x = i >> 5;
+    tab[x * 64 + (i & 31)] = su[x & 15] | (su[x >> 4] << 16);
+  }
+  return step * 65536.0f;
+}
+
+// This lane's part of one vector's score with the fixed-point table; `init`
+// holds -0.75 times the lane's sums of the scaled query (even, odd
+// coordinates).
+template <int S>
+__device__ __forceinline__ float pair16_dot(const Chunk<4> (&ch)[S], const float2 (&q2)[S][8], const char* tab,
+                                            uint32_t lane4, float2 init) {
+  float2 acc = init;
+#pragma unroll
+  for (int s = 0; s < S; ++s) {
+#pragma unroll
+    for (int b = 0; b < 8; ++b) {
+      const uint32_t w = b < 4 ? ch[s].w0 : ch[s].w1;
+      const uint32_t addr = __byte_perm(w, lane4, 0x5504u | ((uint32_t)(b & 3) << 4));
+      const uint32_t e = *reinterpret_cast<const uint32_t*>(tab + addr);
+      const float2 x = make_float2(__uint_as_float(__byte_perm(e, FIX_HALF, 0x7104u)),
+                                   __uint_as_float(__byte_perm(e, FIX_HALF, 0x7324u)));
+      acc = __ffma2_rn(q2[s][b], x, acc);
+    }
+  }
+  return acc.x + acc.y;
+}
+
+// The lookup scan.  Each warp scores 4 consecutive vectors per step (a CTA
+// step covers 32) and issues the next step's code loads before it starts on
+// the current ones (register double buffer), so every warp always has loads
+// in flight.  4-bit codes use a byte-pair table (FIX: the fixed-point one,
+// else the exact fp32 one), other widths a per-code fp32 table replicated in
+// the 32 banks.  With FILT, `bmask` holds one bit per filter block of the
+// query: steps whose block has no allowed tenant are passed over before any
+// of their code bytes is read (Sec. III-B), and in the others a vector whose
+// tenant the query does not allow never enters the top-k.  Filtered and
+// unfiltered scans share every operation on the scores, so filtering by every
+// tenant reproduces the unfiltered result bit for bit.
+template <int BITS, int S, bool FILT, bool FIX>
 __global__ void __launch_bounds__(SCAN_NT, 2)
-k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
-                  const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
-                  const uint32_t* __restrict__ del, int k, int P,
-                  float* __restrict__ cand_s, int* __restrict__ cand_i) {
+k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
+              const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+              const uint32_t* __restrict__ del, const uint32_t* __restrict__ dense,
+              const uint32_t* __restrict__ allow_bits, int words, const uint32_t* __restrict__ bmask,
+              int mask_words, int fblock, int k, int P, float* __restrict__ cand_s, int* __restrict__ cand_i,
+              int* __restrict__ counters, const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids,
+              float* __restrict__ out_scores) {
   constexpr int L = 1 << BITS;
-  constexpr int CB = 2 * BITS;
-  constexpr int V = 4;  // vectors per warp step; a CTA step covers 32
+  constexpr int CB = 2 * BITS;   // bytes of a 16-code chunk
+  constexpr int V = 4;           // vectors per warp step; a CTA step covers 32
+  constexpr bool PAIR = BITS == 4;
+  constexpr int TAB_BYTES = PAIR ? PAIR_TAB_BYTES : L * 32 * 4;
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  float* ctab = reinterpret_cast<float*>(smem_raw);  // [L][32], entry (c, lane) in bank lane
-  float* ls = ctab + L * 32;                          // [P] scores; warp w's list at [w*k, w*k+k)
-  int* li = reinterpret_cast<int*>(ls + P);           // [P] ids
+  float* ls = reinterpret_cast<float*>(smem_raw + TAB_BYTES);  // [P] scores; warp w's list at [w*k, w*k+k)
+  int* li = reinterpret_cast<int*>(ls + P);                     // [P] ids
+  __shared__ float red[64];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int q = blockIdx.y;
-  for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  float qs = 1.0f;  // query pre-scale of the fixed-point table
+  if constexpr (PAIR && FIX) {
+    qs = fix_table_init(reinterpret_cast<uint32_t*>(smem_raw), centroids, red, tid, SCAN_NT);
+  } else if constexpr (PAIR) {
+    pair_table_init(reinterpret_cast<float2*>(smem_raw), centroids, tid, SCAN_NT);
+  } else {
+    float* ctab = reinterpret_cast<float*>(smem_raw);
+    for (int i = tid; i < L * 32; i += SCAN_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  }
   for (int i = tid; i < P; i += SCAN_NT) {
     ls[i] = -INFINITY;
     li[i] = INT_MAX;
   }
+  griddep_wait();  // the rotated queries (and allow bitmaps, block masks) are written
   const int nchunks = d >> 4;
   const float* qq = qrot + (size_t)q * d;
-  float qr[S][16];
+  float qr[PAIR ? 1 : S][16];
+  float2 q2[PAIR ? S : 1][8];
+  float2 init = make_float2(0.f, 0.f);
+  if constexpr (PAIR) {
+    load_q2(q2, qq, nchunks, lane);
+    if constexpr (FIX) {
+      float se = 0.f, so = 0.f;
 #pragma unroll
-  for (int s = 0; s < S; ++s) {
-    const int chunk = lane + 32 * s;
+      for (int s = 0; s < S; ++s)
 #pragma unroll
-    for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+        for (int m = 0; m < 8; ++m) {
+          q2[s][m].x *= qs;
+          q2[s][m].y *= qs;
+          se += q2[s][m].x;
+          so += q2[s][m].y;
+        }
+      init = make_float2(-0.75f * se, -0.75f * so);
+    }
+  } else {
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      const int chunk = lane + 32 * s;
+#pragma unroll
+      for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+    }
   }
   __syncthreads();
 
   const int64_t row_bytes = (int64_t)d * BITS / 8;
+  const uint32_t* ab = FILT ? allow_bits + (size_t)q * words : nullptr;
+  const uint32_t* bm = FILT ? bmask + (size_t)q * mask_words : nullptr;
   float* wl_s = ls + warp * k;
   int* wl_i = li + warp * k;
   int cnt = 0;
@@ -434,11 +571,24 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
   const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
   const int my = (lane >> 3) & 3;  // the vector whose total this lane ends up holding
   const uint32_t lane4 = (uint32_t)lane * 4u;
-  const char* tab = reinterpret_cast<const char*>(ctab);
+  const char* tab = reinterpret_cast<const char*>(smem_raw);
+  // the CTA's next step at or after st whose filter block holds an allowed
+  // tenant (every thread takes the same decisions)
+  auto active = [&](int st) {
+    if constexpr (FILT) {
+      while (st < nsteps) {
+        const int fb = st * (SCAN_WARPS * V) / fblock;
+        if ((__ldg(bm + (fb >> 5)) >> (fb & 31)) & 1u) break;
+        st += gridDim.x;
+      }
+    }
+    return st;
+  };
 
   Chunk<BITS> cur[V][S], nxt[V][S];
   float sc_cur = 0.f, sc_nxt = 0.f;
-  auto load_step = [&](int st, Chunk<BITS> (&buf)[V][S], float& sc) {
+  uint32_t tn_cur = 0, tn_nxt = 0;
+  auto load_step = [&](int st, Chunk<BITS> (&buf)[V][S], float& sc, uint32_t& tn) {
     const int v0 = st * (SCAN_WARPS * V) + warp * V;
 #pragma unroll
     for (int i = 0; i < V; ++i) {
@@ -452,24 +602,35 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
     }
     const int vm = v0 + my;
     sc = 0.f;
-    if (st < nsteps && (lane & 7) == 0 && vm < n) sc = scale ? __ldg(scale + vm) : 1.0f;
+    tn = 0;
+    if (st < nsteps && (lane & 7) == 0 && vm < n) {
+      sc = scale ? __ldg(scale + vm) : 1.0f;
+      if (FILT) tn = __ldg(dense + vm);
+    }
   };
-  int st = blockIdx.x;
-  load_step(st, cur, sc_cur);
-  for (; st < nsteps; st += gridDim.x) {
-    load_step(st + gridDim.x, nxt, sc_nxt);   // next step's loads go out first
+  int st = active(blockIdx.x);
+  load_step(st, cur, sc_cur, tn_cur);
+  while (st < nsteps) {
+    const int st_next = active(st + gridDim.x);
+    load_step(st_next, nxt, sc_nxt, tn_nxt);  // next step's loads go out first
     asm volatile("" ::: "memory");
     const int v0 = st * (SCAN_WARPS * V) + warp * V;
     float p[V];
 #pragma unroll
     for (int i = 0; i < V; ++i) {
-      float acc = 0.f;
+      if constexpr (PAIR && FIX) {
+        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, init);
+      } else if constexpr (PAIR) {
+        p[i] = pair_dot<S>(cur[i], q2, tab, lane4 * 2u);
+      } else {
+        float acc = 0.f;
 #pragma unroll
-      for (int s = 0; s < S; ++s)
+        for (int s = 0; s < S; ++s)
 #pragma unroll
-        for (int t = 0; t < 16; ++t)
-          acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + cur[i][s].off(t, lane4)), acc);
-      p[i] = acc;
+          for (int t = 0; t < 16; ++t)
+            acc = fmaf(qr[s][t], *reinterpret_cast<const float*>(tab + cur[i][s].off(t, lane4)), acc);
+        p[i] = acc;
+      }
     }
     const float total = warp_sum4(p);
     const int vm = v0 + my;
@@ -477,7 +638,8 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
       score = total * sc_cur;
-      cand = better(score, vm, th_s, th_i) && !tombstoned(del, vm);
+      const bool allowed = !FILT || ((__ldg(ab + (tn_cur >> 5)) >> (tn_cur & 31)) & 1u);
+      cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
     unsigned m = __ballot_sync(FULL, cand);
     while (m) {  // in vector order; re-checked against the moving threshold
@@ -499,6 +661,8 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
 #pragma unroll
       for (int s = 0; s < S; ++s) cur[i][s] = nxt[i][s];
     sc_cur = sc_nxt;
+    tn_cur = tn_nxt;
+    st = st_next;
   }
   __syncthreads();
   block_sort(ls, li, P);
@@ -507,78 +671,260 @@ k_scan_lut_stream(const float* __restrict__ qrot, int d, const float* __restrict
     cand_s[o] = ls[i];
     cand_i[o] = li[i];
   }
+  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li);
 }
 
-// Unfiltered 4-bit scan with byte-pair lookups (pair_dot); otherwise as
-// k_scan_lut_stream: 4 vectors per warp step, next step's loads in flight.
-template <int S>
-__global__ void __launch_bounds__(SCAN_NT, 2)
-k_scan_pair_stream(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
-                   const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
-                   const uint32_t* __restrict__ del, int k, int P,
-                   float* __restrict__ cand_s, int* __restrict__ cand_i) {
+// ---------------------------------------------------------------------------
+// The lookup scan fed by bulk copies.  k_scan_stream keeps the next step's
+// codes in registers, so the bytes a warp has in flight are bounded by its
+// registers (about 48 KB per SM), too few to cover HBM latency at full rate.
+// Here each of the CTA's RING_WARPS warps streams its own sequence of 4-vector
+// steps through a private ring of `ns` shared-memory slots: lane 0 queues a
+// 1-D bulk copy (cp.async.bulk, completion counted on the slot's mbarrier)
+// for the step `ns` places ahead as soon as a slot's codes are in registers,
+// so ns slots per warp (about 144 KB per SM) are always on their way.  The
+// scoring is k_scan_stream's, operation for operation.  A step that is not
+// whole (the corpus tail) is read with plain loads.  Waits are bounded: a
+// wait that gives up raises the CTA's abort flag and records its site in the
+// status word; every warp then stops, waits (bounded) for its own copies still
+// in flight, and the CTA ends.
+constexpr int RING_WARPS = 16;
+constexpr int RING_NT = RING_WARPS * 32;
+constexpr int RING_MAX_NS = 4;
+
+__device__ __forceinline__ uint32_t sh_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
+
+__device__ __forceinline__ void ring_mbar_init(uint64_t* bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(sh_u32(bar)));
+}
+
+__device__ __forceinline__ void ring_copy(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(sh_u32(bar)), "r"(bytes) : "memory");
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(sh_u32(dst)), "l"(src), "r"(bytes), "r"(sh_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ bool ring_wait_drain(uint64_t* bar, uint32_t parity) {
+  const long long t0 = clock64();
+  for (uint32_t i = 0;; ++i) {
+    if (mbar_try_wait_parity(bar, parity)) return true;
+    if ((i & 63) == 63 && clock64() - t0 > kWaitCycles) return false;
+  }
+}
+
+// Reads 16-code chunk `chunk` of a row held in shared memory.
+template <int BITS>
+__device__ __forceinline__ void chunk_from_smem(Chunk<BITS>& c, const unsigned char* p);
+template <>
+__device__ __forceinline__ void chunk_from_smem<4>(Chunk<4>& c, const unsigned char* p) {
+  const uint2 v = *reinterpret_cast<const uint2*>(p);
+  c.w0 = v.x;
+  c.w1 = v.y;
+}
+template <>
+__device__ __forceinline__ void chunk_from_smem<2>(Chunk<2>& c, const unsigned char* p) {
+  c.w = *reinterpret_cast<const uint32_t*>(p);
+}
+template <>
+__device__ __forceinline__ void chunk_from_smem<8>(Chunk<8>& c, const unsigned char* p) {
+  c.w = *reinterpret_cast<const uint4*>(p);
+}
+template <>
+__device__ __forceinline__ void chunk_from_smem<3>(Chunk<3>& c, const unsigned char* p) {
+  const unsigned short* h = reinterpret_cast<const unsigned short*>(p);
+  c.v = (uint64_t)h[0] | ((uint64_t)h[1] << 16) | ((uint64_t)h[2] << 32);
+}
+
+template <int BITS, int S, bool FILT, bool FIX>
+__global__ void __launch_bounds__(RING_NT, 1)
+k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ centroids,
+            const uint8_t* __restrict__ codes, const float* __restrict__ scale, int n,
+            const uint32_t* __restrict__ del, const uint32_t* __restrict__ dense,
+            const uint32_t* __restrict__ allow_bits, int words, const uint32_t* __restrict__ bmask, int mask_words,
+            int fblock, int k, int P, int ns, float* __restrict__ cand_s, int* __restrict__ cand_i,
+            int* __restrict__ err, int* __restrict__ counters, const uint64_t* __restrict__ ext,
+            int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+  constexpr int L = 1 << BITS;
+  constexpr int CB = 2 * BITS;
   constexpr int V = 4;
+  constexpr bool PAIR = BITS == 4;
+  constexpr int TAB_BYTES = PAIR ? PAIR_TAB_BYTES : L * 32 * 4;
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  float2* ptab = reinterpret_cast<float2*>(smem_raw);  // [256][32]
-  float* ls = reinterpret_cast<float*>(smem_raw + PAIR_TAB_BYTES);
+  const int rb = d * BITS / 8;
+  const int slot_bytes = V * rb;  // a multiple of 16 for d % 32 == 0
+  unsigned char* ring = smem_raw + TAB_BYTES;
+  float* ls = reinterpret_cast<float*>(ring + (size_t)RING_WARPS * ns * slot_bytes);
   int* li = reinterpret_cast<int*>(ls + P);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(li + P + (P & 1));  // 8-byte aligned
+  __shared__ float red[64];
+  __shared__ int stepq[RING_WARPS][RING_MAX_NS];
+  __shared__ volatile int abort_flag;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int q = blockIdx.y;
-  pair_table_init(ptab, centroids, tid, SCAN_NT);
-  for (int i = tid; i < P; i += SCAN_NT) {
+  const int nsteps = (n + V - 1) / V;  // warp steps of 4 vectors
+  const int wstride = gridDim.x * RING_WARPS;
+  uint64_t* wbar = bars + warp * RING_MAX_NS;
+  unsigned char* wring = ring + (size_t)warp * ns * slot_bytes;
+  const uint32_t* bm = FILT ? bmask + (size_t)q * mask_words : nullptr;
+  // this warp's next step at or after `ws` whose filter block holds an allowed tenant
+  auto active = [&](int ws) {
+    if constexpr (FILT) {
+      while (ws < nsteps) {
+        const int fb = ws * V / fblock;
+        if ((__ldg(bm + (fb >> 5)) >> (fb & 31)) & 1u) break;
+        ws += wstride;
+      }
+    }
+    return ws;
+  };
+  uint32_t pend = 0;  // slots with a copy in flight (lane 0's view, shared by shuffle)
+  auto issue = [&](int ws, int s) {
+    __syncwarp();  // every lane has read the slot's previous codes
+    if (lane == 0) {
+      stepq[warp][s] = ws;
+      if (ws < nsteps && (ws + 1) * V <= n) {
+        ring_copy(wring + s * slot_bytes, codes + (size_t)ws * slot_bytes, (uint32_t)slot_bytes, wbar + s);
+        pend |= 1u << s;
+      }
+    }
+    __syncwarp();
+  };
+  if (tid == 0) abort_flag = 0;
+  if (lane == 0) {
+    for (int s = 0; s < ns; ++s) ring_mbar_init(wbar + s);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  if constexpr (FILT) griddep_wait();  // the block masks steer the first copies
+  // the first ns steps go out before the table is built
+  int next_ws = active(blockIdx.x * RING_WARPS + warp);
+  for (int s = 0; s < ns; ++s) {
+    issue(next_ws, s);
+    next_ws = active(next_ws + wstride);
+  }
+  float qs = 1.0f;
+  if constexpr (PAIR && FIX) {
+    qs = fix_table_init(reinterpret_cast<uint32_t*>(smem_raw), centroids, red, tid, RING_NT);
+  } else if constexpr (PAIR) {
+    pair_table_init(reinterpret_cast<float2*>(smem_raw), centroids, tid, RING_NT);
+  } else {
+    float* ctab = reinterpret_cast<float*>(smem_raw);
+    for (int i = tid; i < L * 32; i += RING_NT) ctab[i] = __ldg(centroids + (i >> 5));
+  }
+  for (int i = tid; i < P; i += RING_NT) {
     ls[i] = -INFINITY;
     li[i] = INT_MAX;
   }
+  if constexpr (!FILT) griddep_wait();  // the rotated queries are written
   const int nchunks = d >> 4;
-  float2 q2[S][8];  // (q'_{2m}, q'_{2m+1}) of the 16 coordinates of chunk lane + 32 s
-  load_q2(q2, qrot + (size_t)q * d, nchunks, lane);
+  const float* qq = qrot + (size_t)q * d;
+  float qr[PAIR ? 1 : S][16];
+  float2 q2[PAIR ? S : 1][8];
+  float2 init = make_float2(0.f, 0.f);
+  if constexpr (PAIR) {
+    load_q2(q2, qq, nchunks, lane);
+    if constexpr (FIX) {
+      float se = 0.f, so = 0.f;
+#pragma unroll
+      for (int s = 0; s < S; ++s)
+#pragma unroll
+        for (int m = 0; m < 8; ++m) {
+          q2[s][m].x *= qs;
+          q2[s][m].y *= qs;
+          se += q2[s][m].x;
+          so += q2[s][m].y;
+        }
+      init = make_float2(-0.75f * se, -0.75f * so);
+    }
+  } else {
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      const int chunk = lane + 32 * s;
+#pragma unroll
+      for (int t = 0; t < 16; ++t) qr[s][t] = chunk < nchunks ? qq[chunk * 16 + t] : 0.f;
+    }
+  }
   __syncthreads();
 
-  const int64_t row_bytes = (int64_t)d / 2;
+  const uint32_t* ab = FILT ? allow_bits + (size_t)q * words : nullptr;
   float* wl_s = ls + warp * k;
   int* wl_i = li + warp * k;
   int cnt = 0;
   float th_s = -INFINITY;
   int th_i = INT_MAX;
-  const int nsteps = (n + SCAN_WARPS * V - 1) / (SCAN_WARPS * V);
   const int my = (lane >> 3) & 3;
-  const uint32_t lane8 = (uint32_t)lane * 8u;
-  const char* tab = reinterpret_cast<const char*>(ptab);
-
-  Chunk<4> cur[V][S], nxt[V][S];
-  float sc_cur = 0.f, sc_nxt = 0.f;
-  auto load_step = [&](int st, Chunk<4> (&buf)[V][S], float& sc) {
-    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+  const uint32_t lane4 = (uint32_t)lane * 4u;
+  const char* tab = reinterpret_cast<const char*>(smem_raw);
+  uint32_t par = 0;  // phase parity of each slot's next completion
+  for (int it = 0;; ++it) {
+    const int s = it % ns;
+    const int ws = stepq[warp][s];
+    if (ws >= nsteps) break;
+    if (abort_flag) break;
+    const int v0 = ws * V;
+    Chunk<BITS> cur[V][S];
+    if (v0 + V <= n) {  // whole step: its codes came by bulk copy
+      bool ok = true;
+      if (lane == 0) ok = bounded_wait(wbar + s, (par >> s) & 1u, &abort_flag, err, 20, kWaitCycles);
+      ok = __shfl_sync(FULL, ok ? 1 : 0, 0) != 0;
+      if (!ok) break;
+      par ^= 1u << s;
+      pend &= ~(1u << s);
+      __syncwarp();
+      const unsigned char* src = wring + s * slot_bytes;
 #pragma unroll
-    for (int i = 0; i < V; ++i) {
-      const uint8_t* row = codes + (size_t)(v0 + i) * row_bytes;
+      for (int i = 0; i < V; ++i)
 #pragma unroll
-      for (int s = 0; s < S; ++s) {
-        const int chunk = lane + 32 * s;
-        if (st < nsteps && v0 + i < n && chunk < nchunks) buf[i][s].load(row + chunk * 8);
-        else buf[i][s].zero();
-      }
+        for (int c = 0; c < S; ++c) {
+          const int chunk = lane + 32 * c;
+          if (chunk < nchunks) chunk_from_smem<BITS>(cur[i][c], src + i * rb + chunk * CB);
+          else cur[i][c].zero();
+        }
+    } else {
+#pragma unroll
+      for (int i = 0; i < V; ++i)
+#pragma unroll
+        for (int c = 0; c < S; ++c) {
+          const int chunk = lane + 32 * c;
+          if (v0 + i < n && chunk < nchunks) cur[i][c].load(codes + (size_t)(v0 + i) * rb + chunk * CB);
+          else cur[i][c].zero();
+        }
     }
     const int vm = v0 + my;
-    sc = 0.f;
-    if (st < nsteps && (lane & 7) == 0 && vm < n) sc = scale ? __ldg(scale + vm) : 1.0f;
-  };
-  int st = blockIdx.x;
-  load_step(st, cur, sc_cur);
-  for (; st < nsteps; st += gridDim.x) {
-    load_step(st + gridDim.x, nxt, sc_nxt);
-    asm volatile("" ::: "memory");
-    const int v0 = st * (SCAN_WARPS * V) + warp * V;
+    float sc = 0.f;
+    uint32_t tn = 0;
+    if ((lane & 7) == 0 && vm < n) {
+      sc = scale ? __ldg(scale + vm) : 1.0f;
+      if (FILT) tn = __ldg(dense + vm);
+    }
+    // the slot's codes are in registers: queue the step ns places ahead
+    issue(next_ws, s);
+    next_ws = active(next_ws + wstride);
     float p[V];
 #pragma unroll
-    for (int i = 0; i < V; ++i) p[i] = pair_dot<S>(cur[i], q2, tab, lane8);
+    for (int i = 0; i < V; ++i) {
+      if constexpr (PAIR && FIX) {
+        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, init);
+      } else if constexpr (PAIR) {
+        p[i] = pair_dot<S>(cur[i], q2, tab, lane4 * 2u);
+      } else {
+        float acc = 0.f;
+#pragma unroll
+        for (int c = 0; c < S; ++c)
+#pragma unroll
+          for (int t = 0; t < 16; ++t)
+            acc = fmaf(qr[c][t], *reinterpret_cast<const float*>(tab + cur[i][c].off(t, lane4)), acc);
+        p[i] = acc;
+      }
+    }
     const float total = warp_sum4(p);
-    const int vm = v0 + my;
     float score = -INFINITY;
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
-      score = total * sc_cur;
-      cand = better(score, vm, th_s, th_i) && !tombstoned(del, vm);
+      score = total * sc;
+      const bool allowed = !FILT || ((__ldg(ab + (tn >> 5)) >> (tn & 31)) & 1u);
+      cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
     unsigned m = __ballot_sync(FULL, cand);
     while (m) {
@@ -595,19 +941,19 @@ k_scan_pair_stream(const float* __restrict__ qrot, int d, const float* __restric
         }
       }
     }
-#pragma unroll
-    for (int i = 0; i < V; ++i)
-#pragma unroll
-      for (int s = 0; s < S; ++s) cur[i][s] = nxt[i][s];
-    sc_cur = sc_nxt;
   }
+  // never leave with copies in flight (only after an abort can there be any)
+  if (lane == 0)
+    for (int s = 0; s < ns; ++s)
+      if ((pend >> s) & 1u) ring_wait_drain(wbar + s, (par >> s) & 1u);
   __syncthreads();
   block_sort(ls, li, P);
-  for (int i = tid; i < k; i += SCAN_NT) {
+  for (int i = tid; i < k; i += RING_NT) {
     const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
     cand_s[o] = ls[i];
     cand_i[o] = li[i];
   }
+  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li);
 }
 
 // Merges the candidates of each query into its sorted top-k, P - k at a time.
@@ -655,118 +1001,17 @@ k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t 
   }
 }
 
-// Merge of per-CTA candidate lists that are each sorted best first and hold
-// exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
-// any one list is beaten or matched by that list's k entries, so the global
-// k-th best is at least as good as the best such T and worse candidates are
-// skipped at once.  Each warp keeps a sorted top-k of its share of the rest
-// (ballot, then one warp-wide insertion per candidate that still beats the
-// warp's k-th); warp 0 then folds the sorted warp lists into the result,
-// leaving each list at its first entry that no longer qualifies.  With an
-// id map the result rows are written as their external ids.
+// Merge of every scan CTA's list, one block per query (the tensor-core scan's
+// lists; the lookup scans merge in their own last CTA).
 __global__ void __launch_bounds__(1024)
 k_merge_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k,
               const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  const int nwarps = blockDim.x >> 5;
   float* ws = reinterpret_cast<float*>(smem_raw);  // [nwarps][k]
-  int* wi = reinterpret_cast<int*>(ws + nwarps * k);
-  __shared__ float red_s[32];
-  __shared__ int red_i[32];
+  int* wi = reinterpret_cast<int*>(ws + (blockDim.x >> 5) * k);
   const int64_t q = blockIdx.x;
-  const int total = nlists * k;
-  const float* cs = cand_s + q * total;
-  const int* ci = cand_i + q * total;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // 1. T = best k-th entry over the lists
-  float ts = -INFINITY;
-  int ti = INT_MAX;
-  for (int l = tid; l < nlists; l += blockDim.x) {
-    const float a = cs[l * k + k - 1];
-    const int b = ci[l * k + k - 1];
-    if (better(a, b, ts, ti)) {
-      ts = a;
-      ti = b;
-    }
-  }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float a = __shfl_xor_sync(FULL, ts, o);
-    const int b = __shfl_xor_sync(FULL, ti, o);
-    if (better(a, b, ts, ti)) {
-      ts = a;
-      ti = b;
-    }
-  }
-  if (lane == 0) {
-    red_s[warp] = ts;
-    red_i[warp] = ti;
-  }
-  for (int i = lane; i < k; i += 32) {
-    ws[warp * k + i] = -INFINITY;
-    wi[warp * k + i] = INT_MAX;
-  }
-  __syncthreads();
-  ts = red_s[0];
-  ti = red_i[0];
-  for (int w = 1; w < nwarps; ++w)
-    if (better(red_s[w], red_i[w], ts, ti)) {
-      ts = red_s[w];
-      ti = red_i[w];
-    }
-  // 2. per-warp sorted top-k of the candidates at least as good as T
-  float* ls = ws + warp * k;
-  int* li = wi + warp * k;
-  int cnt = 0;
-  float th_s = -INFINITY;
-  int th_i = INT_MAX;
-  for (int c0 = warp * 32; c0 < total; c0 += blockDim.x) {
-    const int c = c0 + lane;
-    float a = -INFINITY;
-    int b = INT_MAX;
-    if (c < total) {
-      a = cs[c];
-      b = ci[c];
-    }
-    const bool cand = b != INT_MAX && !better(ts, ti, a, b) && better(a, b, th_s, th_i);
-    unsigned m = __ballot_sync(FULL, cand);
-    while (m) {
-      const int src = __ffs(m) - 1;
-      m &= m - 1;
-      const float sv = __shfl_sync(FULL, a, src);
-      const int iv = __shfl_sync(FULL, b, src);
-      if (better(sv, iv, th_s, th_i)) {
-        warp_insert(ls, li, k, cnt, sv, iv);
-        cnt = min(cnt + 1, k);
-        if (cnt == k) {
-          th_s = ls[k - 1];
-          th_i = li[k - 1];
-        }
-      }
-    }
-  }
-  __syncthreads();
-  // 3. warp 0 folds the other warps' sorted lists into its own
-  if (warp == 0) {
-    for (int w = 1; w < nwarps; ++w) {
-      for (int i = 0; i < k; ++i) {
-        const float sv = ws[w * k + i];
-        const int iv = wi[w * k + i];
-        if (iv == INT_MAX || !better(sv, iv, th_s, th_i)) break;  // sorted: the rest are worse
-        warp_insert(ls, li, k, cnt, sv, iv);
-        cnt = min(cnt + 1, k);
-        if (cnt == k) {
-          th_s = ls[k - 1];
-          th_i = li[k - 1];
-        }
-      }
-    }
-    for (int i = lane; i < k; i += 32) {
-      const bool empty = li[i] == INT_MAX;
-      out_ids[q * k + i] = empty ? -1 : ext ? (int64_t)__ldg(ext + li[i]) : (int64_t)li[i];
-      out_scores[q * k + i] = empty ? -INFINITY : ls[i];
-    }
-  }
+  merge_lists_block(cand_s + q * nlists * k, cand_i + q * nlists * k, nlists, k, ext, out_ids + q * k,
+                    out_scores + q * k, ws, wi);
 }
 
 __device__ __forceinline__ int64_t find_tenant(const uint32_t* __restrict__ tenants, int64_t T, uint32_t x) {
@@ -790,6 +1035,35 @@ __global__ void k_allow_bits(const uint32_t* __restrict__ tenants, int64_t T, in
     const int64_t pos = find_tenant(tenants, T, ids[j]);
     if (pos >= 0) atomicOr(o + (pos >> 5), 1u << (pos & 31));
   }
+}
+
+// Bit b of query q's block mask: filter block b holds a tenant the query
+// allows (its tenant bitmap shares a bit with the query's allow bitmap).  A
+// warp owns one mask word (32 blocks): lane w reads word w of each block's
+// bitmap, all 32 blocks' loads in flight at once.
+__global__ void __launch_bounds__(256)
+k_block_mask(const uint32_t* __restrict__ block_bits, int64_t nblocks, int words, const uint32_t* __restrict__ allow,
+             int mask_words, uint32_t* __restrict__ mask) {
+  const int64_t q = blockIdx.y;
+  const int lane = threadIdx.x & 31;
+  griddep_launch_dependents();
+  const int64_t mw = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (mw >= mask_words) return;  // whole warps
+  const uint32_t* a = allow + q * words;
+  uint32_t bits = 0;
+  for (int w0 = 0; w0 < words; w0 += 32) {
+    const int w = w0 + lane;
+    const uint32_t aw = w < words ? __ldg(a + w) : 0u;
+    uint32_t x[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const int64_t b = mw * 32 + j;
+      x[j] = (w < words && b < nblocks) ? (__ldg(block_bits + b * words + w) & aw) : 0u;
+    }
+#pragma unroll
+    for (int j = 0; j < 32; ++j) bits |= (__any_sync(FULL, x[j] != 0u) ? 1u : 0u) << j;
+  }
+  if (lane == 0) mask[q * mask_words + mw] = bits;
 }
 
 // Rows v0 .. v0+n-1 get their dense tenant index and set their bit in their
@@ -819,43 +1093,112 @@ int next_pow2(int x) {
   return p;
 }
 
-template <int BITS, int S>
-cudaError_t scan_lut_typed(dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
-                           const float* centroids, const uint8_t* codes, const float* scale, int n,
-                           const uint32_t* del, const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
-                           const uint32_t* allow, int k, int P, float* cs, int* ci) {
-  cudaError_t e;
-  if (BITS == 4 && !allow) {
-    const size_t psmem = (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int));
-    e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_pair_stream<S>), (int)psmem);
+struct ScanArgs {
+  const float* qrot;
+  int d;
+  const float* centroids;
+  const uint8_t* codes;
+  const float* scale;
+  int n;
+  const uint32_t* del;
+  const uint32_t* dense;
+  const uint32_t* allow;
+  int words;
+  const uint32_t* bmask;
+  int mask_words;
+  int fblock;
+  int k, P;
+  float* cs;
+  int* ci;
+  int* err;
+  int* counters;
+  const uint64_t* ext;
+  int64_t* out_ids;
+  float* out_scores;
+  bool pdl;
+};
+
+// Launches `kernel`, with programmatic stream serialization when `pdl` (the
+// kernel then overlaps the tail of the one before it and waits for it with
+// griddep_wait before reading its results).
+template <typename... Params, typename... Args>
+cudaError_t launch_maybe_pdl(bool pdl, void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+// Dynamic shared memory of the ring scan with `ns` slots per warp.
+constexpr size_t kRingSmemMax = 232448 - 2048;  // 227 KB less the static arrays
+size_t ring_smem(int bits, int d, int P, int ns) {
+  const size_t tab = bits == 4 ? (size_t)PAIR_TAB_BYTES : (size_t)(1 << bits) * 32 * sizeof(float);
+  return tab + (size_t)RING_WARPS * ns * 4 * (d * bits / 8) + (size_t)P * (sizeof(float) + sizeof(int)) +
+         (size_t)RING_WARPS * RING_MAX_NS * sizeof(uint64_t);
+}
+
+// Slots per warp of the ring scan (as many as fit, at most RING_MAX_NS), or 0
+// for the register-fed k_scan_stream.  Measured on GB300 (999,000 x 1536,
+// batch 1): the ring reads 3-bit codes 23% faster (1.69 vs 1.37 TB/s), but for
+// 2- and 4-bit codes the scan is bound by the shared-memory datapath the
+// lookups use, and the ring's copies add to that traffic (4-bit 2.83 vs 3.55
+// TB/s, 2-bit 1.18 vs 1.28), so only 3-bit codes take it.
+int ring_slots(int bits, int d, int k) {
+  if (bits != 3) return 0;
+  const int P = next_pow2(RING_WARPS * k);
+  for (int ns = RING_MAX_NS; ns >= 2; --ns)
+    if (ring_smem(bits, d, P, ns) <= kRingSmemMax) return ns;
+  return 0;
+}
+
+template <int BITS, int S, bool FILT, bool FIX>
+cudaError_t scan_typed(dim3 grid, size_t smem, cudaStream_t s, const ScanArgs& a) {
+  const int ns = BITS == 3 ? ring_slots(BITS, a.d, a.k) : 0;
+  if constexpr (BITS == 3) if (ns >= 2) {
+    const int P = next_pow2(RING_WARPS * a.k);
+    const size_t rsmem = ring_smem(BITS, a.d, P, ns);
+    const void* fn = reinterpret_cast<const void*>(k_scan_ring<BITS, S, FILT, FIX>);
+    const cudaError_t e = set_max_dynamic_smem(fn, (int)rsmem);
     if (e != cudaSuccess) return e;
-    k_scan_pair_stream<S><<<grid, SCAN_NT, psmem, s>>>(qrot, d, centroids, codes, scale, n, del, k, P, cs, ci);
-    return cudaGetLastError();
+    return launch_maybe_pdl(a.pdl, k_scan_ring<BITS, S, FILT, FIX>, grid, dim3(RING_NT), rsmem, s, a.qrot, a.d,
+                            a.centroids, a.codes, a.scale, a.n, a.del, a.dense, a.allow, a.words, a.bmask,
+                            a.mask_words, a.fblock, a.k, P, ns, a.cs, a.ci, a.err, a.counters, a.ext, a.out_ids,
+                            a.out_scores);
   }
-  if (!allow) {
-    e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut_stream<BITS, S>), (int)smem);
-    if (e != cudaSuccess) return e;
-    k_scan_lut_stream<BITS, S><<<grid, SCAN_NT, smem, s>>>(qrot, d, centroids, codes, scale, n, del, k, P, cs, ci);
-    return cudaGetLastError();
-  }
-  const size_t fsmem = BITS == 4 ? (size_t)PAIR_TAB_BYTES + (size_t)P * (sizeof(float) + sizeof(int)) : smem;
-  e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_lut<BITS, S>), (int)fsmem);
+  const void* fn = reinterpret_cast<const void*>(k_scan_stream<BITS, S, FILT, FIX>);
+  const cudaError_t e = set_max_dynamic_smem(fn, (int)smem);
   if (e != cudaSuccess) return e;
-  k_scan_lut<BITS, S><<<grid, SCAN_NT, fsmem, s>>>(qrot, d, centroids, codes, scale, n, del, dense, block_bits,
-                                                   words, fblock, allow, k, P, cs, ci);
-  return cudaGetLastError();
+  return launch_maybe_pdl(a.pdl, k_scan_stream<BITS, S, FILT, FIX>, grid, dim3(SCAN_NT), smem, s, a.qrot, a.d,
+                          a.centroids, a.codes, a.scale, a.n, a.del, a.dense, a.allow, a.words, a.bmask,
+                          a.mask_words, a.fblock, a.k, a.P, a.cs, a.ci, a.counters, a.ext, a.out_ids, a.out_scores);
+}
+
+template <int BITS, int S>
+cudaError_t scan_variant(bool filt, bool fix, dim3 grid, size_t smem, cudaStream_t s, const ScanArgs& a) {
+  if constexpr (BITS == 4) {
+    if (fix)
+      return filt ? scan_typed<BITS, S, true, true>(grid, smem, s, a) : scan_typed<BITS, S, false, true>(grid, smem, s, a);
+  } else {
+    (void)fix;
+  }
+  return filt ? scan_typed<BITS, S, true, false>(grid, smem, s, a) : scan_typed<BITS, S, false, false>(grid, smem, s, a);
 }
 
 template <int BITS>
-cudaError_t scan_lut_bits(int S, dim3 grid, size_t smem, cudaStream_t s, const float* qrot, int d,
-                          const float* centroids, const uint8_t* codes, const float* scale, int n,
-                          const uint32_t* del, const uint32_t* dense, const uint32_t* block_bits, int words, int fblock,
-                          const uint32_t* allow, int k, int P, float* cs, int* ci) {
+cudaError_t scan_bits(int S, bool filt, bool fix, dim3 grid, size_t smem, cudaStream_t s, const ScanArgs& a) {
   switch (S) {
-    case 1: return scan_lut_typed<BITS, 1>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 2: return scan_lut_typed<BITS, 2>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 3: return scan_lut_typed<BITS, 3>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
-    case 4: return scan_lut_typed<BITS, 4>(grid, smem, s, qrot, d, centroids, codes, scale, n, del, dense, block_bits, words, fblock, allow, k, P, cs, ci);
+    case 1: return scan_variant<BITS, 1>(filt, fix, grid, smem, s, a);
+    case 2: return scan_variant<BITS, 2>(filt, fix, grid, smem, s, a);
+    case 3: return scan_variant<BITS, 3>(filt, fix, grid, smem, s, a);
+    case 4: return scan_variant<BITS, 4>(filt, fix, grid, smem, s, a);
     default: return cudaErrorInvalidValue;
   }
 }
@@ -863,11 +1206,9 @@ cudaError_t scan_lut_bits(int S, dim3 grid, size_t smem, cudaStream_t s, const f
 }  // namespace
 
 int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d) {
-  (void)k;
-  (void)bits;
-  (void)d;
-  // one resident wave (two CTAs per SM) for a single query
-  const int64_t target = (int64_t)device_sm_count() * 2;
+  // one resident wave for a single query: one ring-scan CTA per SM, or two
+  // register-fed CTAs
+  const int64_t target = (int64_t)device_sm_count() * (ring_slots(bits, d, k) >= 2 ? 1 : 2);
   int64_t gx = (target + nq - 1) / (nq > 0 ? nq : 1);
   const int64_t blocks = (n + 31) / 32;
   if (gx > blocks) gx = blocks;
@@ -875,26 +1216,37 @@ int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d) {
   return (int)gx;
 }
 
+int filter_mask_words(const FilterDev& f) {
+  const int64_t nblocks = (f.n + f.block - 1) / f.block;
+  return (int)((nblocks + 31) / 32);
+}
+
 cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
-                            const FilterDev* f, const uint32_t* allow_bits, int k, int grid_x, float* cand_s,
-                            int32_t* cand_i, cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1) {
+                            const FilterDev* f, const uint32_t* allow_bits, const uint32_t* bmask, bool fix,
+                            int k, int grid_x, float* cand_s, int32_t* cand_i, int* err, int* counters,
+                            const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s,
+                            cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
   const int S = (d + 511) / 512;
   const int P = next_pow2(SCAN_WARPS * k);
-  const size_t smem = (size_t)(1 << bits) * 32 * sizeof(float) + (size_t)P * (sizeof(float) + sizeof(int));
+  const size_t tab = bits == 4 ? (size_t)PAIR_TAB_BYTES : (size_t)(1 << bits) * 32 * sizeof(float);
+  const size_t smem = tab + (size_t)P * (sizeof(float) + sizeof(int));
   const dim3 grid((unsigned)grid_x, (unsigned)nq);
-  const uint32_t* dense = f ? f->dense : nullptr;
-  const uint32_t* bb = f ? f->block_bits : nullptr;
-  const int words = f ? f->words : 0;
-  const int fblock = f ? f->block : 64;
+  ScanArgs a{qrot, d, centroids, codes, scale, (int)n, del,
+             f ? f->dense : nullptr, allow_bits, f ? f->words : 0, bmask, f ? filter_mask_words(*f) : 0,
+             f ? f->block : 64, k, P, cand_s, cand_i, err, counters, ext, out_ids, out_scores,
+             // overlap with the kernel before (not on the legacy default stream, and not
+             // between profiling events, which would serialise the two anyway)
+             s != nullptr && ev0 == nullptr};
+  const bool filt = f != nullptr;
   cudaError_t e;
   if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;
   switch (bits) {
-    case 2: e = scan_lut_bits<2>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 3: e = scan_lut_bits<3>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 4: e = scan_lut_bits<4>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
-    case 8: e = scan_lut_bits<8>(S, grid, smem, s, qrot, d, centroids, codes, scale, (int)n, del, dense, bb, words, fblock, allow_bits, k, P, cand_s, cand_i); break;
+    case 2: e = scan_bits<2>(S, filt, fix, grid, smem, s, a); break;
+    case 3: e = scan_bits<3>(S, filt, fix, grid, smem, s, a); break;
+    case 4: e = scan_bits<4>(S, filt, fix, grid, smem, s, a); break;
+    case 8: e = scan_bits<8>(S, filt, fix, grid, smem, s, a); break;
     default: e = cudaErrorInvalidValue;
   }
   if (e != cudaSuccess) return e;
@@ -932,6 +1284,15 @@ cudaError_t launch_allow_bits(const FilterDev& f, const int64_t* allow_off,
                               cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   k_allow_bits<<<(unsigned)nq, 128, 0, s>>>(f.tenants, f.n_tenants, f.words, allow_off, allow_tenants, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_block_mask(const FilterDev& f, const uint32_t* allow, int64_t nq, uint32_t* mask,
+                              cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  const int mw = filter_mask_words(f);
+  const dim3 grid((unsigned)((mw + 7) / 8), (unsigned)nq);
+  k_block_mask<<<grid, 256, 0, s>>>(f.block_bits, (f.n + f.block - 1) / f.block, f.words, allow, mw, mask);
   return cudaGetLastError();
 }
 

@@ -6,8 +6,9 @@
 // outputs from someone else, or a latency-critical serving loop that must
 // not call cudaMalloc/cudaFree (an allocation can block, synchronise the
 // device or fail under memory pressure in the middle of a request).  For them
-// this entry point keeps its scratch (rotated queries, allow bitmaps, per-CTA
-// top-k candidates) in one file-scope device array of kStaticScratchBytes.  It
+// this entry point keeps its scratch (status word, merge counters, rotated
+// queries, allow bitmaps, block masks, per-CTA top-k candidates) in one
+// file-scope device array of kStaticScratchBytes.  It
 // allocates nothing and calls no allocating routine.
 //
 // The array's name in host code is only a host-side stand-in, never a device
@@ -82,13 +83,16 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
     f = &filter->f;
   }
 
-  // scratch plan: rotated queries | allow bitmaps | candidate scores | candidate ids
+  // scratch plan: status word | merge counters | rotated queries | allow bitmaps | block masks |
+  // candidate scores | ids
   const int gx = tq::scan_lut_grid_x(nq, n, k, bits, d);
+  const size_t head = 256 + tq::up256((size_t)nq * sizeof(int));
   const size_t rot = tq::up256((size_t)nq * d * sizeof(float));
   const size_t allow = f ? tq::up256((size_t)nq * f->words * sizeof(uint32_t)) : 0;
+  const size_t mask = f ? tq::up256((size_t)nq * tq::filter_mask_words(*f) * sizeof(uint32_t)) : 0;
   const size_t cs = tq::up256((size_t)nq * gx * k * sizeof(float));
   const size_t ci = tq::up256((size_t)nq * gx * k * sizeof(int32_t));
-  const size_t need = rot + allow + cs + ci;
+  const size_t need = head + rot + allow + mask + cs + ci;
   if (need > tq::kStaticScratchBytes)
     return fail(TQ_EINVAL,
                 "tq_search_static: these sizes need %zu bytes of scratch but the static scratch holds %zu "
@@ -118,17 +122,21 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
   }
 
   cudaStream_t s = (cudaStream_t)stream;
-  char* base = static_cast<char*>(scratch);
+  int* status = static_cast<int*>(scratch);  // the scans' bounded waits report here
+  int* counters = reinterpret_cast<int*>(static_cast<char*>(scratch) + 256);
+  char* base = static_cast<char*>(scratch) + head;
   float* qrot = reinterpret_cast<float*>(base);
   uint32_t* allow_bits = f ? reinterpret_cast<uint32_t*>(base + rot) : nullptr;
-  float* cand_s = reinterpret_cast<float*>(base + rot + allow);
-  int32_t* cand_i = reinterpret_cast<int32_t*>(base + rot + allow + cs);
-  e = tq::launch_rotate(Q, nq, d, R, qrot, nullptr, s);
+  uint32_t* bmask = f ? reinterpret_cast<uint32_t*>(base + rot + allow) : nullptr;
+  float* cand_s = reinterpret_cast<float*>(base + rot + allow + mask);
+  int32_t* cand_i = reinterpret_cast<int32_t*>(base + rot + allow + mask + cs);
+  e = tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);
   if (e == cudaSuccess && f) e = tq::launch_allow_bits(*f, allow_off, allow_tenants, nq, allow_bits, s);
+  if (e == cudaSuccess && f) e = tq::launch_block_mask(*f, allow_bits, nq, bmask, s);
   if (e == cudaSuccess)
-    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, nullptr, f, allow_bits, k, gx, cand_s,
-                            cand_i, s, nullptr, nullptr);
-  if (e == cudaSuccess) e = tq::launch_merge(cand_s, cand_i, nq, gx * k, k, nullptr, out_ids, out_scores, s);
+    e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, nullptr, f, allow_bits, bmask,
+                            tq::search_path() == TQ_PATH_LUT_FIXED && d >= tq::kFixMinD, k, gx, cand_s, cand_i,
+                            status, counters, nullptr, out_ids, out_scores, s, nullptr, nullptr);
   if (e != cudaSuccess) return fail(TQ_ECUDA, "tq_search_static: %s", cudaGetErrorString(e));
   return tq::ok();
 }

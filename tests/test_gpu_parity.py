@@ -105,7 +105,7 @@ def _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, **kw):
     return ids.cpu().numpy(), sc.cpu().numpy()
 
 
-@pytest.mark.parametrize("path", ["lut", "mma"])
+@pytest.mark.parametrize("path", ["lut", "lut_fixed", "mma"])
 def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
     torch, dev = torch_dev
     tq = cuda_lib
@@ -119,7 +119,7 @@ def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
         tq.set_search_path("auto")
     ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"])
     allowed = np.ones_like(ref.scores64, dtype=bool)
-    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_LUT if path == "lut" else TOL_MMA)
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_MMA if path == "mma" else TOL_LUT)
     exact, _ = O.exact_knn(c["X"], c["Q"], k)
     assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
 
@@ -168,24 +168,59 @@ def test_search_bit_widths(cuda_lib, torch_dev, bits, path):
 
 
 @pytest.mark.parametrize("d,n,nq,k", [(32, 5, 3, 10), (64, 64 * 3 + 17, 9, 7), (96, 1000, 8, 1),
-                                      (160, 777, 2, 256), (2048, 1500, 1, 5)])
-def test_search_shapes_and_edges(cuda_lib, torch_dev, d, n, nq, k):
+                                      (160, 777, 2, 256), (512, 2000, 3, 10), (2048, 1500, 1, 5)])
+@pytest.mark.parametrize("path", ["auto", "lut_fixed"])
+def test_search_shapes_and_edges(cuda_lib, torch_dev, d, n, nq, k, path):
     """n below one block, ragged blocks, small d (lanes idle), k = 1 and 256,
-    the GEMV (nq <= 8) and GEMM (nq > 8) query rotations, d = 2048."""
+    the GEMV (nq <= 8) and GEMM (nq > 8) query rotations, d = 2048, both
+    4-bit tables (the fixed-point one from d = 512 on).  The exact table
+    takes raw Gaussian queries (norms up to 45); the fixed-point one takes
+    unit queries, as in the workloads (its error scales with the query norm)."""
     torch, dev = torch_dev
     tq = cuda_lib
     bits = 4
-    rng = np.random.default_rng(d + n)
     packed = synth.random_codes(n, d * bits // 8, seed=d)
     scale = synth.random_scales(n, seed=n)
     scale[0] = 0.0
     R = O.rotation(d, 5).astype(np.float32)
     c32, _ = _cb(d, bits)
     Q = synth.gaussian_rows(nq, d, seed=nq)
-    ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    if path == "lut_fixed":
+        Q /= np.linalg.norm(Q, axis=1, keepdims=True)
+    tq.set_search_path(path)
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    finally:
+        tq.set_search_path("auto")
     ref = O.search(Q, R, c32, bits, packed, scale, k, d)
     check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_LUT)
-    del rng
+
+
+@pytest.mark.parametrize("d,marginal,bound", [(512, "beta", 1e-5), (1536, "beta", 3e-6), (1536, "gauss", 3e-6)])
+def test_fixed_point_table_error(cuda_lib, torch_dev, d, marginal, bound):
+    """The fixed-point 4-bit table against the float64 oracle on unit queries:
+    256 results per query, each within `bound` of the oracle's score, and the
+    exact fp32 table within 1e-6.  The fixed-point error is the centroids'
+    rounding to the table's step (about 2^-16 of the largest centroid, which
+    grows as 1/sqrt(d)) weighted by the rotated query: about 1.2e-6 rms at
+    d = 512 and 2.5e-7 at d = 1536 for random codes."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    bits, n, nq, k = 4, 6000, 24, 256
+    packed = synth.random_codes(n, d * bits // 8, seed=d + 1)
+    scale = synth.random_scales(n, seed=d + 1)
+    R = O.rotation(d, 6).astype(np.float32)
+    c32 = _cb(d, bits, marginal)[0]
+    Q = synth.gaussian_rows(nq, d, seed=d + 2)
+    Q /= np.linalg.norm(Q, axis=1, keepdims=True)
+    ref = O.search(Q, R, c32, bits, packed, scale, k, d)
+    for path, tol in (("lut_fixed", bound), ("lut", 1e-6)):
+        tq.set_search_path(path)
+        try:
+            ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+        finally:
+            tq.set_search_path("auto")
+        check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, tol)
 
 
 def test_search_unit_scale_and_ties(cuda_lib, torch_dev):
@@ -241,6 +276,31 @@ def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
     exact, _ = O.exact_knn(c["X"], c["Q"], k, tid, off, allow)
     assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
     filt.close()
+
+
+@pytest.mark.parametrize("path", ["lut", "lut_fixed"])
+def test_filter_every_tenant_equals_unfiltered(cuda_lib, torch_dev, filtered_corpus, path):
+    """At d = 1536, with both 4-bit tables: allowing every tenant gives the
+    unfiltered search bit for bit (the same operations on every score)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    k, nq = 10, 40
+    tid, values = synth.zipf_tenants(c["n"], 100)
+    off = np.arange(nq + 1, dtype=np.int64) * len(values)
+    allow = np.tile(values, nq)
+    filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=64)
+    tq.set_search_path(path)
+    try:
+        ids_f, sc_f = _gpu_search(tq, torch, dev, c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                                  c["enc"].scale, k, filter=filt, allow_off=_t(torch, dev, off),
+                                  allow_tenants=_t(torch, dev, allow.view(np.int32)))
+        ids_u, sc_u = _gpu_search(tq, torch, dev, c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                                  c["enc"].scale, k)
+    finally:
+        tq.set_search_path("auto")
+        filt.close()
+    assert np.array_equal(ids_f, ids_u) and np.array_equal(sc_f, sc_u)
 
 
 def test_filter_edge_cases(cuda_lib, torch_dev):
@@ -371,3 +431,56 @@ def test_search_on_side_stream_keeps_its_temporaries(cuda_lib, torch_dev):
             del junk
     finally:
         tq.set_search_path("auto")
+
+
+@pytest.mark.parametrize("bits,filtered,nq", [(4, False, 1), (4, False, 5), (3, False, 2), (2, False, 1),
+                                              (4, True, 3), (8, True, 1)])
+def test_search_on_created_stream_matches_default_stream(cuda_lib, torch_dev, filtered_corpus, bits, filtered, nq):
+    """On a created stream the lookup scan is launched as a programmatic
+    dependent of the kernel before it (its prologue overlaps that kernel's
+    tail) and merges in its last CTA; the results equal the default-stream
+    search (no overlap) bit for bit, in back-to-back searches and with the
+    scan bracketed by profiling events."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    d, n, k = c["d"], 12_000, 10
+    packed = synth.random_codes(n, d * bits // 8, seed=bits + nq)
+    scale = synth.random_scales(n, seed=bits)
+    c32, _ = _cb(d, bits)
+    Qd, Rd, cd = _t(torch, dev, c["Q"][:nq]), _t(torch, dev, c["R"]), _t(torch, dev, c32)
+    pd, sd = _t(torch, dev, packed), _t(torch, dev, scale)
+    kw = {}
+    if filtered:
+        tid, values = synth.zipf_tenants(n, 100)
+        off, allow = synth.allowlists(np.arange(nq), tid, values)
+        kw = dict(filter=tq.Filter(_t(torch, dev, tid.view(np.int32))), allow_off=_t(torch, dev, off),
+                  allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    tq.set_search_path("lut")
+    try:
+        want_i, want_s = tq.search(Qd, Rd, cd, bits, pd, sd, k, **kw)
+        torch.cuda.synchronize()
+        side = torch.cuda.Stream(device=dev)
+        side.wait_stream(torch.cuda.current_stream())
+        ws = torch.empty(tq.search_workspace(nq, n, d, bits, k, kw.get("filter")), dtype=torch.uint8, device=dev)
+        outs = []
+        for rep in range(4):
+            if rep == 3:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                tq.profile_events(e0, e1)
+            try:
+                outs.append(tq.search(Qd, Rd, cd, bits, pd, sd, k, workspace=ws, stream=side, **kw))
+            finally:
+                tq.profile_events(None, None)
+            tq.search_check(ws, stream=side)
+        side.synchronize()
+        for i, s_ in outs:
+            assert torch.equal(i, want_i) and torch.equal(s_, want_s)
+    finally:
+        tq.set_search_path("auto")
+        if filtered:
+            kw["filter"].close()
+    ref = O.search(c["Q"][:nq], c["R"], c32, bits, packed, scale, k, d, *(
+        (tid, off, allow) if filtered else ()))
+    allowed = O.allowed_mask(tid, off, allow, nq, n) if filtered else np.ones((nq, n), bool)
+    check_topk(want_i.cpu().numpy(), want_s.cpu().numpy(), ref.ids, ref.scores64, allowed, k, TOL_LUT)
