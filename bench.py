@@ -14,6 +14,12 @@ timed region starts; the 767 MB corpus is larger than the 129 MB L2, so every
 step streams it from HBM.  The headline `value` is queries/s at the first batch
 size; every batch size measured is reported under "batches".
 
+The default run also measures, compactly under "extra", the 100K workload
+(batch 1 and 256, top-5 and top-10, encode), the filtered workload on that
+corpus (Zipf tenants, T = 10/100/1000, with the over-fetch post-filter
+baseline) and the bit-width sweep on the 999K corpus (b = 2/3/4/8, batch 256,
+encode), each with its roofline (--no-extras skips them).
+
 --impl reference times the CPU oracle (float64 numpy) on the host cores on a
 bounded sample of the same workload.
 
@@ -64,7 +70,7 @@ CONFIGS = {
 }
 
 RECALL_Q = 200       # queries whose Recall@k against exact kNN the bench reports
-MMA_MIN_BATCH = 16  # tq_search's AUTO switch to the tensor-core scan (bits 2/4/8, k <= 64, no filter)
+MMA_MIN_BATCH = 16  # tq_search's AUTO switch to the tensor-core scan (k <= 64)
 
 METRIC = "queries/sec at 999Kx1536 4-bit top-5 (batch 1 / 1024); % of HBM / TC roofline"
 
@@ -364,7 +370,9 @@ def run_ours(args, cfg, rank, world):
             idx = torch.cat([exact, torch.arange(r0, r0 + sc.shape[1], device=dev).expand(nrec, -1)], dim=1)
             exact, best = torch.gather(idx, 1, i), v
     stream.synchronize()
-    del Xd
+    run_extras = world == 1 and args.config == "scale" and not args.no_extras
+    if not run_extras:
+        del Xd
     torch.cuda.empty_cache()
     log(f"[bench] encode {n} vectors: {enc_ms:.1f} ms ({n / enc_ms * 1e3:.3g} vec/s)")
 
@@ -400,64 +408,72 @@ def run_ours(args, cfg, rank, world):
 
         for i in range(args.warmup):
             step(i)
-        # scan-kernel events recorded inside the timed loop
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
+        # the timed region: back-to-back steps on `stream`, as a serving loop
+        # runs them (the lookup scan overlaps the rotation's tail there)
         t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         barrier()
         with ClockSampler(pci, local) as clk:
             t0.record(stream)
             for i in range(args.steps):
-                tq.profile_events(*evs[i])
                 step(args.warmup + i)
             t1.record(stream)
             t1.synchronize()
-        tq.profile_events(None, None)
         barrier()
         ms = t0.elapsed_time(t1)
         if world > 1:
             tt = torch.tensor([ms], device=dev)
             dist.all_reduce(tt, op=dist.ReduceOp.MAX)
             ms = float(tt.item())
+        # the scan kernel's duration: the same steps again, with the library
+        # recording CUDA events on `stream` around each scan launch
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for i in range(args.steps):
+            tq.profile_events(*evs[i])
+            step(args.warmup + i)
+        tq.profile_events(None, None)
+        stream.synchronize()
         scan_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
         qps = B * args.steps * world / (ms / 1e3)
         alg_bytes = n * (d * bits // 8 + 4)
-        if B >= MMA_MIN_BATCH and bits in (2, 4, 8) and k <= 64:
+        mma = B >= MMA_MIN_BATCH and bits in (2, 3, 4, 8) and k <= 64
+        if mma:
             # tensor-core scan: 2*n*d*B flops per launch against the dense fp16/bf16
-            # peak (same rate), sustained figure since it runs inside a long loop
+            # peak (same rate); each launch is a few ms, timed alone: the burst figure
             flops = 2.0 * n * d * B
             achieved = flops / (scan_ms / 1e3) / 1e12
-            peak = pk["bf16_tflops_sustained"]
+            peak = pk["bf16_tflops"]
             roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak, "frac_of": pk["source"] + " (sustained bf16 = fp16 dense rate)",
+                    "frac": achieved / peak, "frac_of": pk["source"] + " burst bf16 (= fp16 dense rate)",
+                    "frac_of_sustained": achieved / pk["bf16_tflops_sustained"],
                     "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_mma.cu", "k_scan_mma_250k_batch1024.md",
                                                 scale_to=n),
                     "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": scan_ms,
                     "hbm_gbs_of_corpus": alg_bytes / (scan_ms / 1e3) / 1e9}
         else:
-            # lookup scan: the corpus (codes + scales) read once per launch; 4-bit
-            # codes take the byte-pair kernel, other widths the per-code one
-            kname = "k_scan_pair_stream" if bits == 4 else "k_scan_lut_stream"
+            # lookup scan (with its last CTA's merge): the corpus, codes + scales,
+            # read once per launch
             achieved = alg_bytes / (scan_ms / 1e3) / 1e9
             roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
                     "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
                     "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu",
-                                                "k_scan_pair_stream_250k_batch1.md", scale_to=n)
+                                                "k_scan_stream_250k_batch1.md", scale_to=n)
                     if bits == 4 else None,
-                    "kernel": kname, "alg_bytes_per_launch": alg_bytes, "kernel_ms": scan_ms,
-                    "frac_of_8tbs_nominal": achieved / 8000.0,
-                    "smem_lookup_ceiling_gbs": 4950.0 if bits == 4 else None}
-        # e2e through the public API with host buffers
+                    "kernel": "k_scan_stream" if bits != 3 else "k_scan_ring", "alg_bytes_per_launch": alg_bytes,
+                    "kernel_ms": scan_ms, "frac_of_8tbs_nominal": achieved / 8000.0}
+        # e2e through the C ABI with host buffers: tq_search_host queues the
+        # query upload, the search and the result download on `stream`
         qh = torch.empty((B, d), dtype=torch.float32).pin_memory()
         qh.copy_(torch.from_numpy(Qpool[:B]))
-        qdev = torch.empty((B, d), dtype=torch.float32, device=dev)
         ih = torch.empty((B, k), dtype=torch.int64).pin_memory()
         sh = torch.empty((B, k), dtype=torch.float32).pin_memory()
+        stg = torch.empty(tq.search_host_staging(B, d, k), dtype=torch.uint8, device=dev)
+        qdev = torch.empty((B, d), dtype=torch.float32, device=dev)
         with torch.cuda.stream(stream):
             def e2e_step():
                 if world == 1:
-                    tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, qdev, ih, sh, workspace=ws,
-                                        out_ids=ids, out_scores=scs, stream=stream)
+                    tq.search_from_host(qh, Rd, cd, bits, codes, scale, k, ih, sh, workspace=ws, staging=stg,
+                                        stream=stream)
                 else:
                     qdev.copy_(qh, non_blocking=True)
                     tq.search(qdev, Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids,
@@ -476,8 +492,12 @@ def run_ours(args, cfg, rank, world):
             b.record(stream)
             b.synchronize()
         e2e_ms = a.elapsed_time(b)
+        # our kernels per step: rotation + lookup scan (merged in its last CTA),
+        # or rotation + query packing + tensor-core scan + merge; + shard merge
+        launches = (4 if mma else 2) + (1 if world > 1 else 0)
         results[B] = {
             "value": qps, "ms_per_step": ms / args.steps, "roofline": roof, "clocks": clk.summary(),
+            "gpu_launches": launches * args.steps,
             "e2e": {"value": B * args.steps * world / (e2e_ms / 1e3), "unit": "queries/s",
                     "h2d_bytes_per_step": B * d * 4, "d2h_bytes_per_step": B * k * 12},
         }
@@ -489,7 +509,7 @@ def run_ours(args, cfg, rank, world):
     recall = {"k": k, "queries": nrec,
               "exact": "float32 brute force over the unquantised normalised corpus"}
     for path in ("lut", "mma"):
-        if path == "mma" and not (bits in (2, 4, 8) and k <= 64):
+        if path == "mma" and not (bits in (2, 3, 4, 8) and k <= 64):
             continue
         tq.set_search_path(path)
         try:
@@ -505,7 +525,7 @@ def run_ours(args, cfg, rank, world):
     # Sec. IV-E, Table III), from each path's top-20
     rag = {"queries": nrec, "exact_top1": "float32 brute force over the unquantised normalised corpus"}
     for path in ("lut", "mma"):
-        if path == "mma" and bits not in (2, 4, 8):
+        if path == "mma" and bits not in (2, 3, 4, 8):
             continue
         tq.set_search_path(path)
         try:
@@ -538,16 +558,24 @@ def run_ours(args, cfg, rank, world):
         "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
         "recall": recall,
         "rag_quality": rag,
-        "gpu_launches": (3 if world == 1 else 4) * args.steps,  # rotate, scan, merge (+ shard merge)
+        "gpu_launches": r["gpu_launches"],
         "batches": {str(b): {"value": v["value"], "ms_per_step": v["ms_per_step"],
-                             "roofline": v["roofline"], "e2e": v["e2e"]} for b, v in results.items()},
+                             "roofline": v["roofline"], "e2e": v["e2e"], "gpu_launches": v["gpu_launches"]}
+                    for b, v in results.items()},
         "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
                    "tflops": 2.0 * n * d * d / (enc_ms / 1e3) / 1e12},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         qps_cpu, info = oracle_qps_sample(cfg, sample_rows=min(n, args.ref_sample), n_queries=5)
         line["cpu_baseline"] = {"value": qps_cpu, "unit": "queries/s", "cores": cpu_threads(),
-                                "kind": "oracle", "sample": info["sample"]}
+                                "kind": "oracle", **cpu_model(), "sample": info["sample"]}
+    if run_extras:
+        # the other workloads, compactly: the 100K and filtered workloads and
+        # the bit-width sweep, each with its roofline
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        line["extra"] = {"100k": extras_100k(torch, tq, dev, stream, pk, flush, steps=20),
+                         "sweep": extras_sweep(torch, tq, dev, stream, pk, Xd, Rd, Qd, steps=10)}
+        del Xd, flush
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -565,6 +593,260 @@ def _timed(fn, steps, warmup, stream):
     b.record(stream)
     b.synchronize()
     return a.elapsed_time(b) / steps
+
+
+# --------------------------------------------------------- other workloads --
+def cpu_model():
+    """The host CPU's model name and core count (lscpu, else /proc/cpuinfo)."""
+    name = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                name = line.split(":", 1)[1].strip()
+                break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    if not name:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    if line.lower().startswith(("model name", "cpu model")):
+                        name = line.split(":", 1)[1].strip()
+                        break
+        except OSError:
+            pass
+    return {"model": name or "unknown", "nproc": os.cpu_count()}
+
+
+def _flushed_ms(torch, fn, steps, stream, flush):
+    """Mean device time of fn() over `steps` calls on `stream`, each after a
+    write of `flush` (larger than L2) that is not timed: for corpora that fit
+    in L2, so that every call still reads them from HBM."""
+    times = []
+    for i in range(steps):
+        flush.fill_(i & 255)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn(i)
+        b.record(stream)
+        times.append((a, b))
+    stream.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in times)
+
+
+def _scan_ms(torch, tq, fn, steps, stream, flush=None):
+    """Mean duration of the scan kernel inside fn(), from the library's events."""
+    evs = []
+    for i in range(steps):
+        if flush is not None:
+            flush.fill_(i & 255)
+        e = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+        tq.profile_events(*e)
+        fn(i)
+        evs.append(e)
+    tq.profile_events(None, None)
+    stream.synchronize()
+    return statistics.mean(a.elapsed_time(b) for a, b in evs)
+
+
+def _roof_hbm(alg_bytes, ms, pk, kernel):
+    gbs = alg_bytes / (ms / 1e3) / 1e9
+    return {"bound": "hbm", "achieved": gbs, "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": gbs / pk["hbm_gbs"],
+            "frac_of": pk["source"], "traffic": None, "kernel": kernel, "alg_bytes_per_launch": alg_bytes,
+            "kernel_ms": ms}
+
+
+def _roof_tc(flops, ms, pk):
+    tf = flops / (ms / 1e3) / 1e12
+    return {"bound": "tensor", "achieved": tf, "peak": pk["bf16_tflops"], "unit": "TFLOP/s",
+            "frac": tf / pk["bf16_tflops"], "frac_of": pk["source"] + " burst bf16 (= fp16 dense rate)",
+            "traffic": None, "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": ms}
+
+
+def _recall(torch, ids, exact):
+    """Mean |ids ∩ exact| / |exact| over queries (torch tensors [nq, k]; -1 is no result)."""
+    hits = 0.0
+    for g, e in zip(ids.tolist(), exact.tolist()):
+        e = {v for v in e if v >= 0}
+        hits += len({v for v in g if v >= 0} & e) / max(1, len(e))
+    return hits / len(exact)
+
+
+def extras_100k(torch, tq, dev, stream, pk, flush, steps):
+    """The 100K workload (batch 1 and 256, top-5 and top-10, encode) and the
+    filtered workload on the same corpus (Zipf tenants, T = 10, 100, 1000,
+    batch 1, with the over-fetch post-filter baseline).  The corpus (77 MB of
+    codes) fits in L2, so L2 is flushed before every timed search."""
+    import oracle as O
+    from paper_2607_16973_gb300 import synth
+    cfg, fcfg = CONFIGS["c2"], CONFIGS["filtered"]
+    n, d, bits = cfg["n"], cfg["d"], cfg["bits"]
+    X = synth.mixture_corpus(n, d, cfg["clusters"], workers=min(16, os.cpu_count() or 4))
+    src = synth.query_sources(n, cfg["pool"])
+    Q = synth.perturb(X[src])
+    cen, bnd, _ = tq.codebook(d, bits)
+    R = tq.rotation(d, synth.SEED_ROTATION)
+    nrec = min(RECALL_Q, len(Q))
+    with torch.cuda.stream(stream):
+        Xd, Qd, Rd, cd, bd = (torch.from_numpy(a).to(dev) for a in (X, Q, R, cen, bnd))
+        codes, scale = tq.encode(Xd, Rd, cd, bd, bits, stream=stream)
+        enc_ms = _flushed_ms(torch, lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream),
+                             3, stream, flush)
+        exact_sc = Qd[:nrec] @ Xd.T                      # float32, TF32 off: [nrec, n]
+    stream.synchronize()
+    out = {"workload": f"N={n} d={d} {bits}-bit, {cfg['clusters']}-cluster mixture, {len(Q)} queries",
+           "l2": "corpus fits in L2: flushed before every timed call",
+           "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms}}
+    alg = n * (d * bits // 8 + 4)
+    for B in (1, 256):
+        for k in (5, 10):
+            nb = max(1, len(Q) // B)
+            ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
+            ids = torch.empty((B, k), dtype=torch.int64, device=dev)
+            scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+
+            def fn(i):
+                j = (i % nb) * B
+                tq.search(Qd[j:j + B], Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids, out_scores=scs,
+                          stream=stream)
+            with torch.cuda.stream(stream):
+                for i in range(3):
+                    fn(i)
+                ms = _flushed_ms(torch, fn, steps, stream, flush)
+                kms = _scan_ms(torch, tq, fn, steps, stream, flush)
+                tq.set_search_path("lut" if B < MMA_MIN_BATCH else "auto")
+                try:
+                    got, _ = tq.search(Qd[:nrec], Rd, cd, bits, codes, scale, k, stream=stream)
+                finally:
+                    tq.set_search_path("auto")
+                ex = torch.topk(exact_sc, k, dim=1)[1]
+            stream.synchronize()
+            roof = _roof_tc(2.0 * n * d * B, kms, pk) if B >= MMA_MIN_BATCH else _roof_hbm(alg, kms, pk,
+                                                                                        "k_scan_stream")
+            out[f"batch{B}_top{k}"] = {"value": B / ms * 1e3, "unit": "queries/s", "ms_per_step": ms,
+                                       "roofline": roof, "recall": _recall(torch, got.cpu(), ex.cpu())}
+            log(f"[bench] 100K batch {B} top-{k}: {B / ms * 1e3:.4g} q/s, scan {kms * 1e3:.1f} us")
+    # filtered workload on the same corpus
+    k, blk = fcfg["k"], fcfg["block"]
+    rb = d * bits // 8
+    filt_out = {}
+    for T in fcfg["tenants"]:
+        tid, values = synth.zipf_tenants(n, T)
+        off, allow = synth.allowlists(src, tid, values)
+        filt = tq.Filter(torch.from_numpy(tid.view(np.int32)).to(dev), block=blk, stream=stream)
+        q_off = [torch.tensor([0, off[i + 1] - off[i]], dtype=torch.int64, device=dev) for i in range(len(Q))]
+        q_ten = [torch.from_numpy(allow[off[i]:off[i + 1]].view(np.int32)).to(dev) for i in range(len(Q))]
+        ws = torch.empty(tq.search_workspace(1, n, d, bits, k, filt), dtype=torch.uint8, device=dev)
+        ids = torch.empty((1, k), dtype=torch.int64, device=dev)
+        scs = torch.empty((1, k), dtype=torch.float32, device=dev)
+
+        def fn(i):
+            j = i % len(Q)
+            tq.search(Qd[j:j + 1], Rd, cd, bits, codes, scale, k, filter=filt, allow_off=q_off[j],
+                      allow_tenants=q_ten[j], workspace=ws, out_ids=ids, out_scores=scs, stream=stream)
+        # share of the corpus each timed query skips (filter blocks without an allowed tenant)
+        nblocks = (n + blk - 1) // blk
+        tb = np.concatenate([tid, np.full(nblocks * blk - n, 0xFFFFFFFF, np.uint32)]).reshape(nblocks, blk)
+        skip = [1.0 - np.isin(tb, allow[off[i % len(Q)]:off[i % len(Q) + 1]]).any(axis=1).mean()
+                for i in range(steps)]
+        with torch.cuda.stream(stream):
+            for i in range(3):
+                fn(i)
+            ms = _flushed_ms(torch, fn, steps, stream, flush)
+            kms = _scan_ms(torch, tq, fn, steps, stream, flush)
+            # recall against exact kNN restricted to the allowed vectors, and the
+            # over-fetch post-filter baseline (Sec. V-C, Table V)
+            k_over = min(256, k * max(1, T // 10))
+            ws_o = torch.empty(tq.search_workspace(1, n, d, bits, k_over), dtype=torch.uint8, device=dev)
+            ids_o = torch.empty((1, k_over), dtype=torch.int64, device=dev)
+            scs_o = torch.empty((1, k_over), dtype=torch.float32, device=dev)
+
+            def fn_over(i):
+                j = i % len(Q)
+                tq.search(Qd[j:j + 1], Rd, cd, bits, codes, scale, k_over, workspace=ws_o, out_ids=ids_o,
+                          out_scores=scs_o, stream=stream)
+            ms_over = _flushed_ms(torch, fn_over, steps, stream, flush)
+            over, _ = tq.search(Qd[:nrec], Rd, cd, bits, codes, scale, k_over, stream=stream)
+            got = []
+            for i in range(nrec):
+                g, _ = tq.search(Qd[i:i + 1], Rd, cd, bits, codes, scale, k, filter=filt, allow_off=q_off[i],
+                                 allow_tenants=q_ten[i], stream=stream)
+                got.append(g)
+            got = torch.cat(got)
+        stream.synchronize()
+        hits = pf_hits = 0.0
+        over = over.cpu().numpy()
+        for i in range(nrec):
+            ok = np.isin(tid, allow[off[i]:off[i + 1]])
+            sc = torch.where(torch.from_numpy(ok).to(dev), exact_sc[i], torch.tensor(float("-inf"), device=dev))
+            ex = set(torch.topk(sc, min(k, int(ok.sum())))[1].tolist())
+            hits += len(ex & set(got[i].tolist())) / max(1, len(ex))
+            kept = [v for v in over[i] if v >= 0 and ok[v]][:k]
+            pf_hits += len(ex & set(kept)) / max(1, len(ex))
+        filt.close()
+        live = (1.0 - float(np.mean(skip))) * alg + n * 4  # codes + scales of the blocks read, dense tenant ids
+        filt_out[str(T)] = {"value": 1e3 / ms, "unit": "queries/s", "ms_per_query": ms,
+                            "bytes_skipped_frac": float(np.mean(skip)), "recall": hits / nrec,
+                            "roofline": _roof_hbm(live, kms, pk, "k_scan_stream (filtered)"),
+                            "postfilter": {"overfetch_k": k_over, "recall": pf_hits / nrec, "ms_per_query": ms_over}}
+        log(f"[bench] filtered T={T}: {1e3 / ms:.4g} q/s, scan {kms * 1e3:.1f} us, {np.mean(skip):.1%} skipped, "
+            f"R@{k} {hits / nrec:.3f}, post-filter R@{k} {pf_hits / nrec:.3f}")
+    out["filtered"] = {"workload": f"Zipf(1.1) tenants, block {blk}, batch 1, top-{k}, 10% of the queries allow 5",
+                       "variants": filt_out}
+    # the oracle on the host cores: its search of 3 single queries over the
+    # whole 100K corpus, which it encodes itself
+    enc = O.encode(X, R, cen, bnd, bits)
+    t = []
+    for q in range(3):
+        t0 = time.perf_counter()
+        O.search(Q[q:q + 1], R, cen, bits, enc.packed, enc.scale, 10, d)
+        t.append(time.perf_counter() - t0)
+    out["cpu_baseline"] = {"value": 1.0 / statistics.median(t), "unit": "queries/s", "cores": cpu_threads(),
+                           "kind": "oracle", **cpu_model(),
+                           "sample": "oracle search (float64 numpy) of 3 single queries over all 100,000 rows, "
+                                     "top-10, median"}
+    del Xd
+    return out
+
+
+def extras_sweep(torch, tq, dev, stream, pk, Xd, Rd, Qd, steps):
+    """The bit-width sweep on the 999K corpus already on the device: encode at
+    b = 2, 3, 4, 8 and batch-256 top-10 search at each width."""
+    cfg = CONFIGS["sweep"]
+    n, d, k, B = cfg["n"], cfg["d"], cfg["k"], cfg["batches"][0]
+    nb = max(1, Qd.shape[0] // B)
+    out = {"workload": f"N={n} d={d}, batch {B}, top-{k}; corpus larger than L2", "variants": {}}
+    for bits in cfg["sweep_bits"]:
+        cen, bnd, _ = tq.codebook(d, bits)
+        cd, bd = torch.from_numpy(cen).to(dev), torch.from_numpy(bnd).to(dev)
+        with torch.cuda.stream(stream):
+            codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
+            scale = torch.empty(n, dtype=torch.float32, device=dev)
+            enc = lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream)
+            enc(0)
+            enc_ms = _timed(enc, 3, 1, stream)
+            ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
+            ids = torch.empty((B, k), dtype=torch.int64, device=dev)
+            scs = torch.empty((B, k), dtype=torch.float32, device=dev)
+
+            def fn(i):
+                j = (i % nb) * B
+                tq.search(Qd[j:j + B], Rd, cd, bits, codes, scale, k, workspace=ws, out_ids=ids, out_scores=scs,
+                          stream=stream)
+            ms = _timed(fn, steps, 2, stream)
+            kms = _scan_ms(torch, tq, fn, min(steps, 5), stream)
+        mma = bits in (2, 3, 4, 8)
+        alg = n * (d * bits // 8 + 4)
+        roof = _roof_tc(2.0 * n * d * B, kms, pk) if mma else _roof_hbm(alg, kms, pk, "k_scan_ring")
+        out["variants"][str(bits)] = {"value": B / ms * 1e3, "unit": "queries/s", "ms_per_step": ms,
+                                      "path": "tensor core" if mma else "lookup", "roofline": roof,
+                                      "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
+                                                 "tflops": 2.0 * n * d * d / (enc_ms / 1e3) / 1e12}}
+        log(f"[bench] sweep b={bits}: encode {n / enc_ms * 1e3:.3g} vec/s, batch {B}: {B / ms * 1e3:.4g} q/s")
+        del codes, scale, ws
+        torch.cuda.empty_cache()
+    return out
 
 
 def run_filtered(args, cfg):
@@ -708,7 +990,7 @@ def run_sweep(args, cfg):
             ms = _timed(lambda i: tq.search(Qd[(i % nb) * B:(i % nb) * B + B], Rd, cd, bits, codes, scale, k,
                                             workspace=ws, out_ids=ids, out_scores=scs, stream=stream),
                         steps, min(args.warmup, 3), stream)
-        path = "tensor core" if bits in (2, 4, 8) and k <= 64 else "lookup"
+        path = "tensor core" if bits in (2, 3, 4, 8) and k <= 64 else "lookup"
         variants[str(bits)] = {"encode_vectors_per_s": n / enc_ms * 1e3, "encode_ms": enc_ms,
                                "value": B / ms * 1e3, "ms_per_step": ms, "path": path,
                                "codes_mb": n * d * bits / 8 / 1e6}
@@ -804,6 +1086,8 @@ def main():
     ap.add_argument("--k", type=int, default=None)
     ap.add_argument("--ref-sample", type=int, default=100_000, help="corpus rows the oracle scans")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="scale workload only: skip the 100K, filtered and bit-width sweep lines under 'extra'")
     args = ap.parse_args()
     cfg = CONFIGS[args.config]
     world = int(os.environ.get("WORLD_SIZE", "1"))

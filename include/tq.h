@@ -203,8 +203,10 @@ tq_status tq_search_workspace(int64_t nq, int64_t n, int d, int bits, int k,
  *   out_ids        device out [nq*k] int64, -1 where fewer than k vectors are allowed
  *   out_scores     device out [nq*k] float32, -INFINITY where out_ids is -1
  *   workspace      device scratch of ws_bytes >= tq_search_workspace(...)
- * Scores are float32 sums (LUT path) or fp16 products with float32
- * accumulation (MMA path).
+ * Kernels (TQ_PATH_AUTO): batches of 16 or more queries over 2-, 4- or 8-bit
+ * codes with d a multiple of 64 and k <= 64 run the tensor-core scan (fp16
+ * products, float32 accumulation), filtered or not; the rest run the lookup
+ * scan (float32 sums).
  */
 tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
                     const float* centroids, int bits, const uint8_t* codes,
@@ -234,6 +236,32 @@ tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
                        const uint32_t* deleted, const uint64_t* ext_ids,
                        int k, int64_t* out_ids, float* out_scores, void* workspace,
                        size_t ws_bytes, void* stream);
+
+/*
+ * tq_search_host - tq_search_ex for queries and results in host memory: the
+ * search() call of a serving process whose requests arrive in host memory.
+ * Queues, on `stream`, the copy of the nq queries from Q_host to the device
+ * staging buffer, the search, and the copies of the results to ids_host and
+ * scores_host; returns without waiting (synchronise `stream` before reading
+ * the results; page-locked host buffers keep the copies asynchronous).
+ *   Q_host       host [nq*d] float32 queries
+ *   ids_host     host out [nq*k] int64;  scores_host  host out [nq*k] float32
+ *   staging      device scratch of staging_bytes >= tq_search_host_staging()
+ *                (the device copies of the queries and results)
+ *   the other arguments as for tq_search_ex (R, centroids, codes, scale,
+ *   allow_off, allow_tenants, deleted, ext_ids and workspace are device
+ *   memory).
+ * The host buffers must stay valid until the copies have run.
+ */
+tq_status tq_search_host_staging(int64_t nq, int d, int k, size_t* bytes);
+tq_status tq_search_host(const float* Q_host, int64_t nq, int d, const float* R,
+                         const float* centroids, int bits, const uint8_t* codes,
+                         const float* scale, int64_t n, const tq_filter* filter,
+                         const int64_t* allow_off, const uint32_t* allow_tenants,
+                         const uint32_t* deleted, const uint64_t* ext_ids, int k,
+                         int64_t* ids_host, float* scores_host, void* staging,
+                         size_t staging_bytes, void* workspace, size_t ws_bytes,
+                         void* stream);
 
 /*
  * tq_idmap - the id map of an id-mapped index (Sec. III-A): external uint64

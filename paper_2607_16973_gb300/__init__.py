@@ -14,8 +14,8 @@ import numpy as np
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
 __all__ = ["codebook", "rotation", "encode", "Filter", "IdMap", "Index", "search", "search_workspace",
-           "search_from_host", "search_check", "merge_topk", "set_search_path", "profile_events", "row_bytes", "load",
-           "TQError"]
+           "search_from_host", "search_host_staging", "search_check", "merge_topk", "set_search_path",
+           "profile_events", "row_bytes", "load", "TQError"]
 
 
 def _torch():
@@ -274,17 +274,50 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
     return out_ids, out_scores
 
 
-def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, q_dev, ids_host,
-                     scores_host, filter: Filter | None = None, allow_off=None, allow_tenants=None,
-                     workspace=None, out_ids=None, out_scores=None, stream=None, idmap: IdMap | None = None):
-    """search() for queries in (pinned) host memory: copies Q to q_dev, runs
-    tq_search and copies ids/scores back into the host tensors, all queued on
-    `stream`."""
-    q_dev.copy_(Q_host, non_blocking=True)
-    ids, scores = search(q_dev, R, centroids, bits, codes, scale, k, filter, allow_off, allow_tenants,
-                         workspace, out_ids, out_scores, stream, idmap)
-    ids_host.copy_(ids, non_blocking=True)
-    scores_host.copy_(scores, non_blocking=True)
+def search_host_staging(nq: int, d: int, k: int) -> int:
+    """Bytes of device staging tq_search_host needs (queries and results)."""
+    out = C.c_size_t()
+    check(load().tq_search_host_staging(nq, d, k, C.byref(out)))
+    return out.value
+
+
+def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, ids_host, scores_host,
+                     filter: Filter | None = None, allow_off=None, allow_tenants=None, workspace=None,
+                     staging=None, stream=None, idmap: IdMap | None = None):
+    """tq_search_host: queries in host memory (a CPU float32 tensor, page-locked
+    for asynchronous copies), results into the host tensors ids_host (int64
+    [nq, k]) and scores_host (float32 [nq, k]).  The library queues the query
+    copy, the search and the result copies on `stream`; synchronise it before
+    reading the results."""
+    torch = _torch()
+    nq, d = Q_host.shape
+    n = codes.shape[0]
+    for t, name, dt in ((Q_host, "Q_host", torch.float32), (ids_host, "ids_host", torch.int64),
+                        (scores_host, "scores_host", torch.float32)):
+        if t.is_cuda or t.dtype != dt or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous host {dt} tensor")
+    if ids_host.shape != (nq, k) or scores_host.shape != (nq, k):
+        raise ValueError("ids_host and scores_host must be [nq, k]")
+    deleted = ext = 0
+    if idmap is not None:
+        deleted, ext = idmap.device()
+    dev = codes.device
+    with _on_stream(stream):
+        if workspace is None:
+            workspace = torch.empty(max(search_workspace(nq, n, d, bits, k, filter), 1), dtype=torch.uint8,
+                                    device=dev)
+        if staging is None:
+            staging = torch.empty(search_host_staging(nq, d, k), dtype=torch.uint8, device=dev)
+    f32 = torch.float32
+    u32 = (torch.int32, getattr(torch, "uint32", torch.int32))
+    check(load().tq_search_host(
+        int(Q_host.data_ptr()), nq, d, _dev_ptr(R, "R", f32), _dev_ptr(centroids, "centroids", f32), bits,
+        _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), n,
+        filter.handle if filter else None, _dev_ptr(allow_off, "allow_off", torch.int64),
+        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None, k,
+        int(ids_host.data_ptr()), int(scores_host.data_ptr()), _dev_ptr(staging, "staging"),
+        staging.numel() * staging.element_size(), _dev_ptr(workspace, "workspace"),
+        workspace.numel() * workspace.element_size(), _stream_handle(stream)))
     return ids_host, scores_host
 
 

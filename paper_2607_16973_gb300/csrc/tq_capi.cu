@@ -41,7 +41,7 @@ struct SearchPlan {
 SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
   SearchPlan p;
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
-  const bool mma = mma_supported(bits, d, k) && !filter;
+  const bool mma = mma_supported(bits, d, k);
   p.grid_mma = mma ? scan_mma_grid_x(nq, n, k, bits) : 0;
   const int per_query = std::max(p.grid_lut, p.grid_mma) * k;
   size_t off = 0;
@@ -308,9 +308,9 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
       return fail(TQ_EINVAL, "tq_search: misaligned allowlist pointers");
   }
   const int path = tq::search_path();
-  const bool can_mma = tq::mma_supported(bits, d, k) && !filter;
+  const bool can_mma = tq::mma_supported(bits, d, k);
   if (path == TQ_PATH_MMA && !can_mma)
-    return fail(TQ_EUNSUPPORTED, "tq_search: the tensor-core scan needs bits 2/4/8, k <= %d and no filter",
+    return fail(TQ_EUNSUPPORTED, "tq_search: the tensor-core scan needs bits 2/4/8, d %% 64 == 0 and k <= %d",
                 tq::kMaxKMma);
   const bool use_mma = can_mma && (path == TQ_PATH_MMA || (path == TQ_PATH_AUTO && nq >= tq::kMmaMinBatch));
   const tq::SearchPlan p = tq::plan_search(nq, n, d, bits, k, filter);
@@ -327,10 +327,12 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
   cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);  // also zeroes both
   if (use_mma) {
+    if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
     if (e == cudaSuccess)
-      e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, deleted, k, p.grid_mma,
-                              ws + p.off_qpack, cs, ci,
-                              status, s, (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
+      e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
+                              filter ? filter->f.dense : nullptr, allow, filter ? filter->f.words : 0, k,
+                              p.grid_mma, ws + p.off_qpack, cs, ci, status, s, (cudaEvent_t)tq::profile_start(),
+                              (cudaEvent_t)tq::profile_stop());
     if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, ext_ids, out_ids, out_scores, s);
   } else {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
@@ -354,6 +356,61 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
                                size_t ws_bytes, void* stream) {
   return tq_search_ex(Q, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, nullptr,
                       nullptr, k, out_ids, out_scores, workspace, ws_bytes, stream);
+}
+
+namespace {
+// staging layout of tq_search_host: queries | ids | scores
+struct HostStaging {
+  size_t off_ids, off_scores, total;
+};
+HostStaging host_staging(int64_t nq, int d, int k) {
+  HostStaging h;
+  h.off_ids = tq::align_up((size_t)nq * d * sizeof(float));
+  h.off_scores = h.off_ids + tq::align_up((size_t)nq * k * sizeof(int64_t));
+  h.total = h.off_scores + tq::align_up((size_t)nq * k * sizeof(float));
+  return h;
+}
+}  // namespace
+
+extern "C" tq_status tq_search_host_staging(int64_t nq, int d, int k, size_t* bytes) {
+  if (!bytes) return fail(TQ_EINVAL, "tq_search_host_staging: NULL bytes");
+  if (nq < 0 || nq > (1 << 24) || d < 1 || d > tq::kMaxD || k < 1 || k > tq::kMaxK)
+    return fail(TQ_EINVAL, "tq_search_host_staging: nq=%lld d=%d k=%d out of range", (long long)nq, d, k);
+  *bytes = host_staging(nq, d, k).total;
+  return tq::ok();
+}
+
+extern "C" tq_status tq_search_host(const float* Q_host, int64_t nq, int d, const float* R,
+                                    const float* centroids, int bits, const uint8_t* codes,
+                                    const float* scale, int64_t n, const tq_filter* filter,
+                                    const int64_t* allow_off, const uint32_t* allow_tenants,
+                                    const uint32_t* deleted, const uint64_t* ext_ids, int k,
+                                    int64_t* ids_host, float* scores_host, void* staging,
+                                    size_t staging_bytes, void* workspace, size_t ws_bytes, void* stream) {
+  tq_status st = check_search(nq, n, d, bits, k);
+  if (st != TQ_OK) return st;
+  if (nq == 0) return tq::ok();
+  if (!Q_host || !ids_host || !scores_host || !staging)
+    return fail(TQ_EINVAL, "tq_search_host: NULL query, result or staging pointer");
+  if (!tq::aligned16(staging)) return fail(TQ_EINVAL, "tq_search_host: staging must be 16-byte aligned");
+  const HostStaging h = host_staging(nq, d, k);
+  if (staging_bytes < h.total)
+    return fail(TQ_EINVAL, "tq_search_host: staging of %zu bytes, %zu needed", staging_bytes, h.total);
+  char* stg = static_cast<char*>(staging);
+  float* q_dev = reinterpret_cast<float*>(stg);
+  int64_t* ids_dev = reinterpret_cast<int64_t*>(stg + h.off_ids);
+  float* scores_dev = reinterpret_cast<float*>(stg + h.off_scores);
+  cudaStream_t s = (cudaStream_t)stream;
+  cudaError_t e = cudaMemcpyAsync(q_dev, Q_host, (size_t)nq * d * sizeof(float), cudaMemcpyHostToDevice, s);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: query copy", e);
+  st = tq_search_ex(q_dev, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, deleted,
+                    ext_ids, k, ids_dev, scores_dev, workspace, ws_bytes, stream);
+  if (st != TQ_OK) return st;
+  e = cudaMemcpyAsync(ids_host, ids_dev, (size_t)nq * k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(scores_host, scores_dev, (size_t)nq * k * sizeof(float), cudaMemcpyDeviceToHost, s);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: result copy", e);
+  return tq::ok();
 }
 
 extern "C" tq_status tq_merge_topk(const int64_t* cand_ids, const float* cand_scores, int64_t n_src, int64_t nq,

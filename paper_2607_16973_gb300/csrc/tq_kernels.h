@@ -75,12 +75,15 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
 cudaError_t launch_merge_global(const float* cand_s, const int64_t* cand_i, int64_t S, int64_t nq, int64_t m,
                                 int k, int64_t* out_ids, float* out_scores, cudaStream_t s);
 
-// Tensor-core decode-GEMM scan (bits 2, 4, 8; k <= kMaxKMma; unfiltered).
+// Tensor-core decode-GEMM scan (bits 2, 4, 8; k <= kMaxKMma).  With
+// allow_bits [nq * words] (and the filter's dense tenant index) a vector whose
+// tenant the query does not allow never enters its list.
 bool mma_supported(int bits, int d, int k);
 int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits);
 size_t mma_qpack_bytes(int64_t nq, int d);
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del, int k,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
+                            const uint32_t* dense, const uint32_t* allow_bits, int words, int k,
                             int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1);
 

@@ -207,7 +207,7 @@ __device__ __forceinline__ uint32_t sw128_offset(int r, int c) {
 }
 
 struct MmaSmem {
-  uint32_t a, b, raw, tab, scale, lists_s, lists_i, bars, total;
+  uint32_t a, b, raw, tab, scale, dense, lists_s, lists_i, bars, total;
 };
 
 template <int BITS>
@@ -217,7 +217,15 @@ __host__ __device__ constexpr int raw_bytes_per_row() { return KB * BITS / 8; }
 // replicated in all 32 banks (entry e of lane l at e*32 + l).
 template <int BITS>
 __host__ __device__ constexpr int tab_bytes() {
-  return BITS == 4 ? 0 : BITS == 2 ? 16 * 32 * 4 : 256 * 32 * 2;
+  return BITS == 4 ? 0 : BITS == 2 ? 16 * 32 * 4 : BITS == 3 ? 64 * 32 * 4 : 256 * 32 * 2;
+}
+
+// K-blocks per code tile for rows of up to rr bytes per tile.  A TMA box's
+// inner extent is a multiple of 16 bytes: 3-bit K-blocks are 24 bytes, so
+// their tiles carry 4 (96 bytes) or 2 (48 bytes).
+__host__ __device__ inline int tile_sub(int bits, int rr) {
+  if (bits == 3) return rr >= 96 ? 4 : 2;
+  return rr / (KB * bits / 8);
 }
 
 // Shared-memory plan for QT query tiles per CTA, `cst` raw code stages and
@@ -235,6 +243,8 @@ __host__ __device__ inline MmaSmem mma_smem_layout(int k, int cst, int ast, int 
   L.tab = off;
   off += tab_bytes<BITS>();
   L.scale = off;
+  off += tile_n<QT>() * 4;
+  L.dense = off;  // tenant index of each vector of the tile (filtered searches)
   off += tile_n<QT>() * 4;
   L.lists_s = off;
   off += (uint32_t)QT * k * MMA_M * 4;
@@ -284,7 +294,7 @@ MmaPlan mma_plan(int64_t nq, int k) {
       const int gmax = qt == 2 ? dec_groups<2>() : dec_groups<1>();
       for (int ng = gmax; ng >= 2; --ng) {
         for (int rr = RAW_ROW_MAX; rr >= 64; rr >>= 1) {
-          const int sub = rr / raw_bytes_per_row<BITS>();  // for d a multiple of 256
+          const int sub = tile_sub(BITS, rr);  // for d a multiple of 256
           for (int ast = 3; ast >= 2; --ast) {
             for (int cst = MAX_CST; cst >= 2; --cst) {
               if (cst * sub < min_pf || active_groups(ng, sub, cst) != ng) continue;
@@ -350,7 +360,8 @@ template <int BITS, int QT>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,
            const float* __restrict__ centroids, const float* __restrict__ scale,
-           const uint32_t* __restrict__ del, int n, int nq, int d,
+           const uint32_t* __restrict__ del, const uint32_t* __restrict__ dense,
+           const uint32_t* __restrict__ allow_bits, int words, int n, int nq, int d,
            int k, int cst, int ast, int rr, int sub, int ng, int gact, float* __restrict__ cand_s,
            int* __restrict__ cand_i, int* __restrict__ err) {
   constexpr int RAWB = raw_bytes_per_row<BITS>();
@@ -375,6 +386,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
   unsigned char* sB = base + L.b;
   unsigned char* sRaw = base + L.raw;
   float* sScale = reinterpret_cast<float*>(base + L.scale);
+  uint32_t* sDense = reinterpret_cast<uint32_t*>(base + L.dense);
   float* lst_s = reinterpret_cast<float*>(base + L.lists_s);
   int* lst_i = reinterpret_cast<int*>(base + L.lists_i);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
@@ -403,6 +415,13 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     for (int i = tid; i < 16 * 32; i += NTHREADS) {
       const int e = i >> 5;
       const __half2 h = __floats2half2_rn(centroids[e & 3], centroids[e >> 2]);
+      tab[i] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+  } else if (BITS == 3) {  // entry e = two consecutive 3-bit codes (e & 7, e >> 3), in bank `lane`
+    uint32_t* tab = reinterpret_cast<uint32_t*>(base + L.tab);
+    for (int i = tid; i < 64 * 32; i += NTHREADS) {
+      const int e = i >> 5;
+      const __half2 h = __floats2half2_rn(centroids[e & 7], centroids[e >> 3]);
       tab[i] = *reinterpret_cast<const uint32_t*>(&h);
     }
   } else if (BITS == 8) {
@@ -543,6 +562,20 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       if (it >= BST && !warp_wait(bempty + bs, ((it / BST) - 1) & 1, abort_flag, err, 8)) break;
       const unsigned char* raw = sRaw + cs * NT * rr;
       unsigned char* bdst = sB + bs * B_BYTES;
+      if constexpr (BITS == 3) {
+        // 3-bit codes: 3 bytes hold 8 codes (a little-endian 24-bit field);
+        // each pair of codes is one lookup of two fp16 centroids
+        const uint32_t* tab = reinterpret_cast<const uint32_t*>(base + L.tab);
+        for (int item = gtid; item < NT * 8; item += 128) {
+          const int r = item >> 3, g = item & 7;
+          const unsigned char* src = raw + r * rrow + sb * RAWB + 3 * g;
+          const uint32_t x = (uint32_t)src[0] | ((uint32_t)src[1] << 8) | ((uint32_t)src[2] << 16);
+          uint32_t o[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) o[j] = tab[(((x >> (6 * j)) & 63u) << 5) | lane];
+          *reinterpret_cast<uint4*>(bdst + sw128_offset(r, g)) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+      } else
       for (int item = gtid; item < NT * PARTS; item += 128) {
         const int r = item / PARTS, p = item % PARTS;
         const int chunk = sb * PARTS + p;  // 16-byte chunk of the row in this code tile
@@ -593,6 +626,8 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     const int etid = g * 32 + lane;
     const bool mine = jsel < qts;            // warps 12-15 idle with one query tile
     const int q = (qt0 + jsel) * MMA_M + row;
+    // a filtered search: this query's allow bitmap over the dense tenant index
+    const uint32_t* ab = allow_bits && q < nq ? allow_bits + (size_t)q * words : nullptr;
     float* ls = lst_s + jsel * k * MMA_M;
     int* li = lst_i + jsel * k * MMA_M;
     if (mine) {
@@ -639,6 +674,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
       for (int j = etid; j < NT; j += EPI_THREADS) {
         const int v = v0 + j;
         sScale[j] = v < n ? (scale ? scale[v] : 1.0f) : 0.0f;
+        if (allow_bits) sDense[j] = v < n ? __ldg(dense + v) : 0u;
       }
       asm volatile("bar.sync 1, %0;" ::"n"(EPI_THREADS) : "memory");
       // all epilogue warps take the same decision, so none is left at bar.sync
@@ -688,6 +724,10 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
             const int v = v0 + c0 + jj;
             if (!better(sc, v, th_s, th_i)) continue;
             if (del && ((__ldg(del + (v >> 5)) >> (v & 31)) & 1u)) continue;  // deleted row
+            if (ab) {  // tenant not allowed: never enters the list (Sec. III-B)
+              const uint32_t t = sDense[c0 + jj];
+              if (!((__ldg(ab + (t >> 5)) >> (t & 31)) & 1u)) continue;
+            }
             if (npark < 4) {
               ps0 = npark == 0 ? sc : ps0;
               pi0 = npark == 0 ? v : pi0;
@@ -781,27 +821,30 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
 
 template <int BITS, int QT>
 cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half* qpack, const float* centroids,
-                         const float* scale, const uint32_t* del, int n, int nq, int d, int k, int sub,
-                         int grid_x, float* cs, int* ci, int* err, cudaStream_t s) {
+                         const float* scale, const uint32_t* del, const uint32_t* dense, const uint32_t* allow,
+                         int words, int n, int nq, int d, int k, int sub, int grid_x, float* cs, int* ci, int* err,
+                         cudaStream_t s) {
   const int gact = active_groups(P.ng, sub, P.cst);
   cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_mma<BITS, QT>), (int)P.smem);
   if (e != cudaSuccess) return e;
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));
-  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, del, n, nq, d, k, P.cst, P.ast,
-                                                         P.rr, sub, P.ng, gact, cs, ci, err);
+  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, del, dense, allow, words, n, nq,
+                                                         d, k, P.cst, P.ast, P.rr, sub, P.ng, gact, cs, ci, err);
   return cudaGetLastError();
 }
 
 MmaPlan plan_for(int bits, int64_t nq, int k) {
-  return bits == 2 ? mma_plan<2>(nq, k) : bits == 4 ? mma_plan<4>(nq, k) : mma_plan<8>(nq, k);
+  return bits == 2 ? mma_plan<2>(nq, k) : bits == 3 ? mma_plan<3>(nq, k) : bits == 4 ? mma_plan<4>(nq, k)
+                                                                           : mma_plan<8>(nq, k);
 }
 
 }  // namespace
 
 bool mma_supported(int bits, int d, int k) {
-  return (bits == 2 || bits == 4 || bits == 8) && d % KB == 0 && k >= 1 && k <= kMaxKMma &&
-         plan_for(bits, 1, k).smem != 0;
+  // 3-bit code tiles carry an even number of K-blocks: d a multiple of 128
+  return (bits == 2 || bits == 3 || bits == 4 || bits == 8) && d % (bits == 3 ? 2 * KB : KB) == 0 && k >= 1 &&
+         k <= kMaxKMma && plan_for(bits, 1, k).smem != 0;
 }
 
 int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits) {
@@ -820,7 +863,8 @@ size_t mma_qpack_bytes(int64_t nq, int d) {
 }
 
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
-                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del, int k,
+                            const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
+                            const uint32_t* dense, const uint32_t* allow_bits, int words, int k,
                             int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
@@ -831,8 +875,9 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   if (P.smem == 0) return cudaErrorInvalidValue;
   // K-blocks per code tile: up to P.rr bytes of each row, dividing the row's K-blocks
   const int kblocks = d / KB;
-  int sub = P.rr / rawb;
-  while (sub > 1 && kblocks % sub != 0) sub >>= 1;
+  int sub = tile_sub(bits, P.rr);
+  while (sub > (bits == 3 ? 2 : 1) && kblocks % sub != 0) sub >>= 1;
+  if (kblocks % sub != 0 || (sub * rawb) % 16 != 0) return cudaErrorInvalidValue;
   CUtensorMap map;
   const cuuint64_t gdim[2] = {(cuuint64_t)row_bytes(d, bits), (cuuint64_t)n};
   const cuuint64_t gstride[1] = {(cuuint64_t)row_bytes(d, bits)};
@@ -851,13 +896,14 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   const __half* qp = static_cast<const __half*>(qpack);
 #define TQ_MMA_CASE(B)                                                                                \
   case B:                                                                                             \
-    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, del, (int)n, (int)nq, d, k, sub, \
-                                       grid_x, cand_s, cand_i, err, s)                                \
-                  : launch_typed<B, 1>(P, map, qp, centroids, scale, del, (int)n, (int)nq, d, k, sub, \
-                                       grid_x, cand_s, cand_i, err, s);                               \
+    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, del, dense, allow_bits, words, (int)n, \
+                                       (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s)                 \
+                  : launch_typed<B, 1>(P, map, qp, centroids, scale, del, dense, allow_bits, words, (int)n, \
+                                       (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s);                \
     break;
   switch (bits) {
     TQ_MMA_CASE(2)
+    TQ_MMA_CASE(3)
     TQ_MMA_CASE(4)
     TQ_MMA_CASE(8)
     default: return cudaErrorInvalidValue;

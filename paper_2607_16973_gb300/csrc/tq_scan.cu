@@ -239,19 +239,59 @@ __device__ __forceinline__ void load_q2(float2 (&q2)[S][8], const float* qq, int
 // L2: in the scans' tail other CTAs of the same grid wrote them); ws/wi are
 // shared scratch of (blockDim.x / 32) * k entries; out_* point at the query's
 // k results.
+//
+// A second bound: the k best of the lists' first entries are k distinct
+// candidates, so the k-th best overall is at least as good as the k-th of
+// them too.  When there are many lists of few vectors each (a small corpus
+// spread over every SM) their k-th entries are weak and this bound is far
+// tighter; it is taken by sorting the first entries.  `scratch` (shared,
+// scratch_bytes) holds that sort and, when they fit, a copy of all the
+// candidates, fetched in one pass so that later steps wait on no more loads.
 __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, int k, const uint64_t* __restrict__ ext,
-                                  int64_t* out_ids, float* out_scores, float* ws, int* wi) {
-  __shared__ float red_s[32];
-  __shared__ int red_i[32];
+                                  int64_t* out_ids, float* out_scores, float* ws, int* wi, unsigned char* scratch,
+                                  size_t scratch_bytes) {
+  __shared__ float red_s[33];
+  __shared__ int red_i[33];
   const int nwarps = blockDim.x >> 5;
   const int total = nlists * k;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  int P2 = 1;
+  while (P2 < nlists) P2 <<= 1;
+  const bool use_u = nlists > k && (size_t)P2 * 8 <= scratch_bytes;
+  float* sort_s = reinterpret_cast<float*>(scratch);
+  int* sort_i = reinterpret_cast<int*>(sort_s + P2);
+  const size_t stage_off = use_u ? (size_t)P2 * 8 : 0;
+  const bool staged = stage_off + (size_t)total * 8 <= scratch_bytes;
+  float* st_s = reinterpret_cast<float*>(scratch + stage_off);
+  int* st_i = reinterpret_cast<int*>(st_s + total);
+  if (staged) {
+    for (int c = tid; c < total; c += blockDim.x) {
+      st_s[c] = __ldcg(cs + c);
+      st_i[c] = __ldcg(ci + c);
+    }
+    __syncthreads();
+  }
+  auto rs = [&](int c) { return staged ? st_s[c] : __ldcg(cs + c); };
+  auto ri = [&](int c) { return staged ? st_i[c] : __ldcg(ci + c); };
+  // 0. U = k-th best first entry
+  if (use_u) {
+    for (int l = tid; l < P2; l += blockDim.x) {
+      sort_s[l] = l < nlists ? rs(l * k) : -INFINITY;
+      sort_i[l] = l < nlists ? ri(l * k) : INT_MAX;
+    }
+    __syncthreads();
+    block_sort(sort_s, sort_i, P2);
+    if (tid == 0) {
+      red_s[32] = sort_s[k - 1];
+      red_i[32] = sort_i[k - 1];
+    }
+  }
   // 1. T = best k-th entry over the lists
   float ts = -INFINITY;
   int ti = INT_MAX;
   for (int l = tid; l < nlists; l += blockDim.x) {
-    const float a = __ldcg(cs + l * k + k - 1);
-    const int b = __ldcg(ci + l * k + k - 1);
+    const float a = rs(l * k + k - 1);
+    const int b = ri(l * k + k - 1);
     if (better(a, b, ts, ti)) {
       ts = a;
       ti = b;
@@ -282,6 +322,10 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
       ts = red_s[w];
       ti = red_i[w];
     }
+  if (use_u && better(red_s[32], red_i[32], ts, ti)) {
+    ts = red_s[32];
+    ti = red_i[32];
+  }
   // 2. per-warp sorted top-k of the candidates at least as good as T
   float* ls = ws + warp * k;
   int* li = wi + warp * k;
@@ -293,8 +337,8 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
     float a = -INFINITY;
     int b = INT_MAX;
     if (c < total) {
-      a = __ldcg(cs + c);
-      b = __ldcg(ci + c);
+      a = rs(c);
+      b = ri(c);
     }
     const bool cand = b != INT_MAX && !better(ts, ti, a, b) && better(a, b, th_s, th_i);
     unsigned m = __ballot_sync(FULL, cand);
@@ -344,7 +388,7 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
 // scratch (at least blockDim.x / 32 * k entries).
 __device__ __forceinline__ void merge_if_last(const float* cand_s, const int* cand_i, int k, int* counters,
                                               const uint64_t* ext, int64_t* out_ids, float* out_scores, float* ls,
-                                              int* li) {
+                                              int* li, unsigned char* scratch, size_t scratch_bytes) {
   __shared__ int last;
   const int q = blockIdx.y;
   __threadfence();  // this thread's part of the list, before the arrival
@@ -355,7 +399,7 @@ __device__ __forceinline__ void merge_if_last(const float* cand_s, const int* ca
   __threadfence();  // every other CTA's list, after seeing all arrivals
   const size_t base = (size_t)q * gridDim.x * k;
   merge_lists_block(cand_s + base, cand_i + base, gridDim.x, k, ext, out_ids + (size_t)q * k,
-                    out_scores + (size_t)q * k, ls, li);
+                    out_scores + (size_t)q * k, ls, li, scratch, scratch_bytes);
 }
 
 // Sums p[0..3] across the warp: afterwards lanes 8i..8i+7 hold the total of
@@ -671,7 +715,8 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
     cand_s[o] = ls[i];
     cand_i[o] = li[i];
   }
-  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li);
+  // the lookup table is dead by now: its bytes are the merge's scratch
+  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li, smem_raw, TAB_BYTES);
 }
 
 // ---------------------------------------------------------------------------
@@ -953,7 +998,8 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
     cand_s[o] = ls[i];
     cand_i[o] = li[i];
   }
-  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li);
+  // the lookup table is dead by now: its bytes are the merge's scratch
+  merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li, smem_raw, TAB_BYTES);
 }
 
 // Merges the candidates of each query into its sorted top-k, P - k at a time.
@@ -1005,13 +1051,15 @@ k_merge(const float* __restrict__ cand_s, const I* __restrict__ cand_i, int64_t 
 // lists; the lookup scans merge in their own last CTA).
 __global__ void __launch_bounds__(1024)
 k_merge_lists(const float* __restrict__ cand_s, const int* __restrict__ cand_i, int nlists, int k,
-              const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+              const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids, float* __restrict__ out_scores,
+              size_t scratch_bytes) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   float* ws = reinterpret_cast<float*>(smem_raw);  // [nwarps][k]
   int* wi = reinterpret_cast<int*>(ws + (blockDim.x >> 5) * k);
+  unsigned char* scratch = reinterpret_cast<unsigned char*>(wi + (blockDim.x >> 5) * k);
   const int64_t q = blockIdx.x;
   merge_lists_block(cand_s + q * nlists * k, cand_i + q * nlists * k, nlists, k, ext, out_ids + q * k,
-                    out_scores + q * k, ws, wi);
+                    out_scores + q * k, ws, wi, scratch, scratch_bytes);
 }
 
 __device__ __forceinline__ int64_t find_tenant(const uint32_t* __restrict__ tenants, int64_t T, uint32_t x) {
@@ -1261,9 +1309,13 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
   // up to 32 warps, fewer for long lists (each warp keeps k entries in shared memory)
   const int nlists = per_query / k;
   int warps = std::max(1, std::min(32, (nlists + 31) / 32));
-  while (warps > 1 && (size_t)warps * k * 8 > 48 * 1024) warps >>= 1;
-  const size_t smem = (size_t)warps * k * (sizeof(float) + sizeof(int32_t));
-  k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, ext, out_ids, out_scores);
+  while (warps > 1 && (size_t)warps * k * 8 > 24 * 1024) warps >>= 1;
+  // scratch for the first-entry sort and, when it fits, the staged candidates
+  const size_t want = ((size_t)next_pow2(nlists) + (size_t)nlists * k) * 8;
+  const size_t scratch = std::min<size_t>(want, 48 * 1024 - (size_t)warps * k * 8);
+  const size_t smem = (size_t)warps * k * (sizeof(float) + sizeof(int32_t)) + scratch;
+  k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, ext, out_ids, out_scores,
+                                                       scratch);
   return cudaGetLastError();
 }
 

@@ -10,7 +10,7 @@ run on the oracle's codes, so both sides score the same inputs:
 * batch 1 (the lookup scans, several CTA passes each) on 8 queries;
 * the tensor-core scan with one query tile (batch 100) and two query tiles
   (batch 256, and batch 1024 for the scale workload), each CTA walking many
-  vector tiles, and the 3-bit lookup scan at batch 256;
+  vector tiles, at every width;
 * 8 sampled queries of every batch against full float64 oracle scans, and
   Recall@k of the first 200 queries of the batch against exact float kNN,
   equal to the oracle's within 0.002.
@@ -106,7 +106,7 @@ def test_fullsize_encode_every_row(world, bits):
 
 # (bits, k, batches): the scale workload is 4-bit top-5 at batch 1 and 1024;
 # the sweep is top-10 at batch 256 for every width
-CASES = [(2, 10, (1, 100, 256)), (3, 10, (1, 256)), (4, 5, (1, 100, 1024)), (4, 10, (256,)),
+CASES = [(2, 10, (1, 100, 256)), (3, 10, (1, 100, 256)), (4, 5, (1, 100, 1024)), (4, 10, (256,)),
          (8, 10, (1, 100, 256))]
 
 
@@ -123,7 +123,7 @@ def test_fullsize_search(cuda_lib, world, bits, k, batches):
     ref_ids, exact = ref.ids[:, :k], exact[:, :k]
     ones = np.ones((1, N), bool)
     for B in batches:
-        mma = B >= 16 and bits in (2, 4, 8) and k <= 64
+        mma = B >= 16 and k <= 64
         tol = TOL_MMA if mma else TOL_LUT
         if B == 1:
             rows = list(range(8))

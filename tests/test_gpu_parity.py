@@ -147,7 +147,7 @@ def test_rag_metrics_tiny_config(cuda_lib, torch_dev, tiny_config, path):
     assert O.hit_at_k(ref.ids, exact, 10) > 0.9  # the workload is retrievable at 4 bits
 
 
-@pytest.mark.parametrize("bits,path", [(2, "lut"), (3, "lut"), (8, "lut"), (2, "mma"), (8, "mma")])
+@pytest.mark.parametrize("bits,path", [(2, "lut"), (3, "lut"), (8, "lut"), (2, "mma"), (3, "mma"), (8, "mma")])
 def test_search_bit_widths(cuda_lib, torch_dev, bits, path):
     torch, dev = torch_dev
     tq = cuda_lib
@@ -266,9 +266,13 @@ def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
     off, allow = synth.allowlists(c["src"], tid, values)
     filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=block)
     assert filt.info() == {"n": c["n"], "block": block, "n_tenants": T}
-    ids, sc = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale,
-                          k, filter=filt, allow_off=_t(torch, dev, off),
-                          allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    tq.set_search_path("lut")  # the lookup scan (a batch of 200 would take the tensor-core scan)
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                              c["enc"].scale, k, filter=filt, allow_off=_t(torch, dev, off),
+                              allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    finally:
+        tq.set_search_path("auto")
     ref = O.search(c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"],
                    tid, off, allow)
     allowed = O.allowed_mask(tid, off, allow, len(c["Q"]), c["n"])
@@ -359,11 +363,12 @@ def test_invalid_calls_on_gpu(cuda_lib, torch_dev):
 @pytest.mark.parametrize("bits,d,n,nq,k", [(4, 1536, 3000, 130, 10), (2, 1536, 1000, 17, 5),
                                            (8, 1536, 777, 64, 8), (4, 64, 513, 200, 1),
                                            (4, 2048, 2049, 129, 64), (4, 128, 255, 1, 3),
-                                           (8, 1536, 777, 300, 8), (4, 1536, 1500, 257, 5)])
+                                           (8, 1536, 777, 300, 8), (4, 1536, 1500, 257, 5),
+                                           (3, 1536, 1000, 17, 5), (3, 1536, 777, 300, 8), (3, 256, 600, 40, 10)])
 def test_search_mma_parity(cuda_lib, torch_dev, bits, d, n, nq, k):
     """Query tiles of 128 with a ragged last tile, vector tiles of 256 with a
     ragged tail (rows past n are filled with zeros by the tensor map), one
-    query, k = 1 and 64, 2/4/8-bit codes (fp16 products, float32 sums)."""
+    query, k = 1 and 64, 2/3/4/8-bit codes (fp16 products, float32 sums)."""
     torch, dev = torch_dev
     tq = cuda_lib
     packed = synth.random_codes(n, d * bits // 8, seed=bits * n)
@@ -383,12 +388,12 @@ def test_search_mma_parity(cuda_lib, torch_dev, bits, d, n, nq, k):
 
 def test_search_mma_unsupported(cuda_lib, torch_dev):
     """Forcing the tensor-core scan where it does not apply is an error, not a
-    silent switch: 3-bit codes, k > 64, d not a multiple of 64, a filter."""
+    silent switch: k > 64, d not a multiple of 64 (of 128 for 3-bit codes)."""
     torch, dev = torch_dev
     tq = cuda_lib
     tq.set_search_path("mma")
     try:
-        for bits, d, k in ((3, 1536, 5), (4, 1536, 65), (4, 96, 5)):
+        for bits, d, k in ((3, 160, 5), (4, 1536, 65), (4, 96, 5)):
             Q = torch.zeros((4, d), device=dev)
             R = torch.eye(d, device=dev)
             c = torch.zeros(1 << bits, device=dev)
@@ -484,3 +489,84 @@ def test_search_on_created_stream_matches_default_stream(cuda_lib, torch_dev, fi
         (tid, off, allow) if filtered else ()))
     allowed = O.allowed_mask(tid, off, allow, nq, n) if filtered else np.ones((nq, n), bool)
     check_topk(want_i.cpu().numpy(), want_s.cpu().numpy(), ref.ids, ref.scores64, allowed, k, TOL_LUT)
+
+
+@pytest.mark.parametrize("filtered", [False, True])
+def test_search_host_buffers(cuda_lib, torch_dev, filtered_corpus, filtered):
+    """tq_search_host (queries from page-locked host memory, results back to
+    host memory, all queued by the library on one stream) returns what
+    tq_search on device buffers returns, bit for bit."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    nq, k = 7, 10
+    args = (_t(torch, dev, c["R"]), _t(torch, dev, c["c32"]), c["bits"], _t(torch, dev, c["enc"].packed),
+            _t(torch, dev, c["enc"].scale), k)
+    kw = {}
+    if filtered:
+        tid, values = synth.zipf_tenants(c["n"], 100)
+        off, allow = synth.allowlists(c["src"][:nq], tid, values)
+        kw = dict(filter=tq.Filter(_t(torch, dev, tid.view(np.int32))), allow_off=_t(torch, dev, off),
+                  allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    Qh = torch.from_numpy(c["Q"][:nq].copy()).pin_memory()
+    ih = torch.full((nq, k), 3, dtype=torch.int64).pin_memory()
+    sh = torch.full((nq, k), 3.0, dtype=torch.float32).pin_memory()
+    side = torch.cuda.Stream(device=dev)
+    try:
+        tq.search_from_host(Qh, *args, ih, sh, stream=side, **kw)
+        side.synchronize()
+        want_i, want_s = tq.search(Qh.to(dev), *args, **kw)
+        torch.cuda.synchronize()
+    finally:
+        if filtered:
+            kw["filter"].close()
+    assert torch.equal(ih, want_i.cpu()) and torch.equal(sh, want_s.cpu())
+
+
+@pytest.mark.parametrize("T,nq,k", [(10, 200, 10), (100, 200, 10), (1000, 200, 10), (100, 40, 64)])
+def test_filtered_search_mma(cuda_lib, torch_dev, filtered_corpus, T, nq, k):
+    """Filtered batches on the tensor-core scan: the epilogue drops a vector
+    whose tenant the query does not allow before it can enter the query's
+    list (Sec. III-B).  Two query tiles (nq = 200) and one (nq = 40, k = 64)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    tid, values = synth.zipf_tenants(c["n"], T)
+    off, allow = synth.allowlists(c["src"][:nq], tid, values)
+    filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=64)
+    tq.set_search_path("mma")
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                              c["enc"].scale, k, filter=filt, allow_off=_t(torch, dev, off),
+                              allow_tenants=_t(torch, dev, allow.view(np.int32)))
+    finally:
+        tq.set_search_path("auto")
+        filt.close()
+    ref = O.search(c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"],
+                   tid, off, allow)
+    allowed = O.allowed_mask(tid, off, allow, nq, c["n"])
+    check_topk(ids, sc, ref.ids, ref.scores64, allowed, k, TOL_MMA)
+    exact, _ = O.exact_knn(c["X"], c["Q"][:nq], k, tid, off, allow)
+    assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
+
+
+def test_filter_every_tenant_equals_unfiltered_mma(cuda_lib, torch_dev, filtered_corpus):
+    """On the tensor-core scan, allowing every tenant gives the unfiltered
+    result bit for bit (AUTO picks the tensor-core scan for 40 queries)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    c = filtered_corpus
+    k, nq = 10, 40
+    tid, values = synth.zipf_tenants(c["n"], 100)
+    off = np.arange(nq + 1, dtype=np.int64) * len(values)
+    allow = np.tile(values, nq)
+    filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=64)
+    try:
+        ids_f, sc_f = _gpu_search(tq, torch, dev, c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                                  c["enc"].scale, k, filter=filt, allow_off=_t(torch, dev, off),
+                                  allow_tenants=_t(torch, dev, allow.view(np.int32)))
+        ids_u, sc_u = _gpu_search(tq, torch, dev, c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed,
+                                  c["enc"].scale, k)
+    finally:
+        filt.close()
+    assert np.array_equal(ids_f, ids_u) and np.array_equal(sc_f, sc_u)
