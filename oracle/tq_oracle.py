@@ -16,7 +16,9 @@ numpy/scipy in float64, written step by step from the paper:
   are reported by their external uint64 ids);
 * Sec. IV-A: exact brute-force inner-product ground truth and Recall@k;
   Sec. IV-E: Hit@k and MRR@20 against the exact top-1;
-* Sec. V-C: the over-fetch post-filter baseline that filtering is compared with.
+* Sec. V-C: the over-fetch post-filter baseline that filtering is compared with;
+* Sec. II-B, TQ+: per-coordinate shift and scale from the first batch (a
+  reading; parity unpinned, see `calibrate`).
 
 Readings where the paper is silent:
 * marginal: the exact coordinate density of a uniformly random unit vector,
@@ -323,31 +325,41 @@ def rotate_normalize(X: np.ndarray, R: np.ndarray):
 
 
 def encode(X: np.ndarray, R: np.ndarray, centroids: np.ndarray, boundaries: np.ndarray,
-           bits: int, scale_mode: str = "norm") -> Encoded:
+           bits: int, scale_mode: str = "norm", calib: "Calibration | None" = None) -> Encoded:
     """Encode rows of X.
 
     Step 1: n = ||x||.  Step 2: y = R x / n (y = 0 when n = 0).  Step 3:
     code_j = #{i : t_i < y_j} with y_j rounded to float32 and the float32
     boundaries t.  Step 4: pack.  Step 5: the per-vector scalar (module header).
     R, centroids and boundaries are the float32 arrays the GPU path also gets;
-    they are promoted to float64 here.
+    they are promoted to float64 here.  With a TQ+ calibration the quantiser
+    sees z_j = (y_j - mu_j) / a_j instead of y_j (see `calibrate`).
     """
     y, n = rotate_normalize(X, R)
-    return quantize(y, n, centroids, boundaries, bits, scale_mode)
+    return quantize(y, n, centroids, boundaries, bits, scale_mode, calib)
 
 
 def quantize(y: np.ndarray, n: np.ndarray, centroids: np.ndarray, boundaries: np.ndarray,
-             bits: int, scale_mode: str = "norm") -> Encoded:
+             bits: int, scale_mode: str = "norm", calib: "Calibration | None" = None) -> Encoded:
     """Steps 3-5 of the encoder on rotated, normalised rows y (float64) with
-    norms n: nearest-centroid codes, packing and the per-vector scalar."""
+    norms n: nearest-centroid codes, packing and the per-vector scalar.  With a
+    TQ+ calibration the codes are those of z = (y - mu) / a and the
+    reconstruction the scalar is taken on is y^ = a c[code] + mu; Encoded.y
+    then holds z, the value compared with the boundaries."""
     if scale_mode not in SCALE_MODES:
         raise ValueError(scale_mode)
     c64 = np.asarray(centroids, dtype=np.float32).astype(np.float64)
     t32 = np.asarray(boundaries, dtype=np.float32)
     assert len(c64) == 1 << bits and len(t32) == len(c64) - 1
     nz = n > 0
-    code = np.searchsorted(t32, y.astype(np.float32), side="left").astype(np.uint16)
-    c = c64[code]
+    if calib is not None:
+        yq = (y - calib.mu[None, :]) / calib.a[None, :]
+        code = np.searchsorted(t32, yq.astype(np.float32), side="left").astype(np.uint16)
+        c = calib.a[None, :] * c64[code] + calib.mu[None, :]
+    else:
+        yq = y
+        code = np.searchsorted(t32, y.astype(np.float32), side="left").astype(np.uint16)
+        c = c64[code]
     if scale_mode == "norm":
         cn = np.sqrt(np.sum(c * c, axis=1))
         scale = np.where(nz & (cn > 0), n / np.where(cn > 0, cn, 1.0), 0.0)
@@ -357,16 +369,61 @@ def quantize(y: np.ndarray, n: np.ndarray, centroids: np.ndarray, boundaries: np
         yc = np.sum(y * c, axis=1)
         scale = np.where(nz & (yc != 0), n / np.where(yc != 0, yc, 1.0), 0.0)
     return Encoded(packed=pack(code, bits), scale=scale.astype(np.float32),
-                   codes=code, y=y, norm=n)
+                   codes=code, y=yq, norm=n)
 
 
 def decode(packed: np.ndarray, scale: np.ndarray, R: np.ndarray, centroids: np.ndarray,
-           d: int, bits: int) -> np.ndarray:
-    """Reconstruction x_hat = scale * R^T c[code] (float64 [n, d])."""
+           d: int, bits: int, calib: "Calibration | None" = None) -> np.ndarray:
+    """Reconstruction x_hat = scale * R^T c[code] (float64 [n, d]); with a TQ+
+    calibration x_hat = scale * R^T (a c[code] + mu)."""
     codes = unpack(packed, d, bits)
     c = np.asarray(centroids, dtype=np.float32).astype(np.float64)[codes]
+    if calib is not None:
+        c = calib.a[None, :] * c + calib.mu[None, :]
     R64 = np.asarray(R, dtype=np.float32).astype(np.float64)
     return (c @ R64) * np.asarray(scale, dtype=np.float64)[:, None]
+
+
+# ---------------------------------------------------------------------------
+# TQ+ calibration (Sec. II-B, "TQ+ calibration and data dependence")
+# PARITY UNPINNED as a reading: the paper says only that per-coordinate shift
+# and scale parameters are fitted from the first batch of indexed vectors to
+# align the empirical coordinate quantiles with the canonical marginal, and
+# that only per-coordinate first and second moments are kept.  The pins in the
+# tests check what the mathematics fixes about this reading, not the reading.
+# ---------------------------------------------------------------------------
+@dataclass
+class Calibration:
+    mu: np.ndarray   # float64 [d]: per-coordinate shift (first moment)
+    a: np.ndarray    # float64 [d]: per-coordinate scale (spread / canonical spread)
+
+
+def calibrate(X: np.ndarray, R: np.ndarray) -> Calibration:
+    """Per-coordinate shift and scale from a first batch X of rows.
+
+    Reading: over the batch's non-zero rows, y = R x / ||x|| (steps 1-2 of the
+    encoder); mu_j = mean of y_j and sigma_j = its population standard
+    deviation (the first and second moments); a_j = sigma_j * sqrt(d), the
+    ratio to the canonical marginal's spread (1/sqrt(d) for the coordinate of
+    a uniform unit vector, the Beta marginal, and for N(0, 1/d)), and a_j = 1
+    where sigma_j = 0.  z_j = (y_j - mu_j) / a_j then has the canonical first
+    two moments over the batch, and the canonical codebook quantises z.  A
+    batch without a non-zero row gives mu = 0, a = 1 (plain TurboQuant)."""
+    y, n = rotate_normalize(X, R)
+    d = y.shape[1]
+    y = y[n > 0]
+    if len(y) == 0:
+        return Calibration(mu=np.zeros(d), a=np.ones(d))
+    mu = y.mean(axis=0)
+    sigma = np.sqrt(np.mean((y - mu[None, :]) ** 2, axis=0))
+    a = np.where(sigma > 0, sigma * np.sqrt(d), 1.0)
+    return Calibration(mu=mu, a=a)
+
+
+def calibration32(calib: Calibration) -> Calibration:
+    """The calibration as the float32 values the GPU path is given, promoted."""
+    return Calibration(mu=calib.mu.astype(np.float32).astype(np.float64),
+                       a=calib.a.astype(np.float32).astype(np.float64))
 
 
 # ---------------------------------------------------------------------------
@@ -412,8 +469,11 @@ class SearchResult:
     scores64: np.ndarray   # float64 [nq, n]: every vector's score (allowed or not)
 
 
-def quantized_scores(Q, R, centroids, bits, packed, scale, d, row_chunk=16384) -> np.ndarray:
-    """s[q, i] = scale_i * sum_j q'_j c[code_ij] with q' = R q, float64 [nq, n]."""
+def quantized_scores(Q, R, centroids, bits, packed, scale, d, row_chunk=16384,
+                     calib: Calibration | None = None) -> np.ndarray:
+    """s[q, i] = scale_i * sum_j q'_j c[code_ij] with q' = R q, float64 [nq, n];
+    with a TQ+ calibration the reconstruction a_j c[code_ij] + mu_j takes the
+    place of c[code_ij]."""
     Q64 = np.asarray(Q, dtype=np.float64)
     R64 = np.asarray(R, dtype=np.float32).astype(np.float64)
     c64 = np.asarray(centroids, dtype=np.float32).astype(np.float64)
@@ -424,20 +484,24 @@ def quantized_scores(Q, R, centroids, bits, packed, scale, d, row_chunk=16384) -
     for r0 in range(0, n, row_chunk):
         r1 = min(n, r0 + row_chunk)
         C = c64[unpack(packed[r0:r1], d, bits)]
+        if calib is not None:
+            C = calib.a[None, :] * C + calib.mu[None, :]
         S[:, r0:r1] = (qr @ C.T) * sc[None, r0:r1]
     return S
 
 
 def search(Q, R, centroids, bits, packed, scale, k, d,
-           tenant_ids=None, allow_off=None, allow_ids=None, deleted=None, ext_ids=None) -> SearchResult:
+           tenant_ids=None, allow_off=None, allow_ids=None, deleted=None, ext_ids=None,
+           calib: Calibration | None = None) -> SearchResult:
     """Top-k inner-product search over the quantised corpus.
 
     Id-mapped index (Sec. III-A: external uint64 ids, O(1) deletion): a row
     with deleted[i] True is never returned, exactly like a row whose tenant
     is not allowed; with ext_ids the k rows, ranked as usual (ties by row,
     i.e. insertion order), are reported as ext_ids[row] (their int64 bit
-    pattern; empty slots stay -1)."""
-    S = quantized_scores(Q, R, centroids, bits, packed, scale, d)
+    pattern; empty slots stay -1).  With a TQ+ calibration the scores are
+    those of the calibrated reconstruction (quantized_scores)."""
+    S = quantized_scores(Q, R, centroids, bits, packed, scale, d, calib=calib)
     nq, n = S.shape
     allowed = allowed_mask(tenant_ids, allow_off, allow_ids, nq, n)
     if deleted is not None:

@@ -608,3 +608,99 @@ def test_postfilter_by_hand_and_full_overfetch_equals_filtering(tenant_index):
     small = O.search(Q, R, cb.centroids32, bits, enc.packed, enc.scale, 10, d)
     pf = O.postfilter_topk(small.ids, mask, 10)
     assert O.recall_at_k(pf, filt.ids) < 1.0  # over-fetch 1 loses results of small tenants
+
+
+# ---------------------------------------------------------------- TQ+ ---------
+# The calibration is a reading of the paper (parity unpinned); these pins check
+# what the mathematics fixes about it.
+def _unit(a):
+    a = np.asarray(a, np.float64)
+    return a / np.linalg.norm(a, axis=1, keepdims=True)
+
+
+def test_tqplus_identity_calibration_is_plain_tq():
+    """mu = 0, a = 1 leaves every code, scale and score as plain TurboQuant."""
+    d, bits = 64, 4
+    X = synth.mixture_corpus(300, d, 4, seed=1)
+    R = O.rotation(d, 2).astype(np.float32)
+    cb = O.codebook(d, bits)
+    ident = O.Calibration(mu=np.zeros(d), a=np.ones(d))
+    for mode in O.SCALE_MODES:
+        plain = O.encode(X, R, cb.centroids32, cb.boundaries32, bits, mode)
+        cal = O.encode(X, R, cb.centroids32, cb.boundaries32, bits, mode, calib=ident)
+        assert np.array_equal(plain.packed, cal.packed) and np.array_equal(plain.scale, cal.scale)
+    Q = synth.gaussian_rows(5, d, seed=3)
+    a = O.search(Q, R, cb.centroids32, bits, plain.packed, plain.scale, 7, d)
+    b = O.search(Q, R, cb.centroids32, bits, plain.packed, plain.scale, 7, d, calib=ident)
+    assert np.array_equal(a.ids, b.ids) and np.array_equal(a.scores64, b.scores64)
+
+
+def test_tqplus_on_canonical_data_is_near_identity():
+    """Rows uniform on the sphere already follow the canonical marginal after
+    any rotation: the fitted shift is within sampling error of 0 and the scale
+    of 1, and almost every code is the plain one."""
+    d, n, bits = 256, 20_000, 4
+    X = _unit(np.random.default_rng(7).standard_normal((n, d)))
+    R = O.rotation(d, 3).astype(np.float32)
+    cal = O.calibrate(X, R)
+    assert np.max(np.abs(cal.mu)) < 5 * (1 / np.sqrt(d)) / np.sqrt(n)
+    assert np.max(np.abs(cal.a - 1)) < 5 * np.sqrt(1 / (2 * n)) + 0.01
+    cb = O.codebook(d, bits)
+    plain = O.encode(X[:2000], R, cb.centroids32, cb.boundaries32, bits)
+    tqp = O.encode(X[:2000], R, cb.centroids32, cb.boundaries32, bits, calib=cal)
+    assert np.mean(plain.codes == tqp.codes) > 0.97
+
+
+def test_tqplus_distortion_is_scaled_canonical_distortion():
+    """Coordinates with their own means and spreads (R = identity, Gaussian
+    rows with per-coordinate mean m_j and spread s_j, normalised): after
+    calibration z_j = (y_j - mu_j) / a_j is close to N(0, 1/d), so the
+    per-coordinate error of the reconstruction a_j c + mu_j is a_j^2 D for the
+    Gaussian-marginal codebook's distortion D.  A dropped sqrt(d), a wrong
+    sign of the shift or a misplaced scale breaks this by far more than 3%."""
+    d, n, bits = 256, 40_000, 4
+    rng = np.random.default_rng(11)
+    m = rng.uniform(-0.5, 0.5, d)
+    sd = rng.uniform(0.5, 2.0, d)
+    X = m[None, :] + sd[None, :] * rng.standard_normal((n, d))
+    R = np.eye(d, dtype=np.float32)
+    cal = O.calibrate(X[: n // 2], R)
+    cb = O.codebook(d, bits, "gauss")
+    enc = O.encode(X[n // 2:], R, cb.centroids32, cb.boundaries32, bits, calib=cal)
+    y = _unit(X[n // 2:])
+    yhat = cal.a[None, :] * cb.centroids32.astype(np.float64)[enc.codes] + cal.mu[None, :]
+    ratio = np.mean((y - yhat) ** 2, axis=0) / (cal.a ** 2 * cb.distortion)
+    assert np.mean(ratio) == pytest.approx(1.0, abs=0.03)
+    # plain TurboQuant on the same rows is worse: its cells do not follow the
+    # coordinates' shifted and scaled spread (about 1.6 times the error here)
+    plain = O.encode(X[n // 2:], R, cb.centroids32, cb.boundaries32, bits)
+    err_plain = np.mean((y - cb.centroids32.astype(np.float64)[plain.codes]) ** 2)
+    assert np.mean((y - yhat) ** 2) < 0.75 * err_plain
+
+
+def test_tqplus_score_is_inner_product_with_reconstruction():
+    """The calibrated score s * sum_j q'_j (a_j c_j + mu_j) equals the inner
+    product of the query with the decoded vector s R^T (a c + mu)."""
+    d, bits = 96, 3
+    X = synth.mixture_corpus(200, d, 4, seed=5)
+    R = O.rotation(d, 4).astype(np.float32)
+    cb = O.codebook(d, bits)
+    cal = O.calibrate(X[:100], R)
+    enc = O.encode(X, R, cb.centroids32, cb.boundaries32, bits, calib=cal)
+    Q = synth.gaussian_rows(6, d, seed=6).astype(np.float64)
+    S = O.quantized_scores(Q, R, cb.centroids32, bits, enc.packed, enc.scale, d, calib=cal)
+    Xh = O.decode(enc.packed, enc.scale, R, cb.centroids32, d, bits, calib=cal)
+    assert np.allclose(S, Q @ Xh.T, rtol=1e-12, atol=1e-12)
+    # NORM scaling keeps each row's length: ||x_hat|| = ||x||
+    assert np.allclose(np.linalg.norm(Xh, axis=1), np.linalg.norm(X.astype(np.float64), axis=1), rtol=1e-6)
+
+
+def test_tqplus_degenerate_batches():
+    d = 32
+    R = O.rotation(d, 1).astype(np.float32)
+    cal = O.calibrate(np.zeros((3, d), np.float32), R)  # no non-zero row: plain TurboQuant
+    assert np.array_equal(cal.mu, np.zeros(d)) and np.array_equal(cal.a, np.ones(d))
+    x = synth.gaussian_rows(1, d, seed=2)
+    cal = O.calibrate(np.concatenate([x, np.zeros((1, d), np.float32)]), R)  # one row: no spread
+    y, _ = O.rotate_normalize(x, R)
+    assert np.allclose(cal.mu, y[0], atol=1e-15) and np.array_equal(cal.a, np.ones(d))
