@@ -136,6 +136,34 @@ tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
                     int scale_mode, uint8_t* codes, float* scale, void* stream);
 
 /*
+ * TQ+ calibration (Sec. II-B, "TQ+ calibration and data dependence"): the
+ * paper fits per-coordinate shift and scale parameters from the first batch
+ * of indexed vectors so that the coordinate quantiles match the canonical
+ * marginal, keeping only first and second moments; it gives no formula.  This
+ * library's reading: over the batch's non-zero rows, y = R x / ||x||;
+ * mu_j = mean of y_j, sigma_j = its population standard deviation, a_j =
+ * sigma_j sqrt(d) (the canonical marginal's spread is 1/sqrt(d)), a_j = 1
+ * where sigma_j = 0 (mu = 0, a = 1 without a non-zero row).  Encoding then
+ * quantises z_j = (y_j - mu_j) / a_j with the canonical codebook, and the
+ * reconstruction is a_j c[code_j] + mu_j.
+ *
+ * tq_calibrate_workspace  bytes of device scratch tq_calibrate needs for n rows
+ * tq_calibrate   X device [n*d] float32 (n >= 1), R as for tq_encode;
+ *                mu, a device out [d] float32; deterministic (fixed summation
+ *                order).
+ * tq_encode_ex   tq_encode with a calibration (cal_mu, cal_a device [d], or
+ *                both NULL for plain TurboQuant): codes of z, and the
+ *                per-vector scalar (scale_mode) taken on the reconstruction.
+ */
+tq_status tq_calibrate_workspace(int64_t n, int d, size_t* bytes);
+tq_status tq_calibrate(const float* X, int64_t n, int d, const float* R, float* mu, float* a,
+                       void* workspace, size_t ws_bytes, void* stream);
+tq_status tq_encode_ex(const float* X, int64_t n, int d, const float* R,
+                       const float* centroids, const float* boundaries, int bits,
+                       int scale_mode, const float* cal_mu, const float* cal_a,
+                       uint8_t* codes, float* scale, void* stream);
+
+/*
  * tq_filter_build - per-corpus tenant filter for search(allowlist=...)
  * (Sec. III-B: filtering at vector-block granularity).
  *   tenant_ids  device [n] uint32: the tenant of each vector
@@ -217,7 +245,8 @@ tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
 
 /*
  * tq_search_ex - tq_search over an id-mapped index (Sec. III-A: external
- * uint64 ids, O(1) deletion).  Same arguments and results as tq_search, plus:
+ * uint64 ids, O(1) deletion) and/or a TQ+ index (Sec. II-B).  Same arguments
+ * and results as tq_search, plus:
  *   deleted   device [ceil(n/32)] uint32 tombstone bitmap, or NULL: bit i % 32
  *             of word i / 32 set means row i is deleted and is never returned
  *             (like a vector whose tenant is not allowed)
@@ -226,14 +255,18 @@ tq_status tq_search(const float* Q, int64_t nq, int d, const float* R,
  *             the ranking tie-break stays on the row (insertion order), and
  *             -1 (all ones) still marks an empty slot, so it must not be used
  *             as an external id
- * tq_search(...) is tq_search_ex(..., NULL, NULL, ...).  A tq_idmap handle
- * (below) keeps both arrays and the id -> row map.
+ *   cal_mu, cal_a  device [d] float32 each, or both NULL: the TQ+
+ *             calibration the codes were encoded with (tq_encode_ex); the
+ *             scores are then those of the reconstruction a_j c[code_j] + mu_j
+ * tq_search(...) is tq_search_ex(..., NULL, NULL, NULL, NULL, ...).  A
+ * tq_idmap handle (below) keeps the first two arrays and the id -> row map.
  */
 tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
                        const float* centroids, int bits, const uint8_t* codes,
                        const float* scale, int64_t n, const tq_filter* filter,
                        const int64_t* allow_off, const uint32_t* allow_tenants,
                        const uint32_t* deleted, const uint64_t* ext_ids,
+                       const float* cal_mu, const float* cal_a,
                        int k, int64_t* out_ids, float* out_scores, void* workspace,
                        size_t ws_bytes, void* stream);
 
@@ -249,8 +282,8 @@ tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
  *   staging      device scratch of staging_bytes >= tq_search_host_staging()
  *                (the device copies of the queries and results)
  *   the other arguments as for tq_search_ex (R, centroids, codes, scale,
- *   allow_off, allow_tenants, deleted, ext_ids and workspace are device
- *   memory).
+ *   allow_off, allow_tenants, deleted, ext_ids, cal_mu, cal_a and workspace
+ *   are device memory).
  * The host buffers must stay valid until the copies have run.
  */
 tq_status tq_search_host_staging(int64_t nq, int d, int k, size_t* bytes);
@@ -258,7 +291,8 @@ tq_status tq_search_host(const float* Q_host, int64_t nq, int d, const float* R,
                          const float* centroids, int bits, const uint8_t* codes,
                          const float* scale, int64_t n, const tq_filter* filter,
                          const int64_t* allow_off, const uint32_t* allow_tenants,
-                         const uint32_t* deleted, const uint64_t* ext_ids, int k,
+                         const uint32_t* deleted, const uint64_t* ext_ids,
+                         const float* cal_mu, const float* cal_a, int k,
                          int64_t* ids_host, float* scores_host, void* staging,
                          size_t staging_bytes, void* workspace, size_t ws_bytes,
                          void* stream);

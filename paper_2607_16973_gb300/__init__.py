@@ -13,7 +13,7 @@ import numpy as np
 
 from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
 
-__all__ = ["codebook", "rotation", "encode", "Filter", "IdMap", "Index", "search", "search_workspace",
+__all__ = ["codebook", "rotation", "encode", "calibrate", "Filter", "IdMap", "Index", "search", "search_workspace",
            "search_from_host", "search_host_staging", "search_check", "merge_topk", "set_search_path",
            "profile_events", "row_bytes", "load", "TQError"]
 
@@ -96,8 +96,10 @@ def rotation(d: int, seed: int) -> np.ndarray:
 
 
 def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
-           codes=None, scale=None, stream=None):
-    """tq_encode on CUDA tensors: returns (codes uint8 [n, d*bits/8], scale f32 [n])."""
+           codes=None, scale=None, stream=None, calib=None):
+    """tq_encode (tq_encode_ex with a TQ+ calibration `calib` = (mu, a), CUDA
+    float32 tensors [d]) on CUDA tensors: returns (codes uint8 [n, d*bits/8],
+    scale f32 [n])."""
     torch = _torch()
     n, d = X.shape
     with _on_stream(stream):
@@ -106,11 +108,30 @@ def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
         if scale is None:
             scale = torch.empty(n, dtype=torch.float32, device=X.device)
     f32 = torch.float32
-    check(load().tq_encode(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32),
-                           _dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32),
-                           bits, SCALE_MODES[scale_mode], _dev_ptr(codes, "codes", torch.uint8),
-                           _dev_ptr(scale, "scale", f32), _stream_handle(stream)))
+    mu, a = calib if calib is not None else (None, None)
+    check(load().tq_encode_ex(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32),
+                              _dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32),
+                              bits, SCALE_MODES[scale_mode], _dev_ptr(mu, "mu", f32) or None,
+                              _dev_ptr(a, "a", f32) or None, _dev_ptr(codes, "codes", torch.uint8),
+                              _dev_ptr(scale, "scale", f32), _stream_handle(stream)))
     return codes, scale
+
+
+def calibrate(X, R, stream=None):
+    """tq_calibrate: the TQ+ per-coordinate shift and scale (Sec. II-B) of the
+    rows of X (CUDA float32 [n, d]): returns (mu, a), CUDA float32 [d] each."""
+    torch = _torch()
+    n, d = X.shape
+    need = C.c_size_t()
+    check(load().tq_calibrate_workspace(n, d, C.byref(need)))
+    with _on_stream(stream):
+        ws = torch.empty(max(need.value, 1), dtype=torch.uint8, device=X.device)
+        mu = torch.empty(d, dtype=torch.float32, device=X.device)
+        a = torch.empty(d, dtype=torch.float32, device=X.device)
+    f32 = torch.float32
+    check(load().tq_calibrate(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32), _dev_ptr(mu, "mu"),
+                              _dev_ptr(a, "a"), _dev_ptr(ws, "workspace"), ws.numel(), _stream_handle(stream)))
+    return mu, a
 
 
 class Filter:
@@ -240,10 +261,11 @@ def search_workspace(nq: int, n: int, d: int, bits: int, k: int, filter: Filter 
 
 def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | None = None,
            allow_off=None, allow_tenants=None, workspace=None, out_ids=None, out_scores=None,
-           stream=None, idmap: IdMap | None = None):
+           stream=None, idmap: IdMap | None = None, calib=None):
     """tq_search (tq_search_ex with an IdMap) on CUDA tensors: returns
     (ids int64 [nq, k], scores f32 [nq, k]); with an IdMap the ids are
-    external ids and deleted rows are skipped."""
+    external ids and deleted rows are skipped; `calib` = (mu, a) searches
+    codes encoded with that TQ+ calibration."""
     torch = _torch()
     nq, d = Q.shape
     n = codes.shape[0]
@@ -267,7 +289,9 @@ def search(Q, R, centroids, bits: int, codes, scale, k: int, filter: Filter | No
         _dev_ptr(Q, "Q", f32), nq, d, _dev_ptr(R, "R", f32), _dev_ptr(centroids, "centroids", f32), bits,
         _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), n,
         filter.handle if filter else None, _dev_ptr(allow_off, "allow_off", torch.int64),
-        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None, k,
+        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None,
+        _dev_ptr(calib[0], "mu", f32) if calib is not None else None,
+        _dev_ptr(calib[1], "a", f32) if calib is not None else None, k,
         _dev_ptr(out_ids, "out_ids", torch.int64),
         _dev_ptr(out_scores, "out_scores", f32), _dev_ptr(workspace, "workspace", contiguous=True),
         workspace.numel() * workspace.element_size(), _stream_handle(stream)))
@@ -283,7 +307,7 @@ def search_host_staging(nq: int, d: int, k: int) -> int:
 
 def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, ids_host, scores_host,
                      filter: Filter | None = None, allow_off=None, allow_tenants=None, workspace=None,
-                     staging=None, stream=None, idmap: IdMap | None = None):
+                     staging=None, stream=None, idmap: IdMap | None = None, calib=None):
     """tq_search_host: queries in host memory (a CPU float32 tensor, page-locked
     for asynchronous copies), results into the host tensors ids_host (int64
     [nq, k]) and scores_host (float32 [nq, k]).  The library queues the query
@@ -314,7 +338,9 @@ def search_from_host(Q_host, R, centroids, bits: int, codes, scale, k: int, ids_
         int(Q_host.data_ptr()), nq, d, _dev_ptr(R, "R", f32), _dev_ptr(centroids, "centroids", f32), bits,
         _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), n,
         filter.handle if filter else None, _dev_ptr(allow_off, "allow_off", torch.int64),
-        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None, k,
+        _dev_ptr(allow_tenants, "allow_tenants", u32), deleted or None, ext or None,
+        _dev_ptr(calib[0], "mu", f32) if calib is not None else None,
+        _dev_ptr(calib[1], "a", f32) if calib is not None else None, k,
         int(ids_host.data_ptr()), int(scores_host.data_ptr()), _dev_ptr(staging, "staging"),
         staging.numel() * staging.element_size(), _dev_ptr(workspace, "workspace"),
         workspace.numel() * workspace.element_size(), _stream_handle(stream)))

@@ -31,13 +31,13 @@ inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct SearchPlan {
   int grid_lut = 1, grid_mma = 0;
-  size_t off_status = 0, off_cnt = 0, off_rot = 0, off_allow = 0, off_mask = 0, off_qpack = 0, off_cs = 0,
-         off_ci = 0, total = 0;
+  size_t off_status = 0, off_cnt = 0, off_bias = 0, off_rot = 0, off_allow = 0, off_mask = 0, off_qpack = 0,
+         off_cs = 0, off_ci = 0, total = 0;
 };
 
 // Workspace layout (both scan paths): status word | merge counters (one per
-// query) | rotated queries | allow bitmaps | block masks | fp16 query tiles
-// (tensor-core path) | candidate scores | ids.
+// query) | TQ+ query terms (one per query) | rotated queries | allow bitmaps |
+// block masks | fp16 query tiles (tensor-core path) | candidate scores | ids.
 SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
   SearchPlan p;
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
@@ -49,6 +49,8 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   off = align_up(off + sizeof(int));
   p.off_cnt = off;
   off = align_up(off + (size_t)nq * sizeof(int));
+  p.off_bias = off;
+  off = align_up(off + (size_t)nq * sizeof(float));
   p.off_rot = off;
   off = align_up(off + (size_t)nq * d * sizeof(float));
   p.off_allow = off;
@@ -70,9 +72,10 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
 
 using tq::fail;
 
-extern "C" tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
-                               const float* centroids, const float* boundaries, int bits,
-                               int scale_mode, uint8_t* codes, float* scale, void* stream) {
+extern "C" tq_status tq_encode_ex(const float* X, int64_t n, int d, const float* R,
+                                  const float* centroids, const float* boundaries, int bits,
+                                  int scale_mode, const float* cal_mu, const float* cal_a, uint8_t* codes,
+                                  float* scale, void* stream) {
   tq_status st = tq::check_common("tq_encode", d, bits);
   if (st != TQ_OK) return st;
   if (n < 0 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_encode: n=%lld outside [0, 2^31-1]", (long long)n);
@@ -85,9 +88,43 @@ extern "C" tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
     return fail(TQ_EINVAL, "tq_encode: X, R and codes must be 16-byte aligned");
   if (((uintptr_t)scale & 3u) || ((uintptr_t)centroids & 3u) || ((uintptr_t)boundaries & 3u))
     return fail(TQ_EINVAL, "tq_encode: scale, centroids and boundaries must be 4-byte aligned");
-  cudaError_t e = tq::launch_encode(X, n, d, R, centroids, boundaries, bits, scale_mode, codes, scale,
-                                    (cudaStream_t)stream);
+  if ((cal_mu == nullptr) != (cal_a == nullptr))
+    return fail(TQ_EINVAL, "tq_encode_ex: a TQ+ calibration needs both mu and a");
+  if (((uintptr_t)cal_mu & 3u) || ((uintptr_t)cal_a & 3u))
+    return fail(TQ_EINVAL, "tq_encode_ex: mu and a must be 4-byte aligned");
+  cudaError_t e = tq::launch_encode(X, n, d, R, centroids, boundaries, bits, scale_mode, cal_mu, cal_a, codes,
+                                    scale, (cudaStream_t)stream);
   if (e != cudaSuccess) return tq::cuda_fail("tq_encode", e);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,
+                               const float* boundaries, int bits, int scale_mode, uint8_t* codes, float* scale,
+                               void* stream) {
+  return tq_encode_ex(X, n, d, R, centroids, boundaries, bits, scale_mode, nullptr, nullptr, codes, scale, stream);
+}
+
+extern "C" tq_status tq_calibrate_workspace(int64_t n, int d, size_t* bytes) {
+  if (!bytes) return fail(TQ_EINVAL, "tq_calibrate_workspace: NULL bytes");
+  if (n < 1 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_calibrate_workspace: n=%lld outside [1, 2^31-1]", (long long)n);
+  if (d < 32 || d > tq::kMaxD || d % 32 != 0)
+    return fail(TQ_EINVAL, "tq_calibrate_workspace: d=%d must be a multiple of 32 in [32, %d]", d, tq::kMaxD);
+  *bytes = tq::calibrate_workspace(n, d);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_calibrate(const float* X, int64_t n, int d, const float* R, float* mu, float* a,
+                                  void* workspace, size_t ws_bytes, void* stream) {
+  size_t need = 0;
+  tq_status st = tq_calibrate_workspace(n, d, &need);
+  if (st != TQ_OK) return st;
+  if (!X || !R || !mu || !a || !workspace) return fail(TQ_EINVAL, "tq_calibrate: NULL device pointer");
+  if (!tq::aligned16(X) || !tq::aligned16(R) || !tq::aligned16(workspace))
+    return fail(TQ_EINVAL, "tq_calibrate: X, R and workspace must be 16-byte aligned");
+  if (((uintptr_t)mu & 3u) || ((uintptr_t)a & 3u)) return fail(TQ_EINVAL, "tq_calibrate: misaligned mu or a");
+  if (ws_bytes < need) return fail(TQ_EINVAL, "tq_calibrate: workspace of %zu bytes, %zu needed", ws_bytes, need);
+  const cudaError_t e = tq::launch_calibrate(X, n, d, R, mu, a, workspace, (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_calibrate", e);
   return tq::ok();
 }
 
@@ -285,8 +322,8 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
                                   const float* centroids, int bits, const uint8_t* codes,
                                   const float* scale, int64_t n, const tq_filter* filter,
                                   const int64_t* allow_off, const uint32_t* allow_tenants,
-                                  const uint32_t* deleted, const uint64_t* ext_ids, int k,
-                                  int64_t* out_ids, float* out_scores, void* workspace,
+                                  const uint32_t* deleted, const uint64_t* ext_ids, const float* cal_mu,
+                                  const float* cal_a, int k, int64_t* out_ids, float* out_scores, void* workspace,
                                   size_t ws_bytes, void* stream) {
   tq_status st = check_search(nq, n, d, bits, k);
   if (st != TQ_OK) return st;
@@ -307,6 +344,10 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
     if (((uintptr_t)allow_off & 7u) || ((uintptr_t)allow_tenants & 3u))
       return fail(TQ_EINVAL, "tq_search: misaligned allowlist pointers");
   }
+  if ((cal_mu == nullptr) != (cal_a == nullptr))
+    return fail(TQ_EINVAL, "tq_search_ex: a TQ+ calibration needs both mu and a");
+  if (((uintptr_t)cal_mu & 3u) || ((uintptr_t)cal_a & 3u))
+    return fail(TQ_EINVAL, "tq_search_ex: mu and a must be 4-byte aligned");
   const int path = tq::search_path();
   const bool can_mma = tq::mma_supported(bits, d, k);
   if (path == TQ_PATH_MMA && !can_mma)
@@ -325,12 +366,14 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
   uint32_t* bmask = filter ? reinterpret_cast<uint32_t*>(ws + p.off_mask) : nullptr;
   float* cs = reinterpret_cast<float*>(ws + p.off_cs);
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
+  float* bias = cal_mu ? reinterpret_cast<float*>(ws + p.off_bias) : nullptr;
   cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);  // also zeroes both
+  if (e == cudaSuccess && cal_mu) e = tq::launch_calib_query(qrot, nq, d, cal_mu, cal_a, bias, s);
   if (use_mma) {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
     if (e == cudaSuccess)
       e = tq::launch_scan_mma(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
-                              filter ? filter->f.dense : nullptr, allow, filter ? filter->f.words : 0, k,
+                              filter ? filter->f.dense : nullptr, allow, filter ? filter->f.words : 0, bias, k,
                               p.grid_mma, ws + p.off_qpack, cs, ci, status, s, (cudaEvent_t)tq::profile_start(),
                               (cudaEvent_t)tq::profile_stop());
     if (e == cudaSuccess) e = tq::launch_merge(cs, ci, nq, p.grid_mma * k, k, ext_ids, out_ids, out_scores, s);
@@ -341,7 +384,7 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
       e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
                               filter ? &filter->f : nullptr, allow, bmask,
                               path == TQ_PATH_LUT_FIXED && d >= tq::kFixMinD,
-                              k, p.grid_lut, cs, ci, status, counters, ext_ids, out_ids, out_scores, s,
+                              k, p.grid_lut, cs, ci, status, counters, ext_ids, out_ids, out_scores, bias, s,
                               (cudaEvent_t)tq::profile_start(), (cudaEvent_t)tq::profile_stop());
   }
   if (e != cudaSuccess) return tq::cuda_fail("tq_search", e);
@@ -355,7 +398,7 @@ extern "C" tq_status tq_search(const float* Q, int64_t nq, int d, const float* R
                                int64_t* out_ids, float* out_scores, void* workspace,
                                size_t ws_bytes, void* stream) {
   return tq_search_ex(Q, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, nullptr,
-                      nullptr, k, out_ids, out_scores, workspace, ws_bytes, stream);
+                      nullptr, nullptr, nullptr, k, out_ids, out_scores, workspace, ws_bytes, stream);
 }
 
 namespace {
@@ -384,8 +427,8 @@ extern "C" tq_status tq_search_host(const float* Q_host, int64_t nq, int d, cons
                                     const float* centroids, int bits, const uint8_t* codes,
                                     const float* scale, int64_t n, const tq_filter* filter,
                                     const int64_t* allow_off, const uint32_t* allow_tenants,
-                                    const uint32_t* deleted, const uint64_t* ext_ids, int k,
-                                    int64_t* ids_host, float* scores_host, void* staging,
+                                    const uint32_t* deleted, const uint64_t* ext_ids, const float* cal_mu,
+                                    const float* cal_a, int k, int64_t* ids_host, float* scores_host, void* staging,
                                     size_t staging_bytes, void* workspace, size_t ws_bytes, void* stream) {
   tq_status st = check_search(nq, n, d, bits, k);
   if (st != TQ_OK) return st;
@@ -404,7 +447,7 @@ extern "C" tq_status tq_search_host(const float* Q_host, int64_t nq, int d, cons
   cudaError_t e = cudaMemcpyAsync(q_dev, Q_host, (size_t)nq * d * sizeof(float), cudaMemcpyHostToDevice, s);
   if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: query copy", e);
   st = tq_search_ex(q_dev, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, deleted,
-                    ext_ids, k, ids_dev, scores_dev, workspace, ws_bytes, stream);
+                    ext_ids, cal_mu, cal_a, k, ids_dev, scores_dev, workspace, ws_bytes, stream);
   if (st != TQ_OK) return st;
   e = cudaMemcpyAsync(ids_host, ids_dev, (size_t)nq * k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
   if (e == cudaSuccess)

@@ -98,12 +98,17 @@ struct EncodeSmem {
   uint8_t ctile[BM][BN + 8];  // row stride 136 B keeps 8-byte reads aligned
   float norm[BM], inv[BM], sum_c2[BM], sum_yc[BM];
   float bnd[255], cen[256];
+  float cmu[BN], ca[BN], cinv[BN];  // TQ+ shift, scale and 1/scale of the tile's columns
 };
 
-template <int BITS>
+// With CAL (a TQ+ calibration, Sec. II-B): the quantiser sees z = (y - mu) /
+// a per coordinate, and the per-vector scalar is taken on the reconstruction
+// a c + mu.
+template <int BITS, bool CAL>
 __global__ void __launch_bounds__(NT, 2)
 k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict__ R,
          const float* __restrict__ centroids, const float* __restrict__ boundaries, int scale_mode,
+         const float* __restrict__ cal_mu, const float* __restrict__ cal_a,
          uint8_t* __restrict__ codes, float* __restrict__ scale) {
   constexpr int L = 1 << BITS;
   __shared__ EncodeSmem sm;
@@ -142,9 +147,17 @@ k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict_
     __syncthreads();
     for (int nt = 0; nt < ntiles; ++nt) {
       const int col0 = nt * BN;
+      if constexpr (CAL) {
+        for (int c = tid; c < BN; c += NT) {
+          const bool in = col0 + c < d;
+          sm.cmu[c] = in ? cal_mu[col0 + c] : 0.f;
+          sm.ca[c] = in ? cal_a[col0 + c] : 1.f;
+          sm.cinv[c] = 1.0f / sm.ca[c];
+        }  // read after gemm_tile's barriers
+      }
       float acc[8][8];
       gemm_tile(X, row0, n, R, col0, d, sm.g, acc);
-      // step 2-3: y = acc / ||x||, code = #{t < y}
+      // step 2-3: y = acc / ||x||, code = #{t < y} (of z = (y - mu) / a with TQ+)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int r = tile_row(i);
@@ -157,11 +170,12 @@ k_encode(const float* __restrict__ X, int64_t n, int d, const float* __restrict_
           for (int jj = 0; jj < 4; ++jj) {
             const int j = jh * 4 + jj;
             const float y = acc[i][j] * inv;
+            const float zq = CAL ? (y - sm.cmu[tile_col(j)]) * sm.cinv[tile_col(j)] : y;
             int code = 0;
 #pragma unroll
             for (int step = L / 2; step >= 1; step >>= 1)
-              if (y > sm.bnd[code + step - 1]) code += step;
-            const float c = sm.cen[code];
+              if (zq > sm.bnd[code + step - 1]) code += step;
+            const float c = CAL ? fmaf(sm.ca[tile_col(j)], sm.cen[code], sm.cmu[tile_col(j)]) : sm.cen[code];
             if (col0 + tile_col(j) < d) {
               pc2 = fmaf(c, c, pc2);
               pyc = fmaf(y, c, pyc);
@@ -328,6 +342,151 @@ k_rotate_gemv(const float* __restrict__ Q, int64_t nq, int d, const float* __res
   }
 }
 
+// TQ+ calibration (Sec. II-B), pass 1: for each 128-row panel, the sums of y
+// and y^2 (y = R x / ||x||) of every coordinate over the panel's non-zero
+// rows, and their count.  Each CTA walks whole panels and sums in a fixed
+// order, so the result does not depend on scheduling.  The sums are kept in
+// double: y^2 of a float32 y is exact there, so a coordinate that takes one
+// value over the batch comes out with a variance of exactly 0.
+__global__ void __launch_bounds__(NT, 2)
+k_calib_partial(const float* __restrict__ X, int64_t n, int d, const float* __restrict__ R,
+                double* __restrict__ psum, double* __restrict__ psq, int* __restrict__ pcount) {
+  __shared__ GemmSmem g;
+  __shared__ float inv[BM];
+  __shared__ int nz;
+  __shared__ double red1[8][BN], red2[8][BN];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int64_t panels = (n + BM - 1) / BM;
+  const int ntiles = (d + BN - 1) / BN;
+  for (int64_t p = blockIdx.x; p < panels; p += gridDim.x) {
+    const int64_t row0 = p * BM;
+    if (tid == 0) nz = 0;
+    __syncthreads();
+    for (int r = warp; r < BM; r += NT / 32) {
+      float sq = 0.f;
+      if (row0 + r < n) {
+        const float4* xr = reinterpret_cast<const float4*>(X + (row0 + r) * d);
+        for (int j = lane; j < d / 4; j += 32) {
+          const float4 v = __ldg(xr + j);
+          sq = fmaf(v.x, v.x, sq);
+          sq = fmaf(v.y, v.y, sq);
+          sq = fmaf(v.z, v.z, sq);
+          sq = fmaf(v.w, v.w, sq);
+        }
+      }
+#pragma unroll
+      for (int o = 16; o; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+      if (lane == 0) {
+        const float nr = sqrtf(sq);
+        inv[r] = nr > 0.f ? 1.0f / nr : 0.f;
+        if (nr > 0.f) atomicAdd(&nz, 1);
+      }
+    }
+    __syncthreads();
+    if (tid == 0) pcount[p] = nz;
+    for (int nt = 0; nt < ntiles; ++nt) {
+      const int col0 = nt * BN;
+      float acc[8][8];
+      gemm_tile(X, row0, n, R, col0, d, g, acc);
+      double s1[8], s2[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        s1[j] = 0.0;
+        s2[j] = 0.0;
+      }
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const float iv = inv[tile_row(i)];  // 0 for a zero row or a row past n: adds nothing
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const double y = (double)(acc[i][j] * iv);
+          s1[j] += y;
+          s2[j] = fma(y, y, s2[j]);
+        }
+      }
+      // rows ty (even) and ty + 1 (lanes 0-15 and 16-31 of one warp) first
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        s1[j] += __shfl_xor_sync(0xffffffffu, s1[j], 16);
+        s2[j] += __shfl_xor_sync(0xffffffffu, s2[j], 16);
+      }
+      if ((lane & 16) == 0) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          red1[warp][tile_col(j)] = s1[j];
+          red2[warp][tile_col(j)] = s2[j];
+        }
+      }
+      __syncthreads();
+      for (int c = tid; c < BN; c += NT) {
+        if (col0 + c >= d) continue;
+        double a = 0.0, b = 0.0;
+        for (int t = 0; t < 8; ++t) {
+          a += red1[t][c];
+          b += red2[t][c];
+        }
+        psum[p * d + col0 + c] = a;
+        psq[p * d + col0 + c] = b;
+      }
+      __syncthreads();
+    }
+  }
+}
+
+// Pass 2: per coordinate, the panels' sums added in panel order (in double):
+// mu = mean, sigma = population standard deviation, a = sigma sqrt(d) (a = 1
+// where sigma = 0; mu = 0, a = 1 without a non-zero row).
+__global__ void k_calib_finish(const double* __restrict__ psum, const double* __restrict__ psq,
+                               const int* __restrict__ pcount, int64_t panels, int d, float* __restrict__ mu,
+                               float* __restrict__ a) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= d) return;
+  double s1 = 0.0, s2 = 0.0;
+  int64_t cnt = 0;
+  for (int64_t p = 0; p < panels; ++p) {
+    s1 += psum[p * d + j];
+    s2 += psq[p * d + j];
+    cnt += pcount[p];
+  }
+  if (cnt == 0) {
+    mu[j] = 0.f;
+    a[j] = 1.f;
+    return;
+  }
+  const double m = s1 / (double)cnt;
+  const double var = fmax(s2 / (double)cnt - m * m, 0.0);
+  const double sg = sqrt(var);
+  mu[j] = (float)m;
+  a[j] = sg > 0.0 ? (float)(sg * sqrt((double)d)) : 1.f;
+}
+
+// A search over a TQ+ index: q''_j = a_j q'_j (in place) and the query's bias
+// b = sum_j q'_j mu_j, so that scale * (q'' . c[code] + b) = scale * q' .
+// (a c[code] + mu).  One block per query, fixed summation order.
+__global__ void __launch_bounds__(256)
+k_calib_query(float* __restrict__ qrot, int64_t nq, int d, const float* __restrict__ mu,
+              const float* __restrict__ a, float* __restrict__ bias) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  __shared__ float red[8];
+  const int64_t q = blockIdx.x;
+  float* qq = qrot + q * d;
+  float b = 0.f;
+  for (int j = threadIdx.x; j < d; j += blockDim.x) {
+    const float v = qq[j];
+    b = fmaf(v, mu[j], b);
+    qq[j] = v * a[j];
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) b += __shfl_xor_sync(0xffffffffu, b, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = b;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float t = 0.f;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+    bias[q] = t;
+  }
+}
+
 }  // namespace
 
 // SM count of the current device, queried once per device.
@@ -373,18 +532,29 @@ cudaError_t set_max_dynamic_smem(const void* func, int bytes) {
 }
 
 cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,
-                          const float* boundaries, int bits, int scale_mode, uint8_t* codes,
-                          float* scale, cudaStream_t s) {
+                          const float* boundaries, int bits, int scale_mode, const float* cal_mu,
+                          const float* cal_a, uint8_t* codes, float* scale, cudaStream_t s) {
   if (n == 0) return cudaSuccess;
   const int64_t panels = (n + BM - 1) / BM;
   const int grid = (int)std::min<int64_t>(panels, (int64_t)device_sm_count() * 2);
+  const bool cal = cal_mu != nullptr;
+#define TQ_ENC_CASE(B)                                                                                       \
+  case B:                                                                                                    \
+    if (cal)                                                                                                 \
+      k_encode<B, true><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, cal_mu, cal_a,   \
+                                            codes, scale);                                                   \
+    else                                                                                                     \
+      k_encode<B, false><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, nullptr, nullptr, \
+                                             codes, scale);                                                  \
+    break;
   switch (bits) {
-    case 2: k_encode<2><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
-    case 3: k_encode<3><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
-    case 4: k_encode<4><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
-    case 8: k_encode<8><<<grid, NT, 0, s>>>(X, n, d, R, centroids, boundaries, scale_mode, codes, scale); break;
+    TQ_ENC_CASE(2)
+    TQ_ENC_CASE(3)
+    TQ_ENC_CASE(4)
+    TQ_ENC_CASE(8)
     default: return cudaErrorInvalidValue;
   }
+#undef TQ_ENC_CASE
   return cudaGetLastError();
 }
 
@@ -417,6 +587,36 @@ cudaError_t launch_rotate(const float* Q, int64_t nq, int d, const float* R, flo
   }
   dim3 grid((unsigned)((nq + BM - 1) / BM), (unsigned)((d + BN - 1) / BN), split ? 2u : 1u);
   k_rotate_gemm<<<grid, NT, 0, s>>>(Q, nq, d, R, out, status, counters, n_counters);
+  return cudaGetLastError();
+}
+
+}  // namespace tq
+
+namespace tq {
+
+size_t calibrate_workspace(int64_t n, int d) {
+  const int64_t panels = (n + BM - 1) / BM;
+  return (size_t)panels * d * 2 * sizeof(double) + (size_t)panels * sizeof(int);
+}
+
+cudaError_t launch_calibrate(const float* X, int64_t n, int d, const float* R, float* mu, float* a, void* ws,
+                             cudaStream_t s) {
+  const int64_t panels = (n + BM - 1) / BM;
+  double* psum = static_cast<double*>(ws);
+  double* psq = psum + (size_t)panels * d;
+  int* pcount = reinterpret_cast<int*>(psq + (size_t)panels * d);
+  const int grid = (int)std::min<int64_t>(panels, (int64_t)device_sm_count() * 2);
+  k_calib_partial<<<grid, NT, 0, s>>>(X, n, d, R, psum, psq, pcount);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_calib_finish<<<(d + 255) / 256, 256, 0, s>>>(psum, psq, pcount, panels, d, mu, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_calib_query(float* qrot, int64_t nq, int d, const float* mu, const float* a, float* bias,
+                               cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  k_calib_query<<<(unsigned)nq, 256, 0, s>>>(qrot, nq, d, mu, a, bias);
   return cudaGetLastError();
 }
 

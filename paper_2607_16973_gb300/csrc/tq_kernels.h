@@ -19,10 +19,20 @@ struct FilterDev {
   uint32_t* block_bits = nullptr; // device [nblocks * words]
 };
 
-// Encode (Sec. II-B steps 1-5): fused rotation GEMM + quantise + pack + scale.
+// Encode (Sec. II-B steps 1-5): fused rotation GEMM + quantise + pack + scale;
+// with cal_mu/cal_a (nullable, device [d]) a TQ+ calibration.
 cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, const float* centroids,
-                          const float* boundaries, int bits, int scale_mode, uint8_t* codes,
-                          float* scale, cudaStream_t s);
+                          const float* boundaries, int bits, int scale_mode, const float* cal_mu,
+                          const float* cal_a, uint8_t* codes, float* scale, cudaStream_t s);
+
+// TQ+ calibration (Sec. II-B): per-coordinate shift mu and scale a from n
+// rows, into device [d] arrays; ws of calibrate_workspace(n, d) bytes.
+size_t calibrate_workspace(int64_t n, int d);
+cudaError_t launch_calibrate(const float* X, int64_t n, int d, const float* R, float* mu, float* a, void* ws,
+                             cudaStream_t s);
+// Queries of a TQ+ search: qrot *= a in place, bias[q] = sum_j qrot_j mu_j.
+cudaError_t launch_calib_query(float* qrot, int64_t nq, int d, const float* mu, const float* a, float* bias,
+                               cudaStream_t s);
 
 // q' = R q for nq queries: out [nq * d] float32.  Also zeroes the status word
 // and `n_counters` merge counters (each nullable) for the search it starts.
@@ -50,14 +60,15 @@ cudaError_t launch_filter_raw_ids(const FilterDev& f, uint32_t* raw, cudaStream_
 // `err` is the search status word the scan's bounded waits report to.  The
 // last CTA of each query merges the CTA lists into out_ids/out_scores
 // (written as ext[row] with an id map); `counters` [nq] must be zero (the
-// query rotation zeroes them).
+// query rotation zeroes them).  `bias` [nq] (nullable): a TQ+ search's
+// per-query term, added to each raw score before the per-vector scale.
 int scan_lut_grid_x(int64_t nq, int64_t n, int k, int bits, int d);
 cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
                             const FilterDev* f, const uint32_t* allow_bits, const uint32_t* bmask, bool fix,
                             int k, int grid_x, float* cand_s, int32_t* cand_i, int* err, int* counters,
-                            const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s,
-                            cudaEvent_t ev0, cudaEvent_t ev1);
+                            const uint64_t* ext, int64_t* out_ids, float* out_scores, const float* bias,
+                            cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1);
 
 // Per-query bitmap over the filter's blocks: bit b set when block b holds a
 // tenant the query allows.  out [nq * filter_mask_words(f)].
@@ -83,8 +94,8 @@ int scan_mma_grid_x(int64_t nq, int64_t n, int k, int bits);
 size_t mma_qpack_bytes(int64_t nq, int d);
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
-                            const uint32_t* dense, const uint32_t* allow_bits, int words, int k,
-                            int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
+                            const uint32_t* dense, const uint32_t* allow_bits, int words, const float* bias,
+                            int k, int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1);
 
 int device_sm_count();

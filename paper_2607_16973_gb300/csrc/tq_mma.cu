@@ -361,8 +361,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,
            const float* __restrict__ centroids, const float* __restrict__ scale,
            const uint32_t* __restrict__ del, const uint32_t* __restrict__ dense,
-           const uint32_t* __restrict__ allow_bits, int words, int n, int nq, int d,
-           int k, int cst, int ast, int rr, int sub, int ng, int gact, float* __restrict__ cand_s,
+           const uint32_t* __restrict__ allow_bits, int words, const float* __restrict__ bias, int n, int nq,
+           int d, int k, int cst, int ast, int rr, int sub, int ng, int gact, float* __restrict__ cand_s,
            int* __restrict__ cand_i, int* __restrict__ err) {
   constexpr int RAWB = raw_bytes_per_row<BITS>();
   // A code tile carries `sub` consecutive K-blocks of 256 rows: rows of
@@ -628,6 +628,7 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
     const int q = (qt0 + jsel) * MMA_M + row;
     // a filtered search: this query's allow bitmap over the dense tenant index
     const uint32_t* ab = allow_bits && q < nq ? allow_bits + (size_t)q * words : nullptr;
+    const float bq = bias && q < nq ? bias[q] : 0.f;  // a TQ+ index's per-query term (else 0)
     float* ls = lst_s + jsel * k * MMA_M;
     int* li = lst_i + jsel * k * MMA_M;
     if (mine) {
@@ -701,9 +702,10 @@ k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restri
 #pragma unroll
           for (int jj = 0; jj < 16; jj += 4) {
             const float4 s4 = *reinterpret_cast<const float4*>(sScale + c0 + jj);
-            const float2 x = __fmul2_rn(make_float2(__uint_as_float(r[jj]), __uint_as_float(r[jj + 1])),
+            const float2 x = __fmul2_rn(make_float2(__uint_as_float(r[jj]) + bq, __uint_as_float(r[jj + 1]) + bq),
                                         make_float2(s4.x, s4.y));
-            const float2 y = __fmul2_rn(make_float2(__uint_as_float(r[jj + 2]), __uint_as_float(r[jj + 3])),
+            const float2 y = __fmul2_rn(make_float2(__uint_as_float(r[jj + 2]) + bq,
+                                                    __uint_as_float(r[jj + 3]) + bq),
                                         make_float2(s4.z, s4.w));
             r[jj] = __float_as_uint(x.x);
             r[jj + 1] = __float_as_uint(x.y);
@@ -822,15 +824,16 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
 template <int BITS, int QT>
 cudaError_t launch_typed(const MmaPlan& P, const CUtensorMap& map, const __half* qpack, const float* centroids,
                          const float* scale, const uint32_t* del, const uint32_t* dense, const uint32_t* allow,
-                         int words, int n, int nq, int d, int k, int sub, int grid_x, float* cs, int* ci, int* err,
-                         cudaStream_t s) {
+                         int words, const float* bias, int n, int nq, int d, int k, int sub, int grid_x, float* cs,
+                         int* ci, int* err, cudaStream_t s) {
   const int gact = active_groups(P.ng, sub, P.cst);
   cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_scan_mma<BITS, QT>), (int)P.smem);
   if (e != cudaSuccess) return e;
   const int nqt = (nq + MMA_M - 1) / MMA_M;
   const dim3 grid((unsigned)grid_x, (unsigned)((nqt + QT - 1) / QT));
-  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, del, dense, allow, words, n, nq,
-                                                         d, k, P.cst, P.ast, P.rr, sub, P.ng, gact, cs, ci, err);
+  k_scan_mma<BITS, QT><<<grid, NTHREADS, P.smem, s>>>(map, qpack, centroids, scale, del, dense, allow, words, bias,
+                                                         n, nq, d, k, P.cst, P.ast, P.rr, sub, P.ng, gact, cs, ci,
+                                                         err);
   return cudaGetLastError();
 }
 
@@ -864,8 +867,8 @@ size_t mma_qpack_bytes(int64_t nq, int d) {
 
 cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* centroids, int bits,
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
-                            const uint32_t* dense, const uint32_t* allow_bits, int words, int k,
-                            int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
+                            const uint32_t* dense, const uint32_t* allow_bits, int words, const float* bias,
+                            int k, int grid_x, void* qpack, float* cand_s, int32_t* cand_i, int* err, cudaStream_t s,
                             cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
   PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
@@ -896,10 +899,10 @@ cudaError_t launch_scan_mma(const float* qrot, int64_t nq, int d, const float* c
   const __half* qp = static_cast<const __half*>(qpack);
 #define TQ_MMA_CASE(B)                                                                                \
   case B:                                                                                             \
-    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, del, dense, allow_bits, words, (int)n, \
-                                       (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s)                 \
-                  : launch_typed<B, 1>(P, map, qp, centroids, scale, del, dense, allow_bits, words, (int)n, \
-                                       (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s);                \
+    e = P.qt == 2 ? launch_typed<B, 2>(P, map, qp, centroids, scale, del, dense, allow_bits, words, bias, \
+                                       (int)n, (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s)        \
+                  : launch_typed<B, 1>(P, map, qp, centroids, scale, del, dense, allow_bits, words, bias, \
+                                       (int)n, (int)nq, d, k, sub, grid_x, cand_s, cand_i, err, s);       \
     break;
   switch (bits) {
     TQ_MMA_CASE(2)

@@ -548,7 +548,7 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
               const uint32_t* __restrict__ allow_bits, int words, const uint32_t* __restrict__ bmask,
               int mask_words, int fblock, int k, int P, float* __restrict__ cand_s, int* __restrict__ cand_i,
               int* __restrict__ counters, const uint64_t* __restrict__ ext, int64_t* __restrict__ out_ids,
-              float* __restrict__ out_scores) {
+              float* __restrict__ out_scores, const float* __restrict__ bias) {
   constexpr int L = 1 << BITS;
   constexpr int CB = 2 * BITS;   // bytes of a 16-code chunk
   constexpr int V = 4;           // vectors per warp step; a CTA step covers 32
@@ -574,6 +574,7 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
     li[i] = INT_MAX;
   }
   griddep_wait();  // the rotated queries (and allow bitmaps, block masks) are written
+  const float bq = bias ? bias[q] : 0.f;  // a TQ+ index's per-query term (else 0)
   const int nchunks = d >> 4;
   const float* qq = qrot + (size_t)q * d;
   float qr[PAIR ? 1 : S][16];
@@ -681,7 +682,7 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
     float score = -INFINITY;
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
-      score = total * sc_cur;
+      score = (total + bq) * sc_cur;
       const bool allowed = !FILT || ((__ldg(ab + (tn_cur >> 5)) >> (tn_cur & 31)) & 1u);
       cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
@@ -789,7 +790,7 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
             const uint32_t* __restrict__ allow_bits, int words, const uint32_t* __restrict__ bmask, int mask_words,
             int fblock, int k, int P, int ns, float* __restrict__ cand_s, int* __restrict__ cand_i,
             int* __restrict__ err, int* __restrict__ counters, const uint64_t* __restrict__ ext,
-            int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+            int64_t* __restrict__ out_ids, float* __restrict__ out_scores, const float* __restrict__ bias) {
   constexpr int L = 1 << BITS;
   constexpr int CB = 2 * BITS;
   constexpr int V = 4;
@@ -862,6 +863,7 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
     li[i] = INT_MAX;
   }
   if constexpr (!FILT) griddep_wait();  // the rotated queries are written
+  const float bq = bias ? bias[q] : 0.f;  // a TQ+ index's per-query term (else 0)
   const int nchunks = d >> 4;
   const float* qq = qrot + (size_t)q * d;
   float qr[PAIR ? 1 : S][16];
@@ -967,7 +969,7 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
     float score = -INFINITY;
     bool cand = false;
     if ((lane & 7) == 0 && vm < n) {
-      score = total * sc;
+      score = (total + bq) * sc;
       const bool allowed = !FILT || ((__ldg(ab + (tn >> 5)) >> (tn & 31)) & 1u);
       cand = allowed && better(score, vm, th_s, th_i) && !tombstoned(del, vm);
     }
@@ -1164,6 +1166,7 @@ struct ScanArgs {
   int64_t* out_ids;
   float* out_scores;
   bool pdl;
+  const float* bias;
 };
 
 // Launches `kernel`, with programmatic stream serialization when `pdl` (the
@@ -1219,14 +1222,15 @@ cudaError_t scan_typed(dim3 grid, size_t smem, cudaStream_t s, const ScanArgs& a
     return launch_maybe_pdl(a.pdl, k_scan_ring<BITS, S, FILT, FIX>, grid, dim3(RING_NT), rsmem, s, a.qrot, a.d,
                             a.centroids, a.codes, a.scale, a.n, a.del, a.dense, a.allow, a.words, a.bmask,
                             a.mask_words, a.fblock, a.k, P, ns, a.cs, a.ci, a.err, a.counters, a.ext, a.out_ids,
-                            a.out_scores);
+                            a.out_scores, a.bias);
   }
   const void* fn = reinterpret_cast<const void*>(k_scan_stream<BITS, S, FILT, FIX>);
   const cudaError_t e = set_max_dynamic_smem(fn, (int)smem);
   if (e != cudaSuccess) return e;
   return launch_maybe_pdl(a.pdl, k_scan_stream<BITS, S, FILT, FIX>, grid, dim3(SCAN_NT), smem, s, a.qrot, a.d,
                           a.centroids, a.codes, a.scale, a.n, a.del, a.dense, a.allow, a.words, a.bmask,
-                          a.mask_words, a.fblock, a.k, a.P, a.cs, a.ci, a.counters, a.ext, a.out_ids, a.out_scores);
+                          a.mask_words, a.fblock, a.k, a.P, a.cs, a.ci, a.counters, a.ext, a.out_ids, a.out_scores,
+                          a.bias);
 }
 
 template <int BITS, int S>
@@ -1273,8 +1277,8 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
                             const uint8_t* codes, const float* scale, int64_t n, const uint32_t* del,
                             const FilterDev* f, const uint32_t* allow_bits, const uint32_t* bmask, bool fix,
                             int k, int grid_x, float* cand_s, int32_t* cand_i, int* err, int* counters,
-                            const uint64_t* ext, int64_t* out_ids, float* out_scores, cudaStream_t s,
-                            cudaEvent_t ev0, cudaEvent_t ev1) {
+                            const uint64_t* ext, int64_t* out_ids, float* out_scores, const float* bias,
+                            cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
   const int S = (d + 511) / 512;
   const int P = next_pow2(SCAN_WARPS * k);
@@ -1286,7 +1290,7 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
              f ? f->block : 64, k, P, cand_s, cand_i, err, counters, ext, out_ids, out_scores,
              // overlap with the kernel before (not on the legacy default stream, and not
              // between profiling events, which would serialise the two anyway)
-             s != nullptr && ev0 == nullptr};
+             s != nullptr && ev0 == nullptr, bias};
   const bool filt = f != nullptr;
   cudaError_t e;
   if (ev0 && (e = cudaEventRecord(ev0, s)) != cudaSuccess) return e;

@@ -136,7 +136,7 @@ extern "C" tq_status tq_search_static(const float* Q, int64_t nq, int d, const f
   if (e == cudaSuccess)
     e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, nullptr, f, allow_bits, bmask,
                             tq::search_path() == TQ_PATH_LUT_FIXED && d >= tq::kFixMinD, k, gx, cand_s, cand_i,
-                            status, counters, nullptr, out_ids, out_scores, s, nullptr, nullptr);
+                            status, counters, nullptr, out_ids, out_scores, nullptr, s, nullptr, nullptr);
   if (e != cudaSuccess) return fail(TQ_ECUDA, "tq_search_static: %s", cudaGetErrorString(e));
   return tq::ok();
 }

@@ -10,14 +10,15 @@ allowlists (Sec. III-B), the per-block tenant bitmaps growing with the index.
 
 Everything here is bookkeeping around the C ABI: rows are encoded by
 tq_encode straight into the index's device arrays, the filter grows by
-tq_filter_append, and search is tq_search_ex.  Files use the flat format of
-`flatfile`.
+tq_filter_append, and search is tq_search_ex.  With `tq_plus=True` the first
+batch added fixes a TQ+ calibration (tq_calibrate) that every later encode and
+search uses.  Files use the flat format of `flatfile`.
 """
 from __future__ import annotations
 
 import numpy as np
 
-from . import Filter, IdMap, codebook, encode, rotation, row_bytes, search
+from . import Filter, IdMap, calibrate, codebook, encode, rotation, row_bytes, search
 from . import _used_on, flatfile
 
 FORMAT_VERSION = 1
@@ -39,7 +40,7 @@ class Index:
 
     def __init__(self, d: int, bits: int = 4, capacity: int = 1 << 20, *, seed: int = 1536,
                  marginal: str = "beta", scale_mode: str = "norm", id_map: bool = False,
-                 tenants: bool = False, block: int = 64, device=None, tables=None):
+                 tenants: bool = False, block: int = 64, device=None, tables=None, tq_plus: bool = False):
         torch = _torch()
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
         self.d, self.bits, self.capacity = int(d), int(bits), int(capacity)
@@ -58,6 +59,10 @@ class Index:
         self.id_map = IdMap(self.capacity) if id_map else None
         self.tenant_ids = torch.empty(self.capacity, dtype=torch.int32, device=self.device) if tenants else None
         self.filter: Filter | None = None
+        # TQ+ (Sec. II-B): per-coordinate shift and scale fitted on the first
+        # add() batch, then used for every encode and search
+        self.tq_plus = bool(tq_plus)
+        self.calib = None
 
     def _set_tables(self, R, centroids, boundaries) -> None:
         torch = _torch()
@@ -114,11 +119,14 @@ class Index:
         first = self.n
         rows = slice(first, first + m)
         codes, scale = self.codes[rows], self.scale[rows]
+        if self.tq_plus and self.calib is None:  # the first batch fixes the calibration
+            self.calib = calibrate(X, self.R, stream=stream)
         if codes.data_ptr() % 16 == 0:
             encode(X, self.R, self.centroids, self.boundaries, self.bits, self.scale_mode, codes, scale,
-                   stream=stream)
+                   stream=stream, calib=self.calib)
         else:  # a row offset off the 16-byte grid tq_encode needs: encode aside, then copy
-            c, s = encode(X, self.R, self.centroids, self.boundaries, self.bits, self.scale_mode, stream=stream)
+            c, s = encode(X, self.R, self.centroids, self.boundaries, self.bits, self.scale_mode, stream=stream,
+                          calib=self.calib)
             with torch.cuda.stream(stream) if stream is not None else _null():
                 codes.copy_(c)
                 scale.copy_(s)
@@ -174,7 +182,7 @@ class Index:
                 _used_on(t, stream)
         return search(Q, self.R, self.centroids, self.bits, self.codes[: self.n], self.scale[: self.n], k,
                       filter=self.filter if allow is not None else None, allow_off=off, allow_tenants=ten,
-                      workspace=workspace, stream=stream, idmap=self.id_map)
+                      workspace=workspace, stream=stream, idmap=self.id_map, calib=self.calib)
 
     # ----------------------------------------------------------- persistence
     def save(self, path: str) -> None:
@@ -185,7 +193,8 @@ class Index:
         n = self.n
         fields = {"format": "turboquant-index", "version": FORMAT_VERSION, "d": self.d, "bits": self.bits,
                   "n": n, "seed": self.seed, "marginal": self.marginal, "scale_mode": self.scale_mode,
-                  "block": self.block, "id_map": self.id_map is not None, "tenants": self.tenant_ids is not None}
+                  "block": self.block, "id_map": self.id_map is not None, "tenants": self.tenant_ids is not None,
+                  "tq_plus": self.tq_plus}
         arrays = {"R": self.R.cpu().numpy(), "centroids": self.centroids.cpu().numpy(),
                   "boundaries": self.boundaries.cpu().numpy(), "codes": self.codes[:n].cpu().numpy(),
                   "scale": self.scale[:n].cpu().numpy()}
@@ -193,6 +202,8 @@ class Index:
             arrays["tenant_ids"] = self.tenant_ids[:n].cpu().numpy().view(np.uint32)
         if self.id_map is not None:
             arrays["ext_ids"], arrays["deleted"] = self.id_map.export()
+        if self.calib is not None:
+            arrays["calib_mu"], arrays["calib_a"] = (t.cpu().numpy() for t in self.calib)
         flatfile.write(path, fields, arrays)
 
     @classmethod
@@ -220,6 +231,11 @@ class Index:
         idx.scale = torch.empty(cap, dtype=torch.float32, device=idx.device)
         idx.codes[:n].copy_(torch.from_numpy(a["codes"]))
         idx.scale[:n].copy_(torch.from_numpy(a["scale"]))
+        idx.tq_plus = bool(fields.get("tq_plus", False))
+        idx.calib = None
+        if "calib_mu" in a:
+            idx.calib = tuple(torch.from_numpy(np.ascontiguousarray(a[k], np.float32)).to(idx.device)
+                              for k in ("calib_mu", "calib_a"))
         idx.id_map = None
         if fields["id_map"]:
             idx.id_map = IdMap(cap)

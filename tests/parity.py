@@ -18,8 +18,10 @@ TOL_LUT = 1e-5
 TOL_MMA = 2e-3
 
 
-def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bits, mode):
-    """Returns the number of boundary-window code flips (all of them checked)."""
+def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bits, mode, calib=None):
+    """Returns the number of boundary-window code flips (all of them checked).
+    With a TQ+ calibration (the oracle's, as given to both sides) enc.y holds
+    the quantised z and the scalar is checked on the reconstruction a c + mu."""
     gpu_packed = np.asarray(gpu_packed)
     gpu_scale = np.asarray(gpu_scale)
     assert gpu_packed.shape == enc.packed.shape
@@ -39,6 +41,10 @@ def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bi
     # scale: against the oracle on clean rows, against the definition on the rest
     n = np.linalg.norm(np.asarray(X, np.float64), axis=1)
     c = centroids32.astype(np.float64)[U]
+    yy = enc.y
+    if calib is not None:
+        c = calib.a[None, :] * c + calib.mu[None, :]
+        yy = enc.y * calib.a[None, :] + calib.mu[None, :]   # back from z to y
     if mode == "norm":
         cn = np.linalg.norm(c, axis=1)
         want = np.where(n > 0, n / np.where(cn > 0, cn, 1), 0.0)
@@ -47,7 +53,7 @@ def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bi
         want = n
         rtol = 2e-6
     else:
-        yc = np.sum(enc.y * c, axis=1)
+        yc = np.sum(yy * c, axis=1)
         want = np.where(n > 0, n / np.where(yc != 0, yc, 1), 0.0)
         rtol = 2e-5
     assert np.allclose(gpu_scale[clean], enc.scale[clean], rtol=rtol, atol=1e-30)

@@ -122,12 +122,27 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert search(ws=null) == _lib.TQ_EINVAL
     assert search(nq=0) == _lib.TQ_OK
     # search over an id map: misaligned tombstone bitmap / external ids
-    ex = list(args[:12]) + [p + 2, null] + list(args[12:])
+    ex = list(args[:12]) + [p + 2, null, null, null] + list(args[12:])
     assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
     ex[12], ex[13] = null, p + 4
     assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
-    ex[13], ex[14] = null, 0
+    ex[13], ex[16] = null, 0
     assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
+    # a TQ+ calibration needs both arrays, 4-byte aligned
+    ex[16] = 5
+    ex[14] = p
+    assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL and b"both mu and a" in lib.tq_last_error()
+    ex[14], ex[15] = p + 1, p
+    assert lib.tq_search_ex(*ex) == _lib.TQ_EINVAL
+    # TQ+ calibration and calibrated encode: argument checks (no device memory is touched)
+    sz = C.c_size_t()
+    assert lib.tq_calibrate_workspace(0, 64, C.byref(sz)) == _lib.TQ_EINVAL
+    assert lib.tq_calibrate_workspace(10, 48, C.byref(sz)) == _lib.TQ_EINVAL
+    assert lib.tq_calibrate_workspace(300, 64, C.byref(sz)) == _lib.TQ_OK
+    assert sz.value == 3 * 64 * 16 + 3 * 4   # 3 panels of 128 rows: sums, squares (double), counts
+    assert lib.tq_calibrate(p, 300, 64, p, p, p, p, sz.value - 1, null) == _lib.TQ_EINVAL
+    assert lib.tq_calibrate(null, 300, 64, p, p, p, p, sz.value, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode_ex(p, 10, 64, p, p, p, 4, 0, p, null, p, p, null) == _lib.TQ_EINVAL
     # id map: capacity, NULL handle / ids (no device memory is touched)
     m = C.c_void_p()
     assert lib.tq_idmap_create(0, C.byref(m)) == _lib.TQ_EINVAL
