@@ -321,6 +321,8 @@ def run_ours(args, cfg, rank, world):
     batches = [int(b) for b in args.batches.split(",")] if args.batches else cfg["batches"]
     if args.k:
         k = args.k
+    if args.bits:
+        bits = args.bits
     stream = torch.cuda.Stream(device=dev)
 
     def barrier():
@@ -1084,6 +1086,8 @@ def main():
     ap.add_argument("--config", choices=sorted(CONFIGS), default="scale")
     ap.add_argument("--batches", default=None, help="comma-separated batch sizes (first = headline)")
     ap.add_argument("--k", type=int, default=None)
+    ap.add_argument("--bits", type=int, default=None, choices=[2, 3, 4, 8],
+                    help="code width for the scale/c2/tiny/prof workloads (default: 4)")
     ap.add_argument("--ref-sample", type=int, default=100_000, help="corpus rows the oracle scans")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",

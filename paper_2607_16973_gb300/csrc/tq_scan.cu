@@ -240,58 +240,25 @@ __device__ __forceinline__ void load_q2(float2 (&q2)[S][8], const float* qq, int
 // shared scratch of (blockDim.x / 32) * k entries; out_* point at the query's
 // k results.
 //
-// A second bound: the k best of the lists' first entries are k distinct
-// candidates, so the k-th best overall is at least as good as the k-th of
-// them too.  When there are many lists of few vectors each (a small corpus
-// spread over every SM) their k-th entries are weak and this bound is far
-// tighter; it is taken by sorting the first entries.  `scratch` (shared,
-// scratch_bytes) holds that sort and, when they fit, a copy of all the
-// candidates, fetched in one pass so that later steps wait on no more loads.
+// The candidates at least as good as that bound are few (about k to a few
+// times k): they are gathered into `scratch` (shared, scratch_bytes) and
+// sorted by the whole block, the result being the first k.  Only when they
+// do not fit does each warp insert its share into a sorted list of k.
 __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, int k, const uint64_t* __restrict__ ext,
                                   int64_t* out_ids, float* out_scores, float* ws, int* wi, unsigned char* scratch,
                                   size_t scratch_bytes) {
-  __shared__ float red_s[33];
-  __shared__ int red_i[33];
+  __shared__ float red_s[32];
+  __shared__ int red_i[32];
+  __shared__ int nsurv;
   const int nwarps = blockDim.x >> 5;
   const int total = nlists * k;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  int P2 = 1;
-  while (P2 < nlists) P2 <<= 1;
-  const bool use_u = nlists > k && (size_t)P2 * 8 <= scratch_bytes;
-  float* sort_s = reinterpret_cast<float*>(scratch);
-  int* sort_i = reinterpret_cast<int*>(sort_s + P2);
-  const size_t stage_off = use_u ? (size_t)P2 * 8 : 0;
-  const bool staged = stage_off + (size_t)total * 8 <= scratch_bytes;
-  float* st_s = reinterpret_cast<float*>(scratch + stage_off);
-  int* st_i = reinterpret_cast<int*>(st_s + total);
-  if (staged) {
-    for (int c = tid; c < total; c += blockDim.x) {
-      st_s[c] = __ldcg(cs + c);
-      st_i[c] = __ldcg(ci + c);
-    }
-    __syncthreads();
-  }
-  auto rs = [&](int c) { return staged ? st_s[c] : __ldcg(cs + c); };
-  auto ri = [&](int c) { return staged ? st_i[c] : __ldcg(ci + c); };
-  // 0. U = k-th best first entry
-  if (use_u) {
-    for (int l = tid; l < P2; l += blockDim.x) {
-      sort_s[l] = l < nlists ? rs(l * k) : -INFINITY;
-      sort_i[l] = l < nlists ? ri(l * k) : INT_MAX;
-    }
-    __syncthreads();
-    block_sort(sort_s, sort_i, P2);
-    if (tid == 0) {
-      red_s[32] = sort_s[k - 1];
-      red_i[32] = sort_i[k - 1];
-    }
-  }
   // 1. T = best k-th entry over the lists
   float ts = -INFINITY;
   int ti = INT_MAX;
   for (int l = tid; l < nlists; l += blockDim.x) {
-    const float a = rs(l * k + k - 1);
-    const int b = ri(l * k + k - 1);
+    const float a = __ldcg(cs + l * k + k - 1);
+    const int b = __ldcg(ci + l * k + k - 1);
     if (better(a, b, ts, ti)) {
       ts = a;
       ti = b;
@@ -310,10 +277,7 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
     red_s[warp] = ts;
     red_i[warp] = ti;
   }
-  for (int i = lane; i < k; i += 32) {
-    ws[warp * k + i] = -INFINITY;
-    wi[warp * k + i] = INT_MAX;
-  }
+  if (tid == 0) nsurv = 0;
   __syncthreads();
   ts = red_s[0];
   ti = red_i[0];
@@ -322,10 +286,56 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
       ts = red_s[w];
       ti = red_i[w];
     }
-  if (use_u && better(red_s[32], red_i[32], ts, ti)) {
-    ts = red_s[32];
-    ti = red_i[32];
+  // 2. gather the candidates at least as good as T (eight loads per thread in flight)
+  const int cap = (int)min((size_t)8192, scratch_bytes / 8);
+  float* ss = reinterpret_cast<float*>(scratch);
+  int* si = reinterpret_cast<int*>(ss + cap);
+  for (int c0 = tid; c0 < total; c0 += 8 * blockDim.x) {
+    float va[8];
+    int vb[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int c = c0 + u * blockDim.x;
+      va[u] = c < total ? __ldcg(cs + c) : -INFINITY;
+      vb[u] = c < total ? __ldcg(ci + c) : INT_MAX;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (vb[u] != INT_MAX && !better(ts, ti, va[u], vb[u])) {
+        const int p = atomicAdd(&nsurv, 1);
+        if (p < cap) {
+          ss[p] = va[u];
+          si[p] = vb[u];
+        }
+      }
+    }
   }
+  __syncthreads();
+  const int nsv = nsurv;
+  int P = 1;
+  while (P < nsv || P < k) P <<= 1;
+  if (P <= cap) {  // 3. sort them (the order is total: the result does not depend on the gathering order)
+    for (int i = nsv + tid; i < P; i += blockDim.x) {
+      ss[i] = -INFINITY;
+      si[i] = INT_MAX;
+    }
+    __syncthreads();
+    block_sort(ss, si, P);
+    for (int i = tid; i < k; i += blockDim.x) {
+      const bool empty = si[i] == INT_MAX;
+      out_ids[i] = empty ? -1 : ext ? (int64_t)__ldg(ext + si[i]) : (int64_t)si[i];
+      out_scores[i] = empty ? -INFINITY : ss[i];
+    }
+    return;
+  }
+  // too many to sort in the scratch: each warp inserts its share into a list of k
+  auto rs = [&](int c) { return __ldcg(cs + c); };
+  auto ri = [&](int c) { return __ldcg(ci + c); };
+  for (int i = lane; i < k; i += 32) {
+    ws[warp * k + i] = -INFINITY;
+    wi[warp * k + i] = INT_MAX;
+  }
+  __syncthreads();
   // 2. per-warp sorted top-k of the candidates at least as good as T
   float* ls = ws + warp * k;
   int* li = wi + warp * k;
@@ -391,12 +401,14 @@ __device__ __forceinline__ void merge_if_last(const float* cand_s, const int* ca
                                               int* li, unsigned char* scratch, size_t scratch_bytes) {
   __shared__ int last;
   const int q = blockIdx.y;
-  __threadfence();  // this thread's part of the list, before the arrival
-  __syncthreads();
-  if (threadIdx.x == 0) last = atomicAdd(counters + q, 1) == (int)gridDim.x - 1;
+  __syncthreads();  // the CTA's list is written ...
+  if (threadIdx.x == 0) {
+    __threadfence();  // ... and, through the barrier, released at GPU scope before the arrival
+    last = atomicAdd(counters + q, 1) == (int)gridDim.x - 1;
+    if (last) __threadfence();  // acquire every other CTA's list
+  }
   __syncthreads();
   if (!last) return;
-  __threadfence();  // every other CTA's list, after seeing all arrivals
   const size_t base = (size_t)q * gridDim.x * k;
   merge_lists_block(cand_s + base, cand_i + base, gridDim.x, k, ext, out_ids + (size_t)q * k,
                     out_scores + (size_t)q * k, ls, li, scratch, scratch_bytes);
@@ -424,27 +436,26 @@ __device__ __forceinline__ float warp_sum4(float (&p)[4]) {
 // Fixed-point byte-pair table for 4-bit codes.  The exact table above moves
 // 8 bytes through shared memory per packed byte (two fp32 centroids), which
 // bounds the scan by the shared-memory datapath (128 B per cycle per SM).
-// Here each centroid is a 15-bit fixed-point value u_v = rint(c_v / step) +
-// 16384, and the entry (x, lane) = u[x & 15] | u[x >> 4] << 16 is 4 bytes: one
-// wavefront per warp lookup instead of two.  A byte permute turns a 16-bit
-// half into a float without any arithmetic: bytes (0, u_lo, u_hi, 0x3F) are
-// the float 0.5 + u * 2^-16 (u < 2^15 keeps bit 23, the exponent's low bit,
-// clear), exact.  With the query pre-scaled, q''_j = q'_j * step * 2^16,
-//   q''_j * (0.5 + u_j 2^-16 - 0.75) = q'_j * (u_j - 16384) * step = q'_j * c^_j,
-// so each lane starts its two accumulators at -0.75 * (its sum of q'') and
-// then needs one fused multiply-add per centroid: per packed byte a byte
-// permute for the address, one 4-byte load, two byte permutes and one paired
-// FMA.  c^_v differs from c_v by the rounding to the step; the step is the
+// Here each centroid is a signed 15-bit integer c_v = rint(centroid_v / step)
+// and the entry (x, lane) = c[x & 15] | c[x >> 4] << 16 is 4 bytes: one
+// wavefront per warp lookup instead of two.  The entry feeds 2-way integer
+// dot products (dp2a: two 16-bit halves times two bytes, added to a 32-bit
+// accumulator) without any conversion: each lane quantises its 48 rotated
+// query coordinates to 24-bit integers q_j = rint(q'_j / s) (s = the lane's
+// largest |q'_j| / (2^23 - 1)), split into bytes q_j = 2^16 h_j + 2^8 m_j + l_j
+// (h signed), and per packed byte makes three dp2a's, one per byte plane of
+// the coordinate pair.  Per lane and vector, 2^16 A_h + 2^8 A_m + A_l is the
+// exact integer sum_j q_j c_j, and s * step times it the lane's part of the
+// score.  The rounding of the centroids to the step is the only error beyond
+// float32 (about 2^-16 of the largest centroid per centroid): the step is the
 // one, among FIX_CANDIDATES values in [d0, 1.25 d0) (d0 = max|c| / 16383),
 // whose largest rounding error over the 16 centroids is least, chosen the
 // same way by every CTA.
 constexpr int FIX_CANDIDATES = 2048;
-constexpr uint32_t FIX_HALF = 0x3F000000u;  // byte 3 of 0.5f, byte 0 zero
 
 // Fills the fixed-point table (uint32 entry (x, lane) at index x * 64 + lane;
-// the other half of each 256-byte row is unused) and returns the step * 2^16
-// the rotated query is multiplied by.  All threads of the CTA call it; `red`
-// is shared scratch of 2 * 32 words.
+// the other half of each 256-byte row is unused) and returns the step.  All
+// threads of the CTA call it; `red` is shared scratch of 2 * 32 words.
 __device__ float fix_table_init(uint32_t* tab, const float* __restrict__ centroids, float* red, int tid, int nt) {
   float c[16];
   float m = 0.f;
@@ -498,22 +509,64 @@ __device__ float fix_table_init(uint32_t* tab, const float* __restrict__ centroi
   }
   const float step = d0 * (1.0f + (float)best_i * (0.25f / FIX_CANDIDATES));
   __shared__ uint32_t su[16];
-  if (tid < 16) su[tid] = (uint32_t)min(32767, max(0, (int)rintf(c[tid] / step) + 16384));
+  if (tid < 16) su[tid] = (uint32_t)min(16383, max(-16383, (int)rintf(c[tid] / step))) & 0xFFFFu;
   __syncthreads();
   for (int i = tid; i < 256 * 32; i += nt) {
     const int x = i >> 5;
     tab[x * 64 + (i & 31)] = su[x & 15] | (su[x >> 4] << 16);
   }
-  return step * 65536.0f;
+  return step;
 }
 
-// This lane's part of one vector's score with the fixed-point table; `init`
-// holds -0.75 times the lane's sums of the scaled query (even, odd
-// coordinates).
+// Quantises this lane's query pairs (q'_{2m}, q'_{2m+1}) to 24-bit integers
+// and replaces each pair, in place, by its byte planes: .x = (l_e, l_o, m_e,
+// m_o) and .y = (h_e, h_o, 0, 0) as bit patterns.  Returns s * step, the
+// factor of the lane's integer sums.
+template <int S>
+__device__ __forceinline__ float fix_query_bytes(float2 (&q2)[S][8], float step) {
+  float mx = 0.f;
+#pragma unroll
+  for (int s = 0; s < S; ++s)
+#pragma unroll
+    for (int m = 0; m < 8; ++m) mx = fmaxf(mx, fmaxf(fabsf(q2[s][m].x), fabsf(q2[s][m].y)));
+  const float sq = mx > 0.f ? mx / 8388607.0f : 1.0f;
+  const float inv = 1.0f / sq;
+#pragma unroll
+  for (int s = 0; s < S; ++s)
+#pragma unroll
+    for (int m = 0; m < 8; ++m) {
+      const int e = min(8388607, max(-8388607, __float2int_rn(q2[s][m].x * inv)));
+      const int o = min(8388607, max(-8388607, __float2int_rn(q2[s][m].y * inv)));
+      const uint32_t lo = (uint32_t)(e & 0xFF) | ((uint32_t)(o & 0xFF) << 8) | ((uint32_t)((e >> 8) & 0xFF) << 16) |
+                          ((uint32_t)((o >> 8) & 0xFF) << 24);
+      const uint32_t hi = (uint32_t)((e >> 16) & 0xFF) | ((uint32_t)((o >> 16) & 0xFF) << 8);
+      q2[s][m] = make_float2(__uint_as_float(lo), __uint_as_float(hi));
+    }
+  return sq * step;
+}
+
+__device__ __forceinline__ int dp2a_lo_su(uint32_t a, uint32_t b, int c) {  // a: two s16, b: bytes 0-1 unsigned
+  int d;
+  asm("dp2a.lo.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+__device__ __forceinline__ int dp2a_hi_su(uint32_t a, uint32_t b, int c) {  // bytes 2-3 unsigned
+  int d;
+  asm("dp2a.hi.s32.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+__device__ __forceinline__ int dp2a_lo_ss(uint32_t a, uint32_t b, int c) {  // bytes 0-1 signed
+  int d;
+  asm("dp2a.lo.s32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
+// This lane's part of one vector's score with the fixed-point table: the
+// exact integer sum, scaled by `f` (fix_query_bytes).
 template <int S>
 __device__ __forceinline__ float pair16_dot(const Chunk<4> (&ch)[S], const float2 (&q2)[S][8], const char* tab,
-                                            uint32_t lane4, float2 init) {
-  float2 acc = init;
+                                            uint32_t lane4, float f) {
+  int al = 0, am = 0, ah = 0;
 #pragma unroll
   for (int s = 0; s < S; ++s) {
 #pragma unroll
@@ -521,12 +574,14 @@ __device__ __forceinline__ float pair16_dot(const Chunk<4> (&ch)[S], const float
       const uint32_t w = b < 4 ? ch[s].w0 : ch[s].w1;
       const uint32_t addr = __byte_perm(w, lane4, 0x5504u | ((uint32_t)(b & 3) << 4));
       const uint32_t e = *reinterpret_cast<const uint32_t*>(tab + addr);
-      const float2 x = make_float2(__uint_as_float(__byte_perm(e, FIX_HALF, 0x7104u)),
-                                   __uint_as_float(__byte_perm(e, FIX_HALF, 0x7324u)));
-      acc = __ffma2_rn(q2[s][b], x, acc);
+      const uint32_t p0 = __float_as_uint(q2[s][b].x), p1 = __float_as_uint(q2[s][b].y);
+      al = dp2a_lo_su(e, p0, al);
+      am = dp2a_hi_su(e, p0, am);
+      ah = dp2a_lo_ss(e, p1, ah);
     }
   }
-  return acc.x + acc.y;
+  const long long t = ((long long)ah << 16) + ((long long)am << 8) + (long long)al;
+  return (float)t * f;
 }
 
 // The lookup scan.  Each warp scores 4 consecutive vectors per step (a CTA
@@ -560,7 +615,7 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
   __shared__ float red[64];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int q = blockIdx.y;
-  float qs = 1.0f;  // query pre-scale of the fixed-point table
+  float qs = 1.0f;  // the fixed-point table's step
   if constexpr (PAIR && FIX) {
     qs = fix_table_init(reinterpret_cast<uint32_t*>(smem_raw), centroids, red, tid, SCAN_NT);
   } else if constexpr (PAIR) {
@@ -579,22 +634,10 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
   const float* qq = qrot + (size_t)q * d;
   float qr[PAIR ? 1 : S][16];
   float2 q2[PAIR ? S : 1][8];
-  float2 init = make_float2(0.f, 0.f);
+  float qf = 0.f;  // fixed-point table: the factor of the lanes' integer sums
   if constexpr (PAIR) {
     load_q2(q2, qq, nchunks, lane);
-    if constexpr (FIX) {
-      float se = 0.f, so = 0.f;
-#pragma unroll
-      for (int s = 0; s < S; ++s)
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          q2[s][m].x *= qs;
-          q2[s][m].y *= qs;
-          se += q2[s][m].x;
-          so += q2[s][m].y;
-        }
-      init = make_float2(-0.75f * se, -0.75f * so);
-    }
+    if constexpr (FIX) qf = fix_query_bytes<S>(q2, qs);
   } else {
 #pragma unroll
     for (int s = 0; s < S; ++s) {
@@ -664,7 +707,7 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
 #pragma unroll
     for (int i = 0; i < V; ++i) {
       if constexpr (PAIR && FIX) {
-        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, init);
+        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, qf);
       } else if constexpr (PAIR) {
         p[i] = pair_dot<S>(cur[i], q2, tab, lane4 * 2u);
       } else {
@@ -849,7 +892,7 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
     issue(next_ws, s);
     next_ws = active(next_ws + wstride);
   }
-  float qs = 1.0f;
+  float qs = 1.0f;  // the fixed-point table's step
   if constexpr (PAIR && FIX) {
     qs = fix_table_init(reinterpret_cast<uint32_t*>(smem_raw), centroids, red, tid, RING_NT);
   } else if constexpr (PAIR) {
@@ -868,22 +911,10 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
   const float* qq = qrot + (size_t)q * d;
   float qr[PAIR ? 1 : S][16];
   float2 q2[PAIR ? S : 1][8];
-  float2 init = make_float2(0.f, 0.f);
+  float qf = 0.f;  // fixed-point table: the factor of the lanes' integer sums
   if constexpr (PAIR) {
     load_q2(q2, qq, nchunks, lane);
-    if constexpr (FIX) {
-      float se = 0.f, so = 0.f;
-#pragma unroll
-      for (int s = 0; s < S; ++s)
-#pragma unroll
-        for (int m = 0; m < 8; ++m) {
-          q2[s][m].x *= qs;
-          q2[s][m].y *= qs;
-          se += q2[s][m].x;
-          so += q2[s][m].y;
-        }
-      init = make_float2(-0.75f * se, -0.75f * so);
-    }
+    if constexpr (FIX) qf = fix_query_bytes<S>(q2, qs);
   } else {
 #pragma unroll
     for (int s = 0; s < S; ++s) {
@@ -952,7 +983,7 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
 #pragma unroll
     for (int i = 0; i < V; ++i) {
       if constexpr (PAIR && FIX) {
-        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, init);
+        p[i] = pair16_dot<S>(cur[i], q2, tab, lane4, qf);
       } else if constexpr (PAIR) {
         p[i] = pair_dot<S>(cur[i], q2, tab, lane4 * 2u);
       } else {
@@ -1314,9 +1345,10 @@ cudaError_t launch_merge(const float* cand_s, const int32_t* cand_i, int64_t nq,
   const int nlists = per_query / k;
   int warps = std::max(1, std::min(32, (nlists + 31) / 32));
   while (warps > 1 && (size_t)warps * k * 8 > 24 * 1024) warps >>= 1;
-  // scratch for the first-entry sort and, when it fits, the staged candidates
-  const size_t want = ((size_t)next_pow2(nlists) + (size_t)nlists * k) * 8;
-  const size_t scratch = std::min<size_t>(want, 48 * 1024 - (size_t)warps * k * 8);
+  // scratch for gathering and sorting the candidates that pass the bound
+  const size_t want = (size_t)next_pow2(std::max(nlists * k, 2)) * 8;
+  // (dynamic plus the kernel's few static bytes stay under the default 48 KB)
+  const size_t scratch = std::min<size_t>(want, 40 * 1024 - (size_t)warps * k * 8);
   const size_t smem = (size_t)warps * k * (sizeof(float) + sizeof(int32_t)) + scratch;
   k_merge_lists<<<(unsigned)nq, 32 * warps, smem, s>>>(cand_s, cand_i, nlists, k, ext, out_ids, out_scores,
                                                        scratch);
