@@ -285,17 +285,20 @@ def run_reference(args, cfg, rank, world):
         O.search(Q[j:j + 1], R, cb.centroids32, bits, enc.packed, enc.scale, k, d)
     el = time.perf_counter() - t0
     scale_up = cfg["n"] / sample_rows
-    per_step_full = el / max(args.steps, 1) * scale_up
+    per_step = el / max(args.steps, 1)          # measured: one query over the sample rows
+    per_step_full = per_step * scale_up
     qps = B / per_step_full
     cores = cpu_threads()
     line = {
         "impl": "reference", "metric": METRIC, "value": qps, "unit": "queries/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_full * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * 1e3,
+        "extrapolated_from": {"rows_per_step": sample_rows, "corpus_rows": cfg["n"], "factor": scale_up,
+                              "ms_per_full_query": per_step_full * 1e3},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
         "config": {"workload": f"{args.config}: N={cfg['n']} d={d} {bits}-bit top-{k}, batch 1",
                    "n": cfg["n"], "d": d, "bits": bits, "k": k, "batch": 1},
-        "cpu_baseline": {"value": qps, "unit": "queries/s", "cores": cores, "kind": "oracle",
+        "cpu_baseline": {"value": qps, "unit": "queries/s", "cores": cores, "kind": "oracle", **cpu_model(),
                          "sample": f"each step: oracle search of 1 query over the first {sample_rows} "
                                    f"rows, time scaled by {cfg['n']}/{sample_rows}"},
         "e2e": {"value": qps, "unit": "queries/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
