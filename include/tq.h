@@ -164,6 +164,38 @@ tq_status tq_encode_ex(const float* X, int64_t n, int d, const float* R,
                        uint8_t* codes, float* scale, void* stream);
 
 /*
+ * Tensor-core encode: tq_encode_ex with the rotation (Sec. II-B step 2) on the
+ * tensor cores in TF32.  TF32 keeps 10 mantissa bits, so each operand is split
+ * into two TF32 parts, v = v_hi + v_lo (v_hi = tf32(v), v_lo = tf32(v - v_hi)),
+ * and y = x_hi.R_hi + x_hi.R_lo + x_lo.R_hi is accumulated in float32: a
+ * relative error of a few 2^-22 per product, so, as with tq_encode, a
+ * coordinate within ~1e-6 of a boundary may land in either neighbouring cell.
+ *
+ * tq_encode_plan_bytes  device bytes of a plan for dimension d; TQ_EUNSUPPORTED
+ *                unless d is a multiple of 32 in [128, 8192]
+ * tq_encode_plan R device [d*d] float32 (tq_rotation's layout); plan: caller-
+ *                owned device memory, 16-byte aligned, of plan_bytes >=
+ *                tq_encode_plan_bytes(d).  Writes a status word and R split
+ *                into R_hi and R_lo.  The plan depends on R only: build it
+ *                once per index, keep it while encoding.
+ * tq_encode_planned  the arguments of tq_encode_ex with the plan in place of
+ *                R (d must be the plan's); same results and argument rules.
+ *                Its waits are bounded: one that gives up (which does not
+ *                happen in normal operation) is recorded in the plan's status
+ *                word, and that call's codes are invalid.
+ * tq_encode_check  waits for `stream`, then returns TQ_ETIMEOUT if an encode
+ *                with this plan gave up since the plan was built or last
+ *                checked (clearing the record), else TQ_OK.
+ */
+tq_status tq_encode_plan_bytes(int d, size_t* bytes);
+tq_status tq_encode_plan(const float* R, int d, void* plan, size_t plan_bytes, void* stream);
+tq_status tq_encode_planned(const float* X, int64_t n, int d, const void* plan,
+                            const float* centroids, const float* boundaries, int bits,
+                            int scale_mode, const float* cal_mu, const float* cal_a,
+                            uint8_t* codes, float* scale, void* stream);
+tq_status tq_encode_check(const void* plan, void* stream);
+
+/*
  * tq_filter_build - per-corpus tenant filter for search(allowlist=...)
  * (Sec. III-B: filtering at vector-block granularity).
  *   tenant_ids  device [n] uint32: the tenant of each vector

@@ -11,9 +11,9 @@ import ctypes as C
 
 import numpy as np
 
-from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQError, check, load)  # noqa: F401
+from ._lib import (MARGINALS, PATHS, SCALE_MODES, TQ_EUNSUPPORTED, TQError, check, load)  # noqa: F401
 
-__all__ = ["codebook", "rotation", "encode", "calibrate", "Filter", "IdMap", "Index", "search", "search_workspace",
+__all__ = ["codebook", "rotation", "encode", "encode_plan", "encode_plan_bytes", "encode_check", "calibrate", "Filter", "IdMap", "Index", "search", "search_workspace",
            "search_from_host", "search_host_staging", "search_check", "merge_topk", "set_search_path",
            "profile_events", "row_bytes", "load", "TQError"]
 
@@ -96,10 +96,11 @@ def rotation(d: int, seed: int) -> np.ndarray:
 
 
 def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
-           codes=None, scale=None, stream=None, calib=None):
+           codes=None, scale=None, stream=None, calib=None, plan=None):
     """tq_encode (tq_encode_ex with a TQ+ calibration `calib` = (mu, a), CUDA
     float32 tensors [d]) on CUDA tensors: returns (codes uint8 [n, d*bits/8],
-    scale f32 [n])."""
+    scale f32 [n]).  With `plan` (encode_plan(R)) the rotation runs on the
+    tensor cores (tq_encode_planned) and R is not read."""
     torch = _torch()
     n, d = X.shape
     with _on_stream(stream):
@@ -109,12 +110,47 @@ def encode(X, R, centroids, boundaries, bits: int, scale_mode: str = "norm",
             scale = torch.empty(n, dtype=torch.float32, device=X.device)
     f32 = torch.float32
     mu, a = calib if calib is not None else (None, None)
-    check(load().tq_encode_ex(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32),
-                              _dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32),
-                              bits, SCALE_MODES[scale_mode], _dev_ptr(mu, "mu", f32) or None,
-                              _dev_ptr(a, "a", f32) or None, _dev_ptr(codes, "codes", torch.uint8),
-                              _dev_ptr(scale, "scale", f32), _stream_handle(stream)))
+    tail = (_dev_ptr(centroids, "centroids", f32), _dev_ptr(boundaries, "boundaries", f32), bits,
+            SCALE_MODES[scale_mode], _dev_ptr(mu, "mu", f32) or None, _dev_ptr(a, "a", f32) or None,
+            _dev_ptr(codes, "codes", torch.uint8), _dev_ptr(scale, "scale", f32), _stream_handle(stream))
+    if plan is not None:
+        check(load().tq_encode_planned(_dev_ptr(X, "X", f32), n, d, _dev_ptr(plan, "plan", torch.uint8), *tail))
+    else:
+        check(load().tq_encode_ex(_dev_ptr(X, "X", f32), n, d, _dev_ptr(R, "R", f32), *tail))
     return codes, scale
+
+
+def encode_plan_bytes(d: int):
+    """tq_encode_plan_bytes: device bytes of a tensor-core encode plan for
+    dimension d, or None where the tensor-core encoder does not apply."""
+    need = C.c_size_t()
+    st = load().tq_encode_plan_bytes(d, C.byref(need))
+    if st == TQ_EUNSUPPORTED:
+        return None
+    check(st)
+    return need.value
+
+
+def encode_plan(R, stream=None):
+    """tq_encode_plan: R (CUDA float32 [d, d]) split into TF32 parts for the
+    tensor-core encoder; returns the plan (CUDA uint8 tensor)."""
+    torch = _torch()
+    d = R.shape[0]
+    need = encode_plan_bytes(d)
+    if need is None:
+        raise TQError(TQ_EUNSUPPORTED, f"no tensor-core encode for d={d}")
+    with _on_stream(stream):
+        plan = torch.empty(need, dtype=torch.uint8, device=R.device)
+    check(load().tq_encode_plan(_dev_ptr(R, "R", torch.float32), d, _dev_ptr(plan, "plan", torch.uint8), need,
+                                _stream_handle(stream)))
+    return plan
+
+
+def encode_check(plan, stream=None) -> None:
+    """tq_encode_check: raises TQError(TQ_ETIMEOUT) if an encode with `plan`
+    gave up on a bounded wait since the last check."""
+    torch = _torch()
+    check(load().tq_encode_check(_dev_ptr(plan, "plan", torch.uint8), _stream_handle(stream)))
 
 
 def calibrate(X, R, stream=None):

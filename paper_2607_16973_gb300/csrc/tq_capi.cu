@@ -104,6 +104,70 @@ extern "C" tq_status tq_encode(const float* X, int64_t n, int d, const float* R,
   return tq_encode_ex(X, n, d, R, centroids, boundaries, bits, scale_mode, nullptr, nullptr, codes, scale, stream);
 }
 
+extern "C" tq_status tq_encode_plan_bytes(int d, size_t* bytes) {
+  if (!bytes) return fail(TQ_EINVAL, "tq_encode_plan_bytes: NULL bytes");
+  if (!tq::encode_tc_supported(d))
+    return fail(TQ_EUNSUPPORTED, "tq_encode_plan_bytes: d=%d is not a multiple of 32 in [128, %d]", d, tq::kMaxD);
+  *bytes = tq::encode_plan_bytes(d);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_encode_plan(const float* R, int d, void* plan, size_t plan_bytes, void* stream) {
+  if (!tq::encode_tc_supported(d))
+    return fail(TQ_EUNSUPPORTED, "tq_encode_plan: d=%d is not a multiple of 32 in [128, %d]", d, tq::kMaxD);
+  if (!R || !plan) return fail(TQ_EINVAL, "tq_encode_plan: NULL device pointer");
+  if (!tq::aligned16(R) || !tq::aligned16(plan)) return fail(TQ_EINVAL, "tq_encode_plan: R and plan must be 16-byte aligned");
+  if (plan_bytes < tq::encode_plan_bytes(d))
+    return fail(TQ_EINVAL, "tq_encode_plan: plan_bytes %zu < %zu", plan_bytes, tq::encode_plan_bytes(d));
+  const cudaError_t e = tq::launch_encode_plan(R, d, plan, (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_encode_plan", e);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_encode_planned(const float* X, int64_t n, int d, const void* plan,
+                                       const float* centroids, const float* boundaries, int bits,
+                                       int scale_mode, const float* cal_mu, const float* cal_a, uint8_t* codes,
+                                       float* scale, void* stream) {
+  tq_status st = tq::check_common("tq_encode_planned", d, bits);
+  if (st != TQ_OK) return st;
+  if (!tq::encode_tc_supported(d))
+    return fail(TQ_EUNSUPPORTED, "tq_encode_planned: d=%d is not a multiple of 32 in [128, %d]", d, tq::kMaxD);
+  if (n < 0 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_encode_planned: n=%lld outside [0, 2^31-1]", (long long)n);
+  if (scale_mode != TQ_SCALE_NORM && scale_mode != TQ_SCALE_NONE && scale_mode != TQ_SCALE_UNBIASED)
+    return fail(TQ_EINVAL, "tq_encode_planned: unknown scale_mode %d", scale_mode);
+  if (n == 0) return tq::ok();
+  if (!X || !plan || !centroids || !boundaries || !codes || !scale)
+    return fail(TQ_EINVAL, "tq_encode_planned: NULL device pointer");
+  if (!tq::aligned16(X) || !tq::aligned16(plan) || !tq::aligned16(codes))
+    return fail(TQ_EINVAL, "tq_encode_planned: X, plan and codes must be 16-byte aligned");
+  if (((uintptr_t)scale & 3u) || ((uintptr_t)centroids & 3u) || ((uintptr_t)boundaries & 3u))
+    return fail(TQ_EINVAL, "tq_encode_planned: scale, centroids and boundaries must be 4-byte aligned");
+  if ((cal_mu == nullptr) != (cal_a == nullptr))
+    return fail(TQ_EINVAL, "tq_encode_planned: a TQ+ calibration needs both mu and a");
+  if (((uintptr_t)cal_mu & 3u) || ((uintptr_t)cal_a & 3u))
+    return fail(TQ_EINVAL, "tq_encode_planned: mu and a must be 4-byte aligned");
+  const cudaError_t e = tq::launch_encode_tc(X, n, d, plan, centroids, boundaries, bits, scale_mode, cal_mu, cal_a,
+                                             codes, scale, (cudaStream_t)stream);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_encode_planned", e);
+  return tq::ok();
+}
+
+extern "C" tq_status tq_encode_check(const void* plan, void* stream) {
+  if (!plan) return fail(TQ_EINVAL, "tq_encode_check: NULL plan");
+  if (!tq::aligned16(plan)) return fail(TQ_EINVAL, "tq_encode_check: plan must be 16-byte aligned");
+  cudaStream_t s = (cudaStream_t)stream;
+  int word = 0;
+  cudaError_t e = cudaMemcpyAsync(&word, plan, sizeof(int), cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess && word != 0) e = cudaMemsetAsync(const_cast<void*>(plan), 0, sizeof(int), s);
+  if (e == cudaSuccess && word != 0) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return tq::cuda_fail("tq_encode_check", e);
+  if (word == 0) return tq::ok();
+  if (word / 1000 == TQ_ETIMEOUT)
+    return fail(TQ_ETIMEOUT, "tq_encode_check: a bounded wait (site %d) gave up; those codes are invalid", word % 1000);
+  return fail(TQ_ECUDA, "tq_encode_check: unexpected status word %d", word);
+}
+
 extern "C" tq_status tq_calibrate_workspace(int64_t n, int d, size_t* bytes) {
   if (!bytes) return fail(TQ_EINVAL, "tq_calibrate_workspace: NULL bytes");
   if (n < 1 || n > INT32_MAX) return fail(TQ_EINVAL, "tq_calibrate_workspace: n=%lld outside [1, 2^31-1]", (long long)n);

@@ -25,6 +25,17 @@ cudaError_t launch_encode(const float* X, int64_t n, int d, const float* R, cons
                           const float* boundaries, int bits, int scale_mode, const float* cal_mu,
                           const float* cal_a, uint8_t* codes, float* scale, cudaStream_t s);
 
+// Tensor-core encode (the same result, the rotation in TF32 with a
+// three-product split on tcgen05): d a multiple of 32 in [128, kMaxD].  The
+// plan (encode_plan_bytes(d) bytes, 16-byte aligned) holds a status word and
+// R split into TF32 parts; launch_encode_tc records a timed-out wait in it.
+bool encode_tc_supported(int d);
+size_t encode_plan_bytes(int d);
+cudaError_t launch_encode_plan(const float* R, int d, void* plan, cudaStream_t s);
+cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan, const float* centroids,
+                             const float* boundaries, int bits, int scale_mode, const float* cal_mu,
+                             const float* cal_a, uint8_t* codes, float* scale, cudaStream_t s);
+
 // TQ+ calibration (Sec. II-B): per-coordinate shift mu and scale a from n
 // rows, into device [d] arrays; ws of calibrate_workspace(n, d) bytes.
 size_t calibrate_workspace(int64_t n, int d);

@@ -236,16 +236,6 @@ __device__ __forceinline__ uint4 decode8_4bit(uint32_t w, const uint32_t (&tl)[4
   return make_uint4(o[0], o[1], o[2], o[3]);
 }
 
-// Lane 0 polls the barrier for the whole warp.
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* err,
-                                          int where) {
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort_flag, err, where) ? 1 : 0;
-  ok = __shfl_sync(0xffffffffu, ok, 0);
-  __syncwarp();
-  return ok != 0;
-}
-
 template <int BITS, int QT>
 __global__ void __launch_bounds__(NTHREADS, 1)
 k_scan_mma(const __grid_constant__ CUtensorMap codes_map, const __half* __restrict__ qpack,

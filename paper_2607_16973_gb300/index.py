@@ -18,7 +18,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import Filter, IdMap, calibrate, codebook, encode, rotation, row_bytes, search
+from . import Filter, IdMap, calibrate, codebook, encode, encode_plan, encode_plan_bytes, rotation, row_bytes, search
 from . import _used_on, flatfile
 
 FORMAT_VERSION = 1
@@ -69,6 +69,9 @@ class Index:
         self.R = torch.from_numpy(np.ascontiguousarray(R, np.float32)).to(self.device)
         self.centroids = torch.from_numpy(np.ascontiguousarray(centroids, np.float32)).to(self.device)
         self.boundaries = torch.from_numpy(np.ascontiguousarray(boundaries, np.float32)).to(self.device)
+        # the tensor-core encoder's split of R, where it applies (else the FFMA encoder runs)
+        with torch.cuda.device(self.device):
+            self.plan = encode_plan(self.R) if encode_plan_bytes(self.d) is not None else None
 
     def __len__(self) -> int:
         return self.n
@@ -123,10 +126,10 @@ class Index:
             self.calib = calibrate(X, self.R, stream=stream)
         if codes.data_ptr() % 16 == 0:
             encode(X, self.R, self.centroids, self.boundaries, self.bits, self.scale_mode, codes, scale,
-                   stream=stream, calib=self.calib)
+                   stream=stream, calib=self.calib, plan=self.plan)
         else:  # a row offset off the 16-byte grid tq_encode needs: encode aside, then copy
             c, s = encode(X, self.R, self.centroids, self.boundaries, self.bits, self.scale_mode, stream=stream,
-                          calib=self.calib)
+                          calib=self.calib, plan=self.plan)
             with torch.cuda.stream(stream) if stream is not None else _null():
                 codes.copy_(c)
                 scale.copy_(s)

@@ -18,10 +18,13 @@ TOL_LUT = 1e-5
 TOL_MMA = 2e-3
 
 
-def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bits, mode, calib=None):
+def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bits, mode, calib=None,
+                 max_rate=1e-4):
     """Returns the number of boundary-window code flips (all of them checked).
     With a TQ+ calibration (the oracle's, as given to both sides) enc.y holds
-    the quantised z and the scalar is checked on the reconstruction a c + mu."""
+    the quantised z and the scalar is checked on the reconstruction a c + mu.
+    `max_rate` bounds the fraction of flipped codes: about 2 E|y error| times
+    the density of boundaries, so it grows with the bit width."""
     gpu_packed = np.asarray(gpu_packed)
     gpu_scale = np.asarray(gpu_scale)
     assert gpu_packed.shape == enc.packed.shape
@@ -35,7 +38,7 @@ def check_encode(gpu_packed, gpu_scale, X, enc, centroids32, boundaries32, d, bi
         y = enc.y[rows, cols]
         assert np.all(np.abs(y - boundaries32[lo].astype(np.float64)) < CODE_WINDOW), \
             "code differs away from a boundary"
-    assert mism.mean() < 1e-4
+    assert mism.mean() < max_rate, f"flip rate {mism.mean():.2e}"
     clean = ~mism.any(axis=1)
     assert np.array_equal(gpu_packed[clean], enc.packed[clean])
     # scale: against the oracle on clean rows, against the definition on the rest

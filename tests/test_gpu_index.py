@@ -70,7 +70,9 @@ def test_filter_append_equals_build(cuda_lib, torch_dev):
 @pytest.mark.parametrize("d,bits,chunks", [(1536, 4, [1000, 1, 2999]), (32, 2, [3, 5, 700])])
 def test_index_ingest_in_pieces(cuda_lib, torch_dev, d, bits, chunks):
     """Rows added in pieces (including offsets off the 16-byte grid at d=32,
-    2 bits) encode exactly as one tq_encode of all rows."""
+    2 bits) encode exactly as one encode of all rows (with the index's
+    tensor-core plan where d allows one: a row's codes do not depend on the
+    batch it came in)."""
     torch, dev = torch_dev
     tq = cuda_lib
     n = sum(chunks)
@@ -80,7 +82,9 @@ def test_index_ingest_in_pieces(cuda_lib, torch_dev, d, bits, chunks):
     for m in chunks:
         assert idx.add(X[r0:r0 + m]) == r0
         r0 += m
-    codes, scale = tq.encode(torch.from_numpy(X).to(dev), idx.R, idx.centroids, idx.boundaries, bits)
+    assert (idx.plan is not None) == (d == 1536)
+    codes, scale = tq.encode(torch.from_numpy(X).to(dev), idx.R, idx.centroids, idx.boundaries, bits,
+                             plan=idx.plan)
     torch.cuda.synchronize()
     assert torch.equal(idx.codes[:n], codes) and torch.equal(idx.scale[:n], scale)
     with pytest.raises(ValueError, match="capacity"):

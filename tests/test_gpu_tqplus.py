@@ -159,7 +159,8 @@ def test_index_tqplus_ingest_and_persist(cuda_lib, tdev, tmp_path):
     ref = O.calibrate(X[:1200], idx.R.cpu().numpy())
     mu, a = (t.cpu().numpy() for t in idx.calib)
     assert np.max(np.abs(mu - ref.mu)) <= 2e-7 and np.max(np.abs(a / ref.a - 1)) <= 2e-5
-    codes, scale = tq.encode(T(X), idx.R, idx.centroids, idx.boundaries, bits, calib=idx.calib)
+    codes, scale = tq.encode(T(X), idx.R, idx.centroids, idx.boundaries, bits, calib=idx.calib,
+                             plan=idx.plan)
     torch.cuda.synchronize()
     assert torch.equal(codes, idx.codes[:3000]) and torch.equal(scale, idx.scale[:3000])
     Q = T(synth.perturb(X[:7] / np.linalg.norm(X[:7], axis=1, keepdims=True)))

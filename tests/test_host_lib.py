@@ -143,6 +143,27 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert lib.tq_calibrate(p, 300, 64, p, p, p, p, sz.value - 1, null) == _lib.TQ_EINVAL
     assert lib.tq_calibrate(null, 300, 64, p, p, p, p, sz.value, null) == _lib.TQ_EINVAL
     assert lib.tq_encode_ex(p, 10, 64, p, p, p, 4, 0, p, null, p, p, null) == _lib.TQ_EINVAL
+    # tensor-core encode plan: sizes and argument checks (no device memory is touched)
+    assert lib.tq_encode_plan_bytes(1536, C.byref(sz)) == _lib.TQ_OK
+    assert sz.value == 256 + 2 * 1536 * 1536 * 4    # status header, R_hi, R_lo
+    for d in (64, 96, 130, 8224):
+        assert lib.tq_encode_plan_bytes(d, C.byref(sz)) == _lib.TQ_EUNSUPPORTED
+    assert lib.tq_encode_plan_bytes(128, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode_plan(p, 96, p, 1 << 20, null) == _lib.TQ_EUNSUPPORTED
+    assert lib.tq_encode_plan(p, 128, p + 8, 1 << 20, null) == _lib.TQ_EINVAL
+    assert lib.tq_encode_plan(p, 128, p, 1000, null) == _lib.TQ_EINVAL
+    planned = lambda **kw: lib.tq_encode_planned(*[kw.get(k, v) for k, v in (
+        ("X", p), ("n", 10), ("d", 128), ("plan", p), ("c", p), ("b", p), ("bits", 4), ("mode", 0),
+        ("mu", null), ("a", null), ("codes", p), ("scale", p), ("s", null))])
+    assert planned(d=96) == _lib.TQ_EUNSUPPORTED
+    assert planned(d=100) == _lib.TQ_EINVAL
+    assert planned(bits=5) == _lib.TQ_EINVAL
+    assert planned(plan=null) == _lib.TQ_EINVAL
+    assert planned(plan=p + 4) == _lib.TQ_EINVAL
+    assert planned(mu=p) == _lib.TQ_EINVAL
+    assert planned(n=-1) == _lib.TQ_EINVAL
+    assert planned(n=0) == _lib.TQ_OK
+    assert lib.tq_encode_check(null, null) == _lib.TQ_EINVAL
     # id map: capacity, NULL handle / ids (no device memory is touched)
     m = C.c_void_p()
     assert lib.tq_idmap_create(0, C.byref(m)) == _lib.TQ_EINVAL
