@@ -350,17 +350,23 @@ def run_ours(args, cfg, rank, world):
         codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
         scale = torch.empty(n, dtype=torch.float32, device=dev)
         Qd = torch.from_numpy(Qpool).to(dev)
+        plan = tq.encode_plan(Rd, stream=stream)  # the index's split of R (built once, like R itself)
     del X
     barrier()
-    enc_ms = []
-    for i in range(3):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream)
-        e1.record(stream)
-        e1.synchronize()
-        enc_ms.append(e0.elapsed_time(e1))
-    enc_ms = min(enc_ms[1:])
+
+    def enc_time(**kw):
+        ts = []
+        for i in range(3):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream, **kw)
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        return min(ts[1:])
+    ffma_ms = enc_time()             # the FFMA encoder, for comparison
+    enc_ms = enc_time(plan=plan)     # the tensor-core encoder: the codes the searches use
+    tq.encode_check(plan, stream=stream)
     # ground truth for Recall@k: exact float32 inner products of the first
     # RECALL_Q queries with the unquantised normalised corpus (torch matmul,
     # outside the timed regions; TF32 off)
@@ -379,7 +385,8 @@ def run_ours(args, cfg, rank, world):
     if not run_extras:
         del Xd
     torch.cuda.empty_cache()
-    log(f"[bench] encode {n} vectors: {enc_ms:.1f} ms ({n / enc_ms * 1e3:.3g} vec/s)")
+    log(f"[bench] encode {n} vectors: {enc_ms:.1f} ms ({n / enc_ms * 1e3:.3g} vec/s; FFMA encoder "
+        f"{ffma_ms:.1f} ms)")
 
     pk = peaks()
     pci = None
@@ -568,7 +575,9 @@ def run_ours(args, cfg, rank, world):
                              "roofline": v["roofline"], "e2e": v["e2e"], "gpu_launches": v["gpu_launches"]}
                     for b, v in results.items()},
         "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
-                   "tflops": 2.0 * n * d * d / (enc_ms / 1e3) / 1e12},
+                   "path": "tensor core (TF32, three-product split)", "roofline": _roof_encode(n, d, enc_ms, pk),
+                   "ffma": {"value": n / ffma_ms * 1e3, "unit": "vectors/s", "ms": ffma_ms,
+                            "tflops": 2.0 * n * d * d / (ffma_ms / 1e3) / 1e12}},
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         qps_cpu, info = oracle_qps_sample(cfg, sample_rows=min(n, args.ref_sample), n_queries=5)
@@ -669,6 +678,22 @@ def _roof_tc(flops, ms, pk):
             "traffic": None, "kernel": "k_scan_mma", "alg_flops_per_launch": flops, "kernel_ms": ms}
 
 
+TF32_PER_BF16 = 1.1 / 2.25  # nominal dense TF32 / BF16 tensor rates of the GB300
+
+
+def _roof_encode(n, d, ms, pk):
+    """Roofline of the tensor-core encoder: three TF32 products per
+    multiply-add of the rotation (2 n d^2 flops each), against the TF32
+    peak taken as the measured burst bf16 peak times the nominal ratio."""
+    flops = 3 * 2.0 * n * d * d
+    tf = flops / (ms / 1e3) / 1e12
+    peak = pk["bf16_tflops"] * TF32_PER_BF16
+    return {"bound": "tensor", "achieved": tf, "peak": peak, "unit": "TFLOP/s", "frac": tf / peak,
+            "frac_of": pk["source"] + " burst bf16 x 1.1/2.25 (TF32 dense rate)", "traffic": None,
+            "kernel": "k_encode_tc", "alg_flops_per_launch": flops, "kernel_ms": ms,
+            "rotation_tflops": 2.0 * n * d * d / (ms / 1e3) / 1e12}
+
+
 def _recall(torch, ids, exact):
     """Mean |ids ∩ exact| / |exact| over queries (torch tensors [nq, k]; -1 is no result)."""
     hits = 0.0
@@ -695,14 +720,16 @@ def extras_100k(torch, tq, dev, stream, pk, flush, steps):
     nrec = min(RECALL_Q, len(Q))
     with torch.cuda.stream(stream):
         Xd, Qd, Rd, cd, bd = (torch.from_numpy(a).to(dev) for a in (X, Q, R, cen, bnd))
-        codes, scale = tq.encode(Xd, Rd, cd, bd, bits, stream=stream)
-        enc_ms = _flushed_ms(torch, lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream),
-                             3, stream, flush)
+        plan = tq.encode_plan(Rd, stream=stream)
+        codes, scale = tq.encode(Xd, Rd, cd, bd, bits, stream=stream, plan=plan)
+        enc_ms = _flushed_ms(torch, lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream,
+                                                        plan=plan), 3, stream, flush)
         exact_sc = Qd[:nrec] @ Xd.T                      # float32, TF32 off: [nrec, n]
     stream.synchronize()
     out = {"workload": f"N={n} d={d} {bits}-bit, {cfg['clusters']}-cluster mixture, {len(Q)} queries",
            "l2": "corpus fits in L2: flushed before every timed call",
-           "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms}}
+           "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
+                      "roofline": _roof_encode(n, d, enc_ms, pk)}}
     alg = n * (d * bits // 8 + 4)
     for B in (1, 256):
         for k in (5, 10):
@@ -822,13 +849,14 @@ def extras_sweep(torch, tq, dev, stream, pk, Xd, Rd, Qd, steps):
     n, d, k, B = cfg["n"], cfg["d"], cfg["k"], cfg["batches"][0]
     nb = max(1, Qd.shape[0] // B)
     out = {"workload": f"N={n} d={d}, batch {B}, top-{k}; corpus larger than L2", "variants": {}}
+    plan = tq.encode_plan(Rd, stream=stream)
     for bits in cfg["sweep_bits"]:
         cen, bnd, _ = tq.codebook(d, bits)
         cd, bd = torch.from_numpy(cen).to(dev), torch.from_numpy(bnd).to(dev)
         with torch.cuda.stream(stream):
             codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
             scale = torch.empty(n, dtype=torch.float32, device=dev)
-            enc = lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream)
+            enc = lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream, plan=plan)
             enc(0)
             enc_ms = _timed(enc, 3, 1, stream)
             ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
@@ -847,7 +875,7 @@ def extras_sweep(torch, tq, dev, stream, pk, Xd, Rd, Qd, steps):
         out["variants"][str(bits)] = {"value": B / ms * 1e3, "unit": "queries/s", "ms_per_step": ms,
                                       "path": "tensor core" if mma else "lookup", "roofline": roof,
                                       "encode": {"value": n / enc_ms * 1e3, "unit": "vectors/s", "ms": enc_ms,
-                                                 "tflops": 2.0 * n * d * d / (enc_ms / 1e3) / 1e12}}
+                                                 "roofline": _roof_encode(n, d, enc_ms, pk)}}
         log(f"[bench] sweep b={bits}: encode {n / enc_ms * 1e3:.3g} vec/s, batch {B}: {B / ms * 1e3:.4g} q/s")
         del codes, scale, ws
         torch.cuda.empty_cache()
@@ -875,7 +903,7 @@ def run_filtered(args, cfg):
     R = tq.rotation(d, synth.SEED_ROTATION)
     Xd, Qd = torch.from_numpy(X).to(dev), torch.from_numpy(Q).to(dev)
     Rd, cd, bd = (torch.from_numpy(a).to(dev) for a in (R, cen, bnd))
-    codes, scale = tq.encode(Xd, Rd, cd, bd, bits)
+    codes, scale = tq.encode(Xd, Rd, cd, bd, bits, plan=tq.encode_plan(Rd))
     torch.cuda.synchronize()
     torch.backends.cuda.matmul.allow_tf32 = False
     nrec = min(RECALL_Q, len(Q))
@@ -980,14 +1008,15 @@ def run_sweep(args, cfg):
     del X
     nb = max(1, len(Qpool) // B)
     variants = {}
+    plan = tq.encode_plan(Rd)
     for bits in cfg["sweep_bits"]:
         cen, bnd, _ = tq.codebook(d, bits)
         cd, bd = torch.from_numpy(cen).to(dev), torch.from_numpy(bnd).to(dev)
         codes = torch.empty((n, d * bits // 8), dtype=torch.uint8, device=dev)
         scale = torch.empty(n, dtype=torch.float32, device=dev)
         with torch.cuda.stream(stream):
-            enc_ms = _timed(lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream), 3, 1,
-                            stream)
+            enc_ms = _timed(lambda i: tq.encode(Xd, Rd, cd, bd, bits, "norm", codes, scale, stream=stream,
+                                                plan=plan), 3, 1, stream)
             ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
             ids = torch.empty((B, k), dtype=torch.int64, device=dev)
             scs = torch.empty((B, k), dtype=torch.float32, device=dev)
@@ -1035,7 +1064,7 @@ def run_idmap(args, cfg):
     R = tq.rotation(d, synth.SEED_ROTATION)
     Xd = torch.from_numpy(X).to(dev)
     Rd, cd, bd, Qd = (torch.from_numpy(a).to(dev) for a in (R, cen, bnd, Qpool))
-    codes, scale = tq.encode(Xd, Rd, cd, bd, bits)
+    codes, scale = tq.encode(Xd, Rd, cd, bd, bits, plan=tq.encode_plan(Rd))
     del Xd, X
     rng = np.random.default_rng(synth.SEED_QUERIES)
     ext = rng.choice(1 << 62, size=n, replace=False).astype(np.uint64)

@@ -14,7 +14,11 @@
 //
 // Work.  A CTA owns panels of 128 rows of X (the MMA's M) and walks the d
 // output coordinates in chunks of 256 (N), each chunk a full contraction over
-// K = d in K-blocks of 32 coordinates (one 128-byte swizzled row of fp32).
+// K = d in K-blocks of 16 coordinates (64-byte rows of fp32 with the 64-byte
+// swizzle: 48 KB stages, four in flight, so the copy and the split of a
+// K-block are hidden behind the MMAs of the three before it).  Chunks walk the
+// K-blocks alternately forwards and backwards, so a chunk starts on the X
+// tiles the previous one read last (still in L2).
 // TMEM holds two 128 x 256 fp32 accumulator sets, so the epilogue of one
 // chunk overlaps the MMAs of the next.  Roles (14 warps):
 //   warps 0-3   converters: thread t owns row t of each X tile, splits it in
@@ -47,10 +51,10 @@ namespace {
 
 constexpr int EM = 128;                     // rows of X per panel (MMA M)
 constexpr int EN = 256;                     // output coordinates per chunk (MMA N)
-constexpr int EK = 32;                      // coordinates per K-block (128 B of fp32)
-constexpr int NSTAGE = 2;                   // K-block stages in flight
-constexpr int X_BYTES = EM * EK * 4;        // 16 KB: an X tile (x_hi after the split)
-constexpr int R_BYTES = EN * EK * 4;        // 32 KB: an R_hi or R_lo tile
+constexpr int EK = 16;                      // coordinates per K-block (64 B of fp32)
+constexpr int NSTAGE = 4;                   // K-block stages in flight
+constexpr int X_BYTES = EM * EK * 4;        // 8 KB: an X tile (x_hi after the split)
+constexpr int R_BYTES = EN * EK * 4;        // 16 KB: an R_hi or R_lo tile
 constexpr int STAGE_BYTES = 2 * X_BYTES + 2 * R_BYTES;  // x_hi, x_lo, r_hi, r_lo
 constexpr int CONV_WARPS = 4, PROD_WARP = 4, MMA_WARP = 5, EPI_WARP0 = 6, EPI_WARPS = 8;
 constexpr int ENC_THREADS = (EPI_WARP0 + EPI_WARPS) * 32;  // 448
@@ -69,7 +73,7 @@ struct EncSmem {
   static constexpr uint32_t inv = nrm + 2 * EM * 4;      // [2][128] 1 / norm
   static constexpr uint32_t part = inv + 2 * EM * 4;     // [2][2][128] double: sum c^2, sum y c of the column-128..255 warps
   static constexpr uint32_t bars = part + 4 * EM * 8;    // mbarriers
-  static constexpr uint32_t nbars = 20;
+  static constexpr uint32_t nbars = 24;
   static constexpr uint32_t misc = bars + nbars * 8;     // TMEM address, abort flag
   static constexpr uint32_t total = misc + 16;
 };
@@ -126,15 +130,15 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   float* sInv = reinterpret_cast<float*>(base + EncSmem::inv);
   double* sPart = reinterpret_cast<double*>(base + EncSmem::part);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + EncSmem::bars);
-  uint64_t* full = bars;             // [2] X and R tiles landed
-  uint64_t* conv = bars + 2;         // [2] X tile split
-  uint64_t* empty = bars + 4;        // [2] MMAs done with the stage
-  uint64_t* acc_full = bars + 6;     // [2] accumulator set complete
-  uint64_t* acc_empty = bars + 8;    // [2] accumulator set read out
-  uint64_t* norm_ready = bars + 10;  // [2] row norms of a panel written (by panel parity)
-  uint64_t* norm_free = bars + 12;   // [2] row norms of a panel read
-  uint64_t* part_ready = bars + 14;  // [2] column-128..255 sums of a panel written
-  uint64_t* fin = bars + 16;         // every MMA of this CTA complete
+  uint64_t* full = bars;             // [NSTAGE] X and R tiles landed
+  uint64_t* conv = bars + 4;         // [NSTAGE] X tile split
+  uint64_t* empty = bars + 8;        // [NSTAGE] MMAs done with the stage
+  uint64_t* acc_full = bars + 12;    // [2] accumulator set complete
+  uint64_t* acc_empty = bars + 14;   // [2] accumulator set read out
+  uint64_t* norm_ready = bars + 16;  // [2] row norms of a panel written (by panel parity)
+  uint64_t* norm_free = bars + 18;   // [2] row norms of a panel read
+  uint64_t* part_ready = bars + 20;  // [2] column-128..255 sums of a panel written
+  uint64_t* fin = bars + 22;         // every MMA of this CTA complete
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + EncSmem::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + EncSmem::misc + 4);
 
@@ -187,14 +191,15 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         const long long cs = it / KB;
         const int c = (int)(cs % C), i = (int)(cs / C);
         const int panel = (int)blockIdx.x + i * (int)gridDim.x;
+        const int kc = (c & 1) ? KB - 1 - kb : kb;  // snake order over the K-blocks
         unsigned char* st = base + s * STAGE_BYTES;
         mbar_arrive_expect_tx(full + s, X_BYTES + 2 * R_BYTES);
-        tma_load_2d(st, &xmap, kb * EK, panel * EM, full + s);
+        tma_load_2d(st, &xmap, kc * EK, panel * EM, full + s);
         // rows c*256 .. of R_hi, then of R_lo (rows d .. 2d-1 of the plan); in a
         // partial last chunk the rows past d are R_lo rows or zero fill, and the
         // epilogue never reads their columns
-        tma_load_2d(st + 2 * X_BYTES, &rmap, kb * EK, c * EN, full + s);
-        tma_load_2d(st + 2 * X_BYTES + R_BYTES, &rmap, kb * EK, d + c * EN, full + s);
+        tma_load_2d(st + 2 * X_BYTES, &rmap, kc * EK, c * EN, full + s);
+        tma_load_2d(st + 2 * X_BYTES + R_BYTES, &rmap, kc * EK, d + c * EN, full + s);
         issued = it + 1;
       }
       // never leave with copies in flight: wait (bounded) for the last one of each stage
@@ -221,9 +226,9 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
 #pragma unroll
         for (int kk = 0; kk < EK / 8; ++kk) {  // K = 8 TF32 values = 32 bytes of each row
           const uint32_t o = (uint32_t)kk * 32u;
-          mma_tf32(dt, sw128_desc(xh + o), sw128_desc(rh + o), (kb | kk) != 0);
-          mma_tf32(dt, sw128_desc(xh + o), sw128_desc(rl + o), 1u);
-          mma_tf32(dt, sw128_desc(xl + o), sw128_desc(rh + o), 1u);
+          mma_tf32(dt, sw64_desc(xh + o), sw64_desc(rh + o), (kb | kk) != 0);
+          mma_tf32(dt, sw64_desc(xh + o), sw64_desc(rl + o), 1u);
+          mma_tf32(dt, sw64_desc(xl + o), sw64_desc(rh + o), 1u);
         }
         mma_commit(empty + s);
         if (kb == KB - 1) mma_commit(acc_full + set);
@@ -234,7 +239,8 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   } else if (warp < CONV_WARPS) {
     // ------------------------------------------------------------- converters
     // Thread t owns row t; reading the 16-byte parts in logical order through
-    // the swizzle keeps a warp's accesses free of bank conflicts.  The row's
+    // the 64-byte swizzle (part q of row t sits at part q ^ ((t >> 1) & 3))
+    // keeps a warp's accesses free of bank conflicts.  The row's
     // sum of squares takes a fixed order: four float partials per K-block,
     // paired, then added in double across K-blocks (a plain float running
     // sum over d terms would lose ~sqrt(d) ulps).
@@ -252,7 +258,7 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
       float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
 #pragma unroll
       for (int q = 0; q < EK / 4; ++q) {
-        const uint32_t off = (uint32_t)t * 128u + ((uint32_t)(q ^ (t & 7)) << 4);
+        const uint32_t off = (uint32_t)t * 64u + ((uint32_t)(q ^ ((t >> 1) & 3)) << 4);
         const float4 v = *reinterpret_cast<const float4*>(xt + off);
         p0 = fmaf(v.x, v.x, p0);
         p1 = fmaf(v.y, v.y, p1);
@@ -432,7 +438,7 @@ cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan,
     const cuuint64_t gstride[1] = {(cuuint64_t)d * sizeof(float)};
     const cuuint32_t box[2] = {(cuuint32_t)EK, (cuuint32_t)EM};
     const CUresult r = enc(&xmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(X), gdim, gstride, box,
-                           estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   }
@@ -441,7 +447,7 @@ cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan,
     const cuuint64_t gstride[1] = {(cuuint64_t)d * sizeof(float)};
     const cuuint32_t box[2] = {(cuuint32_t)EK, (cuuint32_t)EN};
     const CUresult r = enc(&rmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<unsigned char*>(pl + kPlanHeader),
-                           gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           gdim, gstride, box, estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
   }
