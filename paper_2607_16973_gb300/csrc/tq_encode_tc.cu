@@ -67,9 +67,11 @@ constexpr size_t kPlanHeader = 256;
 // Offsets in the 1024-byte-aligned dynamic shared memory.
 struct EncSmem {
   // stage s at s * STAGE_BYTES: x_hi, x_lo, r_hi, r_lo tiles
-  static constexpr uint32_t bnd = NSTAGE * STAGE_BYTES;  // [256] boundaries (255 used)
-  static constexpr uint32_t cen = bnd + 256 * 4;         // [256] centroids
-  static constexpr uint32_t nrm = cen + 256 * 4;         // [2][128] row norms by panel parity
+  // boundaries and centroids: with codes of up to 4 bits one copy per bank
+  // ([entry][32]), so the epilogue's data-dependent lookups never conflict
+  static constexpr uint32_t bnd = NSTAGE * STAGE_BYTES;  // [512] floats
+  static constexpr uint32_t cen = bnd + 512 * 4;         // [512] floats
+  static constexpr uint32_t nrm = cen + 512 * 4;         // [2][128] row norms by panel parity
   static constexpr uint32_t inv = nrm + 2 * EM * 4;      // [2][128] 1 / norm
   static constexpr uint32_t part = inv + 2 * EM * 4;     // [2][2][128] double: sum c^2, sum y c of the column-128..255 warps
   static constexpr uint32_t bars = part + 4 * EM * 8;    // mbarriers
@@ -122,6 +124,7 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
             const float* __restrict__ cal_mu, const float* __restrict__ cal_a, uint8_t* __restrict__ codes,
             float* __restrict__ scale, int* __restrict__ err) {
   constexpr int L = 1 << BITS;
+  constexpr int REP = BITS <= 4 ? 32 : 1;  // copies of each table entry (one per bank)
   extern __shared__ unsigned char smem_dyn[];
   unsigned char* base = smem_dyn + ((1024u - (smem_u32(smem_dyn) & 1023u)) & 1023u);
   float* sBnd = reinterpret_cast<float*>(base + EncSmem::bnd);
@@ -149,9 +152,10 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   const int my_panels = (int)blockIdx.x < panels ? (panels - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
   const long long total_it = (long long)my_panels * C * KB;
 
-  for (int i = tid; i < 256; i += ENC_THREADS) {
-    sCen[i] = i < L ? centroids[i] : 0.f;
-    sBnd[i] = i < L - 1 ? boundaries[i] : INFINITY;
+  for (int i = tid; i < 512; i += ENC_THREADS) {
+    const int e = i / REP;
+    sCen[i] = e < L ? centroids[e] : 0.f;
+    sBnd[i] = e < L - 1 ? boundaries[e] : INFINITY;
   }
   if (tid == 0) {
     for (int s = 0; s < NSTAGE; ++s) {
@@ -291,6 +295,7 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     const int row = quarter * 32 + lane;
     const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(h * (EN / 2));
     const int64_t rbytes = (int64_t)d * BITS / 8;
+    const int rl = lane & (REP - 1);  // this lane's copy of the tables
     float inv = 0.f, nr = 0.f;
     double c2 = 0.0, yc = 0.0;  // the row's sums over this thread's columns (float per 16, then double)
     int64_t grow = 0;
@@ -312,8 +317,9 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         int code = 0;
 #pragma unroll
         for (int step = L / 2; step >= 1; step >>= 1)
-          if (z > sBnd[code + step - 1]) code += step;
-        const float cv = CAL ? fmaf(a, sCen[code], mu) : sCen[code];
+          if (z > sBnd[(code + step - 1) * REP + rl]) code += step;
+        const float cc = sCen[code * REP + rl];
+        const float cv = CAL ? fmaf(a, cc, mu) : cc;
         g2 = fmaf(cv, cv, g2);
         gy = fmaf(y, cv, gy);
         if constexpr (BITS == 8) p8[t >> 2] |= (uint32_t)code << (8 * (t & 3));
