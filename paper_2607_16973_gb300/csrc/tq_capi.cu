@@ -31,13 +31,15 @@ inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct SearchPlan {
   int grid_lut = 1, grid_mma = 0;
-  size_t off_status = 0, off_cnt = 0, off_bias = 0, off_rot = 0, off_allow = 0, off_mask = 0, off_qpack = 0,
-         off_cs = 0, off_ci = 0, total = 0;
+  size_t off_status = 0, off_cnt = 0, off_bias = 0, off_rot = 0, off_part = 0, off_allow = 0, off_mask = 0,
+         off_qpack = 0, off_cs = 0, off_ci = 0, total = 0;
+  bool rot_tc = false;  // the query rotation runs on the tensor cores
 };
 
 // Workspace layout (both scan paths): status word | merge counters (one per
-// query) | TQ+ query terms (one per query) | rotated queries | allow bitmaps |
-// block masks | fp16 query tiles (tensor-core path) | candidate scores | ids.
+// query) | TQ+ query terms (one per query) | rotated queries | partial
+// rotations (tensor-core rotation) | allow bitmaps | block masks | fp16 query
+// tiles (tensor-core scan) | candidate scores | ids.
 SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_filter* filter) {
   SearchPlan p;
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
@@ -53,6 +55,9 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   off = align_up(off + (size_t)nq * sizeof(float));
   p.off_rot = off;
   off = align_up(off + (size_t)nq * d * sizeof(float));
+  p.rot_tc = rotate_tc_applies(nq, d);
+  p.off_part = off;
+  if (p.rot_tc) off = align_up(off + rotate_tc_part_bytes(nq, d));
   p.off_allow = off;
   if (filter) off = align_up(off + (size_t)nq * filter->f.words * sizeof(uint32_t));
   p.off_mask = off;
@@ -431,7 +436,10 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
   float* cs = reinterpret_cast<float*>(ws + p.off_cs);
   int32_t* ci = reinterpret_cast<int32_t*>(ws + p.off_ci);
   float* bias = cal_mu ? reinterpret_cast<float*>(ws + p.off_bias) : nullptr;
-  cudaError_t e = tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);  // also zeroes both
+  // the rotation also clears the status word and zeroes the merge counters
+  cudaError_t e = p.rot_tc ? tq::launch_rotate_tc(Q, nq, d, R, qrot, reinterpret_cast<float*>(ws + p.off_part),
+                                                  status, counters, nq, s)
+                           : tq::launch_rotate(Q, nq, d, R, qrot, status, counters, nq, s);
   if (e == cudaSuccess && cal_mu) e = tq::launch_calib_query(qrot, nq, d, cal_mu, cal_a, bias, s);
   if (use_mma) {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);

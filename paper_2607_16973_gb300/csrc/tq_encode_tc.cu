@@ -416,6 +416,177 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   if (warp == MMA_WARP) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 512;" ::"r"(tmem));
 }
 
+// Query rotation on the tensor cores (Sec. II-B step 2 for a batch of
+// queries): part[s] = Q R^T over split s of the K-blocks, with the same
+// three-product TF32 split; the search is given R itself, so R's tiles are
+// split in shared memory as they arrive, like Q's.  CTA (c, p, s) computes
+// output coordinates c*256 .., query rows p*128 .., K-blocks
+// [s*KB/S, (s+1)*KB/S); k_rotate_reduce adds the S partial products in a
+// fixed order.  Roles (10 warps): warps 0-3 split the Q tile (row t) and the
+// R tile (rows t, t+128); warp 4 issues the copies; warp 5 the MMAs (one
+// 128 x 256 accumulator); warps 6-9 store the accumulator (lane quarter
+// w % 4, all 256 columns).
+constexpr int ROT_EPI0 = 6;
+constexpr int ROT_THREADS = (ROT_EPI0 + 4) * 32;
+constexpr uint32_t kRotBars = NSTAGE * STAGE_BYTES;
+constexpr uint32_t kRotSmem = kRotBars + 16 * 8 + 16 + 1024;
+static_assert(kRotSmem <= kEncDynSmemMax, "rotation shared memory");
+
+__global__ void __launch_bounds__(ROT_THREADS, 1)
+k_rotate_tc(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap rmap, int nq, int d,
+            int S, float* __restrict__ part, int* __restrict__ err) {
+  extern __shared__ unsigned char smem_dyn[];
+  unsigned char* base = smem_dyn + ((1024u - (smem_u32(smem_dyn) & 1023u)) & 1023u);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + kRotBars);
+  uint64_t* full = bars;          // [NSTAGE] Q and R tiles landed
+  uint64_t* conv = bars + 4;      // [NSTAGE] both tiles split
+  uint64_t* empty = bars + 8;     // [NSTAGE] MMAs done with the stage
+  uint64_t* acc_full = bars + 12;
+  uint64_t* fin = bars + 13;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(bars + 16) + 1;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int c = blockIdx.x, p = blockIdx.y, sp = blockIdx.z;
+  const int KB = d / EK;
+  const int kb0 = (int)((long long)sp * KB / S), nk = (int)((long long)(sp + 1) * KB / S) - kb0;
+  if (tid == 0) {
+    // a new search: clear the status word (any wait that gives up records
+    // itself there, seconds after every CTA has started)
+    if (c == 0 && p == 0 && sp == 0) *err = 0;
+    for (int i = 0; i < NSTAGE; ++i) {
+      mbar_init(full + i, 1);
+      mbar_init(conv + i, CONV_WARPS);
+      mbar_init(empty + i, 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(fin, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == MMA_WARP) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], 256;" ::"r"(smem_u32(tmem_slot)));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == PROD_WARP) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % NSTAGE, use = it / NSTAGE;
+        if (use > 0 && !mbar_wait(empty + s, (uint32_t)((use - 1) & 1), abort_flag, err, 51)) break;
+        unsigned char* st = base + s * STAGE_BYTES;
+        mbar_arrive_expect_tx(full + s, X_BYTES + R_BYTES);
+        tma_load_2d(st, &qmap, (kb0 + it) * EK, p * EM, full + s);
+        tma_load_2d(st + 2 * X_BYTES, &rmap, (kb0 + it) * EK, c * EN, full + s);
+        issued = it + 1;
+      }
+      for (int s = 0; s < NSTAGE && s < issued; ++s)
+        mbar_wait_drain(full + s, (uint32_t)(((issued - 1 - s) / NSTAGE) & 1));
+    }
+  } else if (warp == MMA_WARP) {
+    if (lane == 0) {
+      for (int it = 0; it < nk; ++it) {
+        const int s = it % NSTAGE, use = it / NSTAGE;
+        if (!mbar_wait(conv + s, (uint32_t)(use & 1), abort_flag, err, 52)) break;
+        tc_fence_after();
+        const uint32_t xh = smem_u32(base + s * STAGE_BYTES);
+        const uint32_t xl = xh + X_BYTES, rh = xh + 2 * X_BYTES, rl = rh + R_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < EK / 8; ++kk) {
+          const uint32_t o = (uint32_t)kk * 32u;
+          mma_tf32(tmem, sw64_desc(xh + o), sw64_desc(rh + o), (it | kk) != 0);
+          mma_tf32(tmem, sw64_desc(xh + o), sw64_desc(rl + o), 1u);
+          mma_tf32(tmem, sw64_desc(xl + o), sw64_desc(rh + o), 1u);
+        }
+        mma_commit(empty + s);
+        if (it == nk - 1) mma_commit(acc_full);
+      }
+      mma_commit(fin);
+      mbar_wait_drain(fin, 0);
+    }
+  } else if (warp < CONV_WARPS) {
+    // thread t splits row t of the Q tile and rows t, t + 128 of the R tile
+    const int t = tid;
+    auto split_row = [&](unsigned char* hi, unsigned char* lo, int r) {
+#pragma unroll
+      for (int q = 0; q < EK / 4; ++q) {
+        const uint32_t off = (uint32_t)r * 64u + ((uint32_t)(q ^ ((r >> 1) & 3)) << 4);
+        const float4 v = *reinterpret_cast<const float4*>(hi + off);
+        const float4 h = make_float4(tf32_round(v.x), tf32_round(v.y), tf32_round(v.z), tf32_round(v.w));
+        *reinterpret_cast<float4*>(hi + off) = h;
+        *reinterpret_cast<float4*>(lo + off) = make_float4(tf32_round(v.x - h.x), tf32_round(v.y - h.y),
+                                                           tf32_round(v.z - h.z), tf32_round(v.w - h.w));
+      }
+    };
+    for (int it = 0; it < nk; ++it) {
+      const int s = it % NSTAGE, use = it / NSTAGE;
+      if (!warp_wait(full + s, (uint32_t)(use & 1), abort_flag, err, 53)) break;
+      unsigned char* st = base + s * STAGE_BYTES;
+      split_row(st, st + X_BYTES, t);
+      split_row(st + 2 * X_BYTES, st + 2 * X_BYTES + R_BYTES, t);
+      split_row(st + 2 * X_BYTES, st + 2 * X_BYTES + R_BYTES, t + EM);
+      fence_proxy_async();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(conv + s);
+    }
+  } else if (warp >= ROT_EPI0) {
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    const int64_t q = (int64_t)p * EM + row;
+    if (nk > 0 && warp_wait(acc_full, 0, abort_flag, err, 54)) {
+      tc_fence_after();
+      float* dst = part + ((int64_t)sp * nq + q) * d;
+      const uint32_t tl = tmem + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+      for (int g = 0; g < EN / 16; ++g) {
+        uint32_t r[16];
+        tmem_ld16_issue(tl + (uint32_t)(g * 16), r);
+        tmem_wait16(r);
+        const int j0 = c * EN + g * 16;
+        if (q < nq && j0 < d) {
+          float4* o = reinterpret_cast<float4*>(dst + j0);
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+            o[u] = make_float4(__uint_as_float(r[4 * u]), __uint_as_float(r[4 * u + 1]),
+                               __uint_as_float(r[4 * u + 2]), __uint_as_float(r[4 * u + 3]));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == MMA_WARP) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, 256;" ::"r"(tmem));
+}
+
+// out = sum of the S partial products in split order; also zeroes the
+// search's merge counters, and lets the scan launched after it (as a
+// programmatic dependent) start its prologue.
+__global__ void __launch_bounds__(256)
+k_rotate_reduce(const float4* __restrict__ part, int S, int64_t n4, float4* __restrict__ out, int* counters,
+                int64_t n_counters) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  const int64_t i0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (counters)
+    for (int64_t i = i0; i < n_counters; i += stride) counters[i] = 0;
+  for (int64_t i = i0; i < n4; i += stride) {
+    float4 a = __ldcs(part + i);
+    for (int s = 1; s < S; ++s) {
+      const float4 b = __ldcs(part + (int64_t)s * n4 + i);
+      a.x += b.x;
+      a.y += b.y;
+      a.z += b.z;
+      a.w += b.w;
+    }
+    out[i] = a;
+  }
+}
+
 }  // namespace
 
 bool encode_tc_supported(int d) { return d >= 128 && d <= kMaxD && d % EK == 0; }
@@ -484,6 +655,58 @@ cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan,
     default: return cudaErrorInvalidValue;
   }
 #undef TQ_ENC_TC_CASE
+  return cudaGetLastError();
+}
+
+int rotate_tc_splits(int64_t nq, int d) {
+  const int KB = d / EK;
+  const int64_t items = ((nq + EM - 1) / EM) * ((d + EN - 1) / EN);
+  int64_t sp = (int64_t)device_sm_count() / std::max<int64_t>(items, 1);
+  sp = std::min<int64_t>(sp, std::max(1, KB / 8));  // at least 8 K-blocks per split
+  return (int)std::max<int64_t>(sp, 1);
+}
+
+bool rotate_tc_applies(int64_t nq, int d) { return nq >= kRotTcMinBatch && encode_tc_supported(d); }
+
+size_t rotate_tc_part_bytes(int64_t nq, int d) {
+  return rotate_tc_applies(nq, d) ? (size_t)rotate_tc_splits(nq, d) * nq * d * sizeof(float) : 0;
+}
+
+cudaError_t launch_rotate_tc(const float* Q, int64_t nq, int d, const float* R, float* out, float* part,
+                             int* status, int* counters, int64_t n_counters, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  if (!rotate_tc_applies(nq, d) || nq > INT32_MAX) return cudaErrorInvalidValue;
+  PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
+  if (!enc) return cudaErrorNotSupported;
+  CUtensorMap qmap, rmap;
+  const cuuint32_t estride[2] = {1, 1};
+  const cuuint64_t gstride[1] = {(cuuint64_t)d * sizeof(float)};
+  {
+    const cuuint64_t gdim[2] = {(cuuint64_t)d, (cuuint64_t)nq};
+    const cuuint32_t box[2] = {(cuuint32_t)EK, (cuuint32_t)EM};
+    if (enc(&qmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(Q), gdim, gstride, box, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t gdim[2] = {(cuuint64_t)d, (cuuint64_t)d};
+    const cuuint32_t box[2] = {(cuuint32_t)EK, (cuuint32_t)EN};
+    if (enc(&rmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(R), gdim, gstride, box, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  const int S = rotate_tc_splits(nq, d);
+  cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_rotate_tc), (int)kRotSmem);
+  if (e != cudaSuccess) return e;
+  const dim3 grid((unsigned)((d + EN - 1) / EN), (unsigned)((nq + EM - 1) / EM), (unsigned)S);
+  k_rotate_tc<<<grid, ROT_THREADS, kRotSmem, s>>>(qmap, rmap, (int)nq, d, S, part, status);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int64_t n4 = nq * d / 4;
+  const int blocks = (int)std::min<int64_t>((n4 + 255) / 256, (int64_t)device_sm_count() * 8);
+  k_rotate_reduce<<<std::max(blocks, 1), 256, 0, s>>>(reinterpret_cast<const float4*>(part), S, n4,
+                                                       reinterpret_cast<float4*>(out), counters, n_counters);
   return cudaGetLastError();
 }
 

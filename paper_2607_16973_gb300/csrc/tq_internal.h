@@ -23,6 +23,7 @@ constexpr int kMaxK = 256;
 constexpr int kMaxKMma = 64;     // per-thread top-k lists of the tensor-core scan
 constexpr int kMmaMinBatch = 16; // AUTO uses the tensor-core scan from this batch size
 constexpr int kMaxD = 8192;
+constexpr int kRotTcMinBatch = 16;  // query batches rotated on the tensor cores from this size
 // The fixed-point 4-bit centroid table (TQ_PATH_LUT_FIXED) applies from this
 // d on: its rounding error is about 2^-16 of the largest centroid (~3.5 /
 // sqrt(d)), so below it the exact fp32 table keeps unit-query scores within

@@ -36,6 +36,17 @@ cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan,
                              const float* boundaries, int bits, int scale_mode, const float* cal_mu,
                              const float* cal_a, uint8_t* codes, float* scale, cudaStream_t s);
 
+// Query rotation on the tensor cores for batches of kRotTcMinBatch or more
+// (d as for the tensor-core encoder): q' = R q in TF32 with the three-product
+// split, the contraction split over rotate_tc_splits(nq, d) CTAs whose
+// partial products (part, rotate_tc_part_bytes bytes) are added in a fixed
+// order.  Clears the status word and zeroes `n_counters` merge counters.
+bool rotate_tc_applies(int64_t nq, int d);
+int rotate_tc_splits(int64_t nq, int d);
+size_t rotate_tc_part_bytes(int64_t nq, int d);
+cudaError_t launch_rotate_tc(const float* Q, int64_t nq, int d, const float* R, float* out, float* part,
+                             int* status, int* counters, int64_t n_counters, cudaStream_t s);
+
 // TQ+ calibration (Sec. II-B): per-coordinate shift mu and scale a from n
 // rows, into device [d] arrays; ws of calibrate_workspace(n, d) bytes.
 size_t calibrate_workspace(int64_t n, int d);
