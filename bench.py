@@ -504,9 +504,10 @@ def run_ours(args, cfg, rank, world):
             b.record(stream)
             b.synchronize()
         e2e_ms = a.elapsed_time(b)
-        # our kernels per step: rotation + lookup scan (merged in its last CTA),
-        # or rotation + query packing + tensor-core scan + merge; + shard merge
-        launches = (4 if mma else 2) + (1 if world > 1 else 0)
+        # our kernels per step: the rotation (with its reduce from 16 queries on:
+        # the tensor-core rotation), then the lookup scan (merged in its last
+        # CTA) or query packing + tensor-core scan + merge; + the shard merge
+        launches = (2 if B >= 16 else 1) + (3 if mma else 1) + (1 if world > 1 else 0)
         results[B] = {
             "value": qps, "ms_per_step": ms / args.steps, "roofline": roof, "clocks": clk.summary(),
             "gpu_launches": launches * args.steps,
