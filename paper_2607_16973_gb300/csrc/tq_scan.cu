@@ -253,12 +253,32 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
   const int nwarps = blockDim.x >> 5;
   const int total = nlists * k;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // 1. T = best k-th entry over the lists
+  const int cap = (int)min((size_t)8192, scratch_bytes / 8);
+  float* ss = reinterpret_cast<float*>(scratch);
+  int* si = reinterpret_cast<int*>(ss + cap);
+  // Two bounds on the global k-th best, the better one kept: T, the best
+  // k-th entry of any list (that list's k entries are at least as good), and
+  // the k-th best list head (the heads are k distinct candidates).  T is tight
+  // when the best entries crowd into a few lists, the head bound when they are
+  // spread over many.  The heads go to the scratch, loaded with the k-th
+  // entries in the same round trip.
+  const bool heads = nlists >= k && nlists <= min(cap, 512);
+  __shared__ float hb_s;
+  __shared__ int hb_i;
+  if (tid == 0) {
+    nsurv = 0;
+    hb_s = -INFINITY;  // no head bound (too few lists, or too many for one warp's registers)
+    hb_i = INT_MAX;
+  }
   float ts = -INFINITY;
   int ti = INT_MAX;
   for (int l = tid; l < nlists; l += blockDim.x) {
-    const float a = __ldcg(cs + l * k + k - 1);
-    const int b = __ldcg(ci + l * k + k - 1);
+    const float a = __ldcg(cs + (size_t)l * k + k - 1);
+    const int b = __ldcg(ci + (size_t)l * k + k - 1);
+    if (heads) {
+      ss[l] = __ldcg(cs + (size_t)l * k);
+      si[l] = __ldcg(ci + (size_t)l * k);
+    }
     if (better(a, b, ts, ti)) {
       ts = a;
       ti = b;
@@ -277,8 +297,35 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
     red_s[warp] = ts;
     red_i[warp] = ti;
   }
-  if (tid == 0) nsurv = 0;
   __syncthreads();
+  // the k-th best head score, by one warp: the heads' order-preserving
+  // integer keys sit in registers, and the key is found bit by bit from the
+  // top (the largest v with at least k keys >= v is the k-th largest key)
+  if (heads && warp == 0) {
+    uint32_t key[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const int l = lane + 32 * j;
+      uint32_t u = 0;  // below every score's key
+      if (l < nlists) {
+        const uint32_t b = __float_as_uint(ss[l]);
+        u = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+      }
+      key[j] = u;
+    }
+    uint32_t v = 0;
+    for (int bit = 31; bit >= 0; --bit) {
+      const uint32_t cand = v | (1u << bit);
+      int c = 0;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) c += key[j] >= cand ? 1 : 0;
+      if (__reduce_add_sync(FULL, c) >= k) v = cand;
+    }
+    if (lane == 0) {  // every candidate with that score or better passes: the id is the worst one
+      hb_s = __uint_as_float((v & 0x80000000u) ? (v & 0x7FFFFFFFu) : ~v);
+      hb_i = INT_MAX;
+    }
+  }
   ts = red_s[0];
   ti = red_i[0];
   for (int w = 1; w < nwarps; ++w)
@@ -286,10 +333,12 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
       ts = red_s[w];
       ti = red_i[w];
     }
-  // 2. gather the candidates at least as good as T (eight loads per thread in flight)
-  const int cap = (int)min((size_t)8192, scratch_bytes / 8);
-  float* ss = reinterpret_cast<float*>(scratch);
-  int* si = reinterpret_cast<int*>(ss + cap);
+  __syncthreads();  // the head bound is written; the gather below reuses the scratch
+  if (better(hb_s, hb_i, ts, ti)) {
+    ts = hb_s;
+    ti = hb_i;
+  }
+  // 2. gather the candidates at least as good as the bound (eight loads per thread in flight)
   for (int c0 = tid; c0 < total; c0 += 8 * blockDim.x) {
     float va[8];
     int vb[8];
@@ -312,6 +361,31 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
   }
   __syncthreads();
   const int nsv = nsurv;
+  if (nsv <= 32 && k <= 32) {  // 3a. few of them (the usual case): one warp sorts them with shuffles
+    if (warp == 0) {
+      float sv = lane < nsv ? ss[lane] : -INFINITY;
+      int iv = lane < nsv ? si[lane] : INT_MAX;
+#pragma unroll
+      for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          const float os = __shfl_xor_sync(FULL, sv, stride);
+          const int oi = __shfl_xor_sync(FULL, iv, stride);
+          // the lower lane of a pair keeps the better entry in a best-first run
+          const bool keep_better = ((lane & stride) == 0) == ((lane & size) == 0);
+          if (keep_better ? better(os, oi, sv, iv) : better(sv, iv, os, oi)) {
+            sv = os;
+            iv = oi;
+          }
+        }
+      if (lane < k) {
+        const bool empty = iv == INT_MAX;
+        out_ids[lane] = empty ? -1 : ext ? (int64_t)__ldg(ext + iv) : (int64_t)iv;
+        out_scores[lane] = empty ? -INFINITY : sv;
+      }
+    }
+    return;
+  }
   int P = 1;
   while (P < nsv || P < k) P <<= 1;
   if (P <= cap) {  // 3. sort them (the order is total: the result does not depend on the gathering order)
@@ -412,6 +486,51 @@ __device__ __forceinline__ void merge_if_last(const float* cand_s, const int* ca
   const size_t base = (size_t)q * gridDim.x * k;
   merge_lists_block(cand_s + base, cand_i + base, gridDim.x, k, ext, out_ids + (size_t)q * k,
                     out_scores + (size_t)q * k, ls, li, scratch, scratch_bytes);
+}
+
+// The CTA's top-k from its warps' sorted lists (warp w's k entries at w*k,
+// padded with (-inf, INT_MAX)), written to out.  With k <= 32, warp 0 merges
+// them: a list head per lane, k rounds of a warp argmax, the winning lane's
+// list advancing; otherwise the block sorts all P entries.
+__device__ __forceinline__ void cta_lists_out(float* ls, int* li, int nw, int k, int P, float* out_s, int* out_i) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  if (k <= 32 && nw <= 32) {
+    if (tid < 32) {
+      int pos = 0;
+      for (int r = 0; r < k; ++r) {
+        float bs = -INFINITY;
+        int bi = INT_MAX;
+        if (lane < nw && pos < k) {
+          bs = ls[lane * k + pos];
+          bi = li[lane * k + pos];
+        }
+        int bl = lane;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float os = __shfl_xor_sync(FULL, bs, o);
+          const int oi = __shfl_xor_sync(FULL, bi, o);
+          const int ol = __shfl_xor_sync(FULL, bl, o);
+          // identical (padding) entries: the lowest lane wins, so every lane agrees
+          if (better(os, oi, bs, bi) || (os == bs && oi == bi && ol < bl)) {
+            bs = os;
+            bi = oi;
+            bl = ol;
+          }
+        }
+        if (lane == 0) {
+          out_s[r] = bs;
+          out_i[r] = bi;
+        }
+        if (lane == bl) ++pos;
+      }
+    }
+    return;
+  }
+  block_sort(ls, li, P);
+  for (int i = tid; i < k; i += blockDim.x) {
+    out_s[i] = ls[i];
+    out_i[i] = li[i];
+  }
 }
 
 // Sums p[0..3] across the warp: afterwards lanes 8i..8i+7 hold the total of
@@ -753,11 +872,9 @@ k_scan_stream(const float* __restrict__ qrot, int d, const float* __restrict__ c
     st = st_next;
   }
   __syncthreads();
-  block_sort(ls, li, P);
-  for (int i = tid; i < k; i += SCAN_NT) {
-    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
-    cand_s[o] = ls[i];
-    cand_i[o] = li[i];
+  {
+    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k;
+    cta_lists_out(ls, li, SCAN_WARPS, k, P, cand_s + o, cand_i + o);
   }
   // the lookup table is dead by now: its bytes are the merge's scratch
   merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li, smem_raw, TAB_BYTES);
@@ -1025,11 +1142,9 @@ k_scan_ring(const float* __restrict__ qrot, int d, const float* __restrict__ cen
     for (int s = 0; s < ns; ++s)
       if ((pend >> s) & 1u) ring_wait_drain(wbar + s, (par >> s) & 1u);
   __syncthreads();
-  block_sort(ls, li, P);
-  for (int i = tid; i < k; i += RING_NT) {
-    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k + i;
-    cand_s[o] = ls[i];
-    cand_i[o] = li[i];
+  {
+    const size_t o = ((size_t)q * gridDim.x + blockIdx.x) * k;
+    cta_lists_out(ls, li, RING_WARPS, k, P, cand_s + o, cand_i + o);
   }
   // the lookup table is dead by now: its bytes are the merge's scratch
   merge_if_last(cand_s, cand_i, k, counters, ext, out_ids, out_scores, ls, li, smem_raw, TAB_BYTES);
