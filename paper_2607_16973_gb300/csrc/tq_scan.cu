@@ -226,6 +226,25 @@ __device__ __forceinline__ void load_q2(float2 (&q2)[S][8], const float* qq, int
   }
 }
 
+// Sorts one (score, id) pair per lane across the warp, best first (lane 0
+// the best): a bitonic network of shuffles.
+__device__ __forceinline__ void warp_sort32(float& sv, int& iv) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const float os = __shfl_xor_sync(FULL, sv, stride);
+      const int oi = __shfl_xor_sync(FULL, iv, stride);
+      // the lower lane of a pair keeps the better entry in a best-first run
+      const bool keep_better = ((lane & stride) == 0) == ((lane & size) == 0);
+      if (keep_better ? better(os, oi, sv, iv) : better(sv, iv, os, oi)) {
+        sv = os;
+        iv = oi;
+      }
+    }
+}
+
 // Merge of per-CTA candidate lists that are each sorted best first and hold
 // exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
 // any one list is beaten or matched by that list's k entries, so the global
@@ -298,32 +317,50 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
     red_i[warp] = ti;
   }
   __syncthreads();
-  // the k-th best head score, by one warp: the heads' order-preserving
-  // integer keys sit in registers, and the key is found bit by bit from the
-  // top (the largest v with at least k keys >= v is the k-th largest key)
   if (heads && warp == 0) {
-    uint32_t key[16];
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const int l = lane + 32 * j;
-      uint32_t u = 0;  // below every score's key
-      if (l < nlists) {
-        const uint32_t b = __float_as_uint(ss[l]);
-        u = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+    if (k <= 32) {
+      // the k-th best of the lanes' best heads (k distinct heads, so a valid
+      // bound; with ~10 heads a lane it is close to the k-th best head): one
+      // compare per head, then a shuffle sort of the 32 lane maxima
+      float bs = -INFINITY;
+      int bi = INT_MAX;
+      for (int l = lane; l < nlists; l += 32)
+        if (better(ss[l], si[l], bs, bi)) {
+          bs = ss[l];
+          bi = si[l];
+        }
+      warp_sort32(bs, bi);
+      if (lane == k - 1) {
+        hb_s = bs;
+        hb_i = bi;
       }
-      key[j] = u;
-    }
-    uint32_t v = 0;
-    for (int bit = 31; bit >= 0; --bit) {
-      const uint32_t cand = v | (1u << bit);
-      int c = 0;
+    } else {
+      // the k-th best head score exactly: the heads' order-preserving integer
+      // keys sit in registers and the key is found bit by bit from the top
+      // (the largest v with at least k keys >= v is the k-th largest key)
+      uint32_t key[16];
 #pragma unroll
-      for (int j = 0; j < 16; ++j) c += key[j] >= cand ? 1 : 0;
-      if (__reduce_add_sync(FULL, c) >= k) v = cand;
-    }
-    if (lane == 0) {  // every candidate with that score or better passes: the id is the worst one
-      hb_s = __uint_as_float((v & 0x80000000u) ? (v & 0x7FFFFFFFu) : ~v);
-      hb_i = INT_MAX;
+      for (int j = 0; j < 16; ++j) {
+        const int l = lane + 32 * j;
+        uint32_t u = 0;  // below every score's key
+        if (l < nlists) {
+          const uint32_t b = __float_as_uint(ss[l]);
+          u = (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+        }
+        key[j] = u;
+      }
+      uint32_t v = 0;
+      for (int bit = 31; bit >= 0; --bit) {
+        const uint32_t cand = v | (1u << bit);
+        int c = 0;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) c += key[j] >= cand ? 1 : 0;
+        if (__reduce_add_sync(FULL, c) >= k) v = cand;
+      }
+      if (lane == 0) {  // every candidate with that score or better passes: the id is the worst one
+        hb_s = __uint_as_float((v & 0x80000000u) ? (v & 0x7FFFFFFFu) : ~v);
+        hb_i = INT_MAX;
+      }
     }
   }
   ts = red_s[0];
@@ -365,19 +402,7 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
     if (warp == 0) {
       float sv = lane < nsv ? ss[lane] : -INFINITY;
       int iv = lane < nsv ? si[lane] : INT_MAX;
-#pragma unroll
-      for (int size = 2; size <= 32; size <<= 1)
-#pragma unroll
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-          const float os = __shfl_xor_sync(FULL, sv, stride);
-          const int oi = __shfl_xor_sync(FULL, iv, stride);
-          // the lower lane of a pair keeps the better entry in a best-first run
-          const bool keep_better = ((lane & stride) == 0) == ((lane & size) == 0);
-          if (keep_better ? better(os, oi, sv, iv) : better(sv, iv, os, oi)) {
-            sv = os;
-            iv = oi;
-          }
-        }
+      warp_sort32(sv, iv);
       if (lane < k) {
         const bool empty = iv == INT_MAX;
         out_ids[lane] = empty ? -1 : ext ? (int64_t)__ldg(ext + iv) : (int64_t)iv;
