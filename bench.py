@@ -263,6 +263,16 @@ def oracle_qps_sample(cfg, sample_rows: int, n_queries: int, seconds_cap: float 
         "per_query_s_sample": per_q_sample}
 
 
+def arm_config(args, n, d, bits, k, batch, world):
+    """The `config` object of the JSON line, the same for both arms."""
+    return {"workload": f"{args.config}: N={n} d={d} {bits}-bit top-{k}, batch {batch}, "
+                        f"codes {n * d * bits // 8 / 1e6:.1f} MB resident in HBM",
+            "n": n, "d": d, "bits": bits, "k": k, "batch": batch,
+            "l2": "inputs larger than L2 (corpus streamed from HBM every step)",
+            "parallelism": "single GPU" if world == 1 else
+            f"corpus sharded by rows over {world} GPUs ({n} rows each), all-gather of top-k + merge"}
+
+
 # -------------------------------------------------------------- reference --
 def run_reference(args, cfg, rank, world):
     if world > 1 and rank != 0:
@@ -296,8 +306,7 @@ def run_reference(args, cfg, rank, world):
                               "ms_per_full_query": per_step_full * 1e3},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": f"{args.config}: N={cfg['n']} d={d} {bits}-bit top-{k}, batch 1",
-                   "n": cfg["n"], "d": d, "bits": bits, "k": k, "batch": 1},
+        "config": arm_config(args, cfg["n"], d, bits, k, B, world),
         "cpu_baseline": {"value": qps, "unit": "queries/s", "cores": cores, "kind": "oracle", **cpu_model(),
                          "sample": f"each step: oracle search of 1 query over the first {sample_rows} "
                                    f"rows, time scaled by {cfg['n']}/{sample_rows}"},
@@ -562,12 +571,7 @@ def run_ours(args, cfg, rank, world):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms_per_step"],
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded Gaussian-mixture corpus, perturbed-corpus queries)",
-        "config": {"workload": f"{args.config}: N={n} d={d} {bits}-bit top-{k}, batch {head}, "
-                               f"codes {n * d * bits // 8 / 1e6:.1f} MB resident in HBM",
-                   "n": n, "d": d, "bits": bits, "k": k, "batch": head,
-                   "l2": "inputs larger than L2 (corpus streamed from HBM every step)",
-                   "parallelism": "single GPU" if world == 1 else
-                   f"corpus sharded by rows over {world} GPUs ({n} rows each), all-gather of top-k + merge"},
+        "config": arm_config(args, n, d, bits, k, head, world),
         "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
         "recall": recall,
         "rag_quality": rag,
@@ -1121,7 +1125,7 @@ def main():
     ap.add_argument("--k", type=int, default=None)
     ap.add_argument("--bits", type=int, default=None, choices=[2, 3, 4, 8],
                     help="code width for the scale/c2/tiny/prof workloads (default: 4)")
-    ap.add_argument("--ref-sample", type=int, default=100_000, help="corpus rows the oracle scans")
+    ap.add_argument("--ref-sample", type=int, default=50_000, help="corpus rows the oracle scans per step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true",
                     help="scale workload only: skip the 100K, filtered and bit-width sweep lines under 'extra'")
