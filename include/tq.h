@@ -305,18 +305,22 @@ tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float* R,
 /*
  * tq_search_host - tq_search_ex for queries and results in host memory: the
  * search() call of a serving process whose requests arrive in host memory.
- * Queues, on `stream`, the copy of the nq queries from Q_host to the device
- * staging buffer, the search, and the copies of the results to ids_host and
- * scores_host; returns without waiting (synchronise `stream` before reading
- * the results; page-locked host buffers keep the copies asynchronous).
+ * Queues, on `stream`, the query transfer, the search and the result
+ * transfer; returns without waiting (synchronise `stream` before reading the
+ * results).  Page-locked host buffers are used in place: the kernels read the
+ * queries (batches below 16, whose rotation runs on plain loads) and write
+ * the results (when both result buffers are page-locked) over the host link,
+ * with no copy operations; otherwise the queries and results are copied
+ * through the device staging buffer (asynchronously when page-locked).
  *   Q_host       host [nq*d] float32 queries
  *   ids_host     host out [nq*k] int64;  scores_host  host out [nq*k] float32
  *   staging      device scratch of staging_bytes >= tq_search_host_staging()
- *                (the device copies of the queries and results)
+ *                (the device copies of the queries and results, where used)
  *   the other arguments as for tq_search_ex (R, centroids, codes, scale,
  *   allow_off, allow_tenants, deleted, ext_ids, cal_mu, cal_a and workspace
  *   are device memory).
- * The host buffers must stay valid until the copies have run.
+ * The host buffers must stay valid, and the queries unchanged, until the
+ * search has run.
  */
 tq_status tq_search_host_staging(int64_t nq, int d, int k, size_t* bytes);
 tq_status tq_search_host(const float* Q_host, int64_t nq, int d, const float* R,

@@ -495,6 +495,20 @@ extern "C" tq_status tq_search_host_staging(int64_t nq, int d, int k, size_t* by
   return tq::ok();
 }
 
+namespace {
+// The device address of page-locked, mapped host memory (every page-locked
+// allocation is mapped under unified addressing), or nullptr for pageable
+// memory, which the kernels cannot reach.
+void* mapped_host(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();  // not sticky
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+}  // namespace
+
 extern "C" tq_status tq_search_host(const float* Q_host, int64_t nq, int d, const float* R,
                                     const float* centroids, int bits, const uint8_t* codes,
                                     const float* scale, int64_t n, const tq_filter* filter,
@@ -512,19 +526,35 @@ extern "C" tq_status tq_search_host(const float* Q_host, int64_t nq, int d, cons
   if (staging_bytes < h.total)
     return fail(TQ_EINVAL, "tq_search_host: staging of %zu bytes, %zu needed", staging_bytes, h.total);
   char* stg = static_cast<char*>(staging);
-  float* q_dev = reinterpret_cast<float*>(stg);
-  int64_t* ids_dev = reinterpret_cast<int64_t*>(stg + h.off_ids);
-  float* scores_dev = reinterpret_cast<float*>(stg + h.off_scores);
   cudaStream_t s = (cudaStream_t)stream;
-  cudaError_t e = cudaMemcpyAsync(q_dev, Q_host, (size_t)nq * d * sizeof(float), cudaMemcpyHostToDevice, s);
-  if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: query copy", e);
+  // Page-locked buffers are used in place: the query rotation reads the
+  // queries over the host link (when it runs on plain loads: batches the
+  // tensor-core rotation, fed by TMA from device memory, does not take), and
+  // the merge writes the results there; otherwise they go through `staging`.
+  const float* q_dev = tq::rotate_tc_applies(nq, d) ? nullptr : static_cast<const float*>(mapped_host(Q_host));
+  int64_t* ids_dev = static_cast<int64_t*>(mapped_host(ids_host));
+  float* scores_dev = static_cast<float*>(mapped_host(scores_host));
+  const bool out_in_place = ids_dev && scores_dev;
+  cudaError_t e = cudaSuccess;
+  if (!q_dev) {
+    float* q_stg = reinterpret_cast<float*>(stg);
+    e = cudaMemcpyAsync(q_stg, Q_host, (size_t)nq * d * sizeof(float), cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: query copy", e);
+    q_dev = q_stg;
+  }
+  if (!out_in_place) {
+    ids_dev = reinterpret_cast<int64_t*>(stg + h.off_ids);
+    scores_dev = reinterpret_cast<float*>(stg + h.off_scores);
+  }
   st = tq_search_ex(q_dev, nq, d, R, centroids, bits, codes, scale, n, filter, allow_off, allow_tenants, deleted,
                     ext_ids, cal_mu, cal_a, k, ids_dev, scores_dev, workspace, ws_bytes, stream);
   if (st != TQ_OK) return st;
-  e = cudaMemcpyAsync(ids_host, ids_dev, (size_t)nq * k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(scores_host, scores_dev, (size_t)nq * k * sizeof(float), cudaMemcpyDeviceToHost, s);
-  if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: result copy", e);
+  if (!out_in_place) {
+    e = cudaMemcpyAsync(ids_host, ids_dev, (size_t)nq * k * sizeof(int64_t), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(scores_host, scores_dev, (size_t)nq * k * sizeof(float), cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return tq::cuda_fail("tq_search_host: result copy", e);
+  }
   return tq::ok();
 }
 

@@ -491,15 +491,18 @@ def test_search_on_created_stream_matches_default_stream(cuda_lib, torch_dev, fi
     check_topk(want_i.cpu().numpy(), want_s.cpu().numpy(), ref.ids, ref.scores64, allowed, k, TOL_LUT)
 
 
-@pytest.mark.parametrize("filtered", [False, True])
-def test_search_host_buffers(cuda_lib, torch_dev, filtered_corpus, filtered):
-    """tq_search_host (queries from page-locked host memory, results back to
-    host memory, all queued by the library on one stream) returns what
-    tq_search on device buffers returns, bit for bit."""
+@pytest.mark.parametrize("filtered,nq,pinned", [(False, 7, True), (True, 7, True), (False, 7, False),
+                                                (False, 40, True), (True, 40, False)])
+def test_search_host_buffers(cuda_lib, torch_dev, filtered_corpus, filtered, nq, pinned):
+    """tq_search_host (queries from host memory, results back to host memory,
+    all queued by the library on one stream) returns what tq_search on device
+    buffers returns, bit for bit: page-locked buffers used in place (the
+    queries only below 16 per batch), pageable ones through the staging
+    copies."""
     torch, dev = torch_dev
     tq = cuda_lib
     c = filtered_corpus
-    nq, k = 7, 10
+    k = 10
     args = (_t(torch, dev, c["R"]), _t(torch, dev, c["c32"]), c["bits"], _t(torch, dev, c["enc"].packed),
             _t(torch, dev, c["enc"].scale), k)
     kw = {}
@@ -508,9 +511,10 @@ def test_search_host_buffers(cuda_lib, torch_dev, filtered_corpus, filtered):
         off, allow = synth.allowlists(c["src"][:nq], tid, values)
         kw = dict(filter=tq.Filter(_t(torch, dev, tid.view(np.int32))), allow_off=_t(torch, dev, off),
                   allow_tenants=_t(torch, dev, allow.view(np.int32)))
-    Qh = torch.from_numpy(c["Q"][:nq].copy()).pin_memory()
-    ih = torch.full((nq, k), 3, dtype=torch.int64).pin_memory()
-    sh = torch.full((nq, k), 3.0, dtype=torch.float32).pin_memory()
+    pin = (lambda t: t.pin_memory()) if pinned else (lambda t: t)
+    Qh = pin(torch.from_numpy(c["Q"][:nq].copy()))
+    ih = pin(torch.full((nq, k), 3, dtype=torch.int64))
+    sh = pin(torch.full((nq, k), 3.0, dtype=torch.float32))
     side = torch.cuda.Stream(device=dev)
     try:
         tq.search_from_host(Qh, *args, ih, sh, stream=side, **kw)
