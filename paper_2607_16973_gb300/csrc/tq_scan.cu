@@ -245,6 +245,88 @@ __device__ __forceinline__ void warp_sort32(float& sv, int& iv) {
     }
 }
 
+// merge_lists_block for k <= 32 and at most 16 candidates per thread: every
+// candidate comes to shared memory in one round trip of loads, both bounds
+// (see merge_lists_block) are taken there, and the survivors go to a 32-entry
+// buffer that one warp sorts.  Returns false (nothing written) when more than
+// 32 candidates survive, for the general path to redo the merge.
+__device__ bool merge_lists_small(const float* cs, const int* ci, int nlists, int k, const uint64_t* __restrict__ ext,
+                                  int64_t* out_ids, float* out_scores, float* ss, int* si) {
+  __shared__ float sv_s[32];
+  __shared__ int sv_i[32];
+  __shared__ float bs_s[2];
+  __shared__ int bs_i[2];
+  __shared__ int nsv;
+  const int total = nlists * k;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  {
+    float va[16];
+    int vb[16];
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const int c = tid + u * (int)blockDim.x;
+      va[u] = c < total ? __ldcg(cs + c) : 0.f;
+      vb[u] = c < total ? __ldcg(ci + c) : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < 16; ++u) {
+      const int c = tid + u * (int)blockDim.x;
+      if (c < total) {
+        ss[c] = va[u];
+        si[c] = vb[u];
+      }
+    }
+  }
+  if (tid == 0) nsv = 0;
+  __syncthreads();
+  if (warp < 2) {  // warp 0: T, the best k-th entry of a list; warp 1: the k-th best of the lanes' best heads
+    float bs = -INFINITY;
+    int bi = INT_MAX;
+    for (int l = lane; l < nlists; l += 32) {
+      const int c = l * k + (warp == 0 ? k - 1 : 0);
+      if (better(ss[c], si[c], bs, bi)) {
+        bs = ss[c];
+        bi = si[c];
+      }
+    }
+    warp_sort32(bs, bi);
+    const int pick = warp == 0 ? 0 : k - 1;
+    if (lane == pick) {
+      bs_s[warp] = bs;
+      bs_i[warp] = bi;
+    }
+  }
+  __syncthreads();
+  float ts = bs_s[0];
+  int ti = bs_i[0];
+  if (better(bs_s[1], bs_i[1], ts, ti)) {
+    ts = bs_s[1];
+    ti = bs_i[1];
+  }
+  for (int c = tid; c < total; c += blockDim.x)
+    if (si[c] != INT_MAX && !better(ts, ti, ss[c], si[c])) {
+      const int p = atomicAdd(&nsv, 1);
+      if (p < 32) {
+        sv_s[p] = ss[c];
+        sv_i[p] = si[c];
+      }
+    }
+  __syncthreads();
+  const int n_sv = nsv;
+  if (n_sv > 32) return false;  // every thread sees the same count
+  if (warp == 0) {
+    float sv = lane < n_sv ? sv_s[lane] : -INFINITY;
+    int iv = lane < n_sv ? sv_i[lane] : INT_MAX;
+    warp_sort32(sv, iv);
+    if (lane < k) {
+      const bool empty = iv == INT_MAX;
+      out_ids[lane] = empty ? -1 : ext ? (int64_t)__ldg(ext + iv) : (int64_t)iv;
+      out_scores[lane] = empty ? -INFINITY : sv;
+    }
+  }
+  return true;
+}
+
 // Merge of per-CTA candidate lists that are each sorted best first and hold
 // exactly k entries (padding (-inf, INT_MAX) at the end).  The k-th entry T of
 // any one list is beaten or matched by that list's k entries, so the global
@@ -275,6 +357,8 @@ __device__ void merge_lists_block(const float* cs, const int* ci, int nlists, in
   const int cap = (int)min((size_t)8192, scratch_bytes / 8);
   float* ss = reinterpret_cast<float*>(scratch);
   int* si = reinterpret_cast<int*>(ss + cap);
+  if (k <= 32 && nwarps >= 2 && total <= min(cap, 16 * (int)blockDim.x) && nlists >= k)
+    if (merge_lists_small(cs, ci, nlists, k, ext, out_ids, out_scores, ss, si)) return;
   // Two bounds on the global k-th best, the better one kept: T, the best
   // k-th entry of any list (that list's k entries are at least as good), and
   // the k-th best list head (the heads are k distinct candidates).  T is tight
@@ -502,9 +586,11 @@ __device__ __forceinline__ void merge_if_last(const float* cand_s, const int* ca
   const int q = blockIdx.y;
   __syncthreads();  // the CTA's list is written ...
   if (threadIdx.x == 0) {
-    __threadfence();  // ... and, through the barrier, released at GPU scope before the arrival
-    last = atomicAdd(counters + q, 1) == (int)gridDim.x - 1;
-    if (last) __threadfence();  // acquire every other CTA's list
+    // one acquire-release arrival: releases this CTA's list (through the
+    // barrier) and, for the last CTA, acquires every other CTA's
+    int prev;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(prev) : "l"(counters + q) : "memory");
+    last = prev == (int)gridDim.x - 1;
   }
   __syncthreads();
   if (!last) return;
