@@ -666,10 +666,16 @@ int rotate_tc_splits(int64_t nq, int d) {
   return (int)std::max<int64_t>(sp, 1);
 }
 
-bool rotate_tc_applies(int64_t nq, int d) { return nq >= kRotTcMinBatch && encode_tc_supported(d); }
+// (query tiles go on the grid's y dimension: at most 65535 of them)
+bool rotate_tc_applies(int64_t nq, int d) {
+  return nq >= kRotTcMinBatch && nq <= (int64_t)65535 * EM && encode_tc_supported(d);
+}
 
+// One split writes the rotated queries directly: no partial products.
 size_t rotate_tc_part_bytes(int64_t nq, int d) {
-  return rotate_tc_applies(nq, d) ? (size_t)rotate_tc_splits(nq, d) * nq * d * sizeof(float) : 0;
+  if (!rotate_tc_applies(nq, d)) return 0;
+  const int S = rotate_tc_splits(nq, d);
+  return S > 1 ? (size_t)S * nq * d * sizeof(float) : 0;
 }
 
 cudaError_t launch_rotate_tc(const float* Q, int64_t nq, int d, const float* R, float* out, float* part,
@@ -701,8 +707,11 @@ cudaError_t launch_rotate_tc(const float* Q, int64_t nq, int d, const float* R, 
   cudaError_t e = set_max_dynamic_smem(reinterpret_cast<const void*>(k_rotate_tc), (int)kRotSmem);
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((d + EN - 1) / EN), (unsigned)((nq + EM - 1) / EM), (unsigned)S);
-  k_rotate_tc<<<grid, ROT_THREADS, kRotSmem, s>>>(qmap, rmap, (int)nq, d, S, part, status);
+  k_rotate_tc<<<grid, ROT_THREADS, kRotSmem, s>>>(qmap, rmap, (int)nq, d, S, S > 1 ? part : out, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (S == 1)  // the products are the rotated queries; only the merge counters remain
+    return counters && n_counters > 0 ? cudaMemsetAsync(counters, 0, (size_t)n_counters * sizeof(int), s)
+                                      : cudaSuccess;
   const int64_t n4 = nq * d / 4;
   const int blocks = (int)std::min<int64_t>((n4 + 255) / 256, (int64_t)device_sm_count() * 8);
   k_rotate_reduce<<<std::max(blocks, 1), 256, 0, s>>>(reinterpret_cast<const float4*>(part), S, n4,

@@ -39,8 +39,9 @@ cudaError_t launch_encode_tc(const float* X, int64_t n, int d, const void* plan,
 // Query rotation on the tensor cores for batches of kRotTcMinBatch or more
 // (d as for the tensor-core encoder): q' = R q in TF32 with the three-product
 // split, the contraction split over rotate_tc_splits(nq, d) CTAs whose
-// partial products (part, rotate_tc_part_bytes bytes) are added in a fixed
-// order.  Clears the status word and zeroes `n_counters` merge counters.
+// partial products (part, rotate_tc_part_bytes bytes; none with one split,
+// which writes `out` directly) are added in a fixed order.  Clears the
+// status word and zeroes `n_counters` merge counters.
 bool rotate_tc_applies(int64_t nq, int d);
 int rotate_tc_splits(int64_t nq, int d);
 size_t rotate_tc_part_bytes(int64_t nq, int d);

@@ -386,6 +386,31 @@ def test_search_mma_parity(cuda_lib, torch_dev, bits, d, n, nq, k):
     check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k, TOL_MMA)
 
 
+@pytest.mark.parametrize("path,nq", [("lut", 40), ("mma", 3500)])
+def test_search_rotation_splits(cuda_lib, torch_dev, path, nq):
+    """The tensor-core query rotation (batches of 16 or more) with its
+    contraction split over several CTAs (40 queries: one query tile, many
+    splits, and the lookup scan's float32 tolerance) and with one split
+    writing the rotated queries directly (3,500 queries: 28 query tiles)."""
+    torch, dev = torch_dev
+    tq = cuda_lib
+    d, n, bits, k = 1536, 1200, 4, 10
+    packed = synth.random_codes(n, d * bits // 8, seed=nq)
+    scale = synth.random_scales(n, seed=nq + 1)
+    R = O.rotation(d, 13).astype(np.float32)
+    c32, _ = _cb(d, bits)
+    Q = synth.gaussian_rows(nq, d, seed=nq + 2)
+    Q /= np.linalg.norm(Q, axis=1, keepdims=True)
+    tq.set_search_path(path)
+    try:
+        ids, sc = _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k)
+    finally:
+        tq.set_search_path("auto")
+    ref = O.search(Q, R, c32, bits, packed, scale, k, d)
+    check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k,
+               TOL_LUT if path == "lut" else TOL_MMA)
+
+
 def test_search_mma_unsupported(cuda_lib, torch_dev):
     """Forcing the tensor-core scan where it does not apply is an error, not a
     silent switch: k > 64, d not a multiple of 64 (of 128 for 3-bit codes)."""
