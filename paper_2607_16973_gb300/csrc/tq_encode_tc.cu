@@ -10,23 +10,26 @@
 // which leaves a relative error of a few 2^-22 per product (the dropped
 // x_lo . r_lo term and the rounding of the low parts), the same order as an
 // fp32 FFMA dot product.  R is split once into a caller-owned plan
-// (tq_encode_plan); X is split in shared memory as its tiles arrive.
+// (tq_encode_plan); X is split as its tiles arrive.
 //
 // Work.  A CTA owns panels of 128 rows of X (the MMA's M) and walks the d
 // output coordinates in chunks of 256 (N), each chunk a full contraction over
 // K = d in K-blocks of 16 coordinates (64-byte rows of fp32 with the 64-byte
-// swizzle: 48 KB stages, four in flight, so the copy and the split of a
-// K-block are hidden behind the MMAs of the three before it).  Chunks walk the
-// K-blocks alternately forwards and backwards, so a chunk starts on the X
-// tiles the previous one read last (still in L2).
-// TMEM holds two 128 x 256 fp32 accumulator sets, so the epilogue of one
-// chunk overlaps the MMAs of the next.  Roles (14 warps):
-//   warps 0-3   converters: thread t owns row t of each X tile, splits it in
-//               place into x_hi and a separate x_lo tile, and sums x^2 over
-//               the first chunk's K-blocks (the row norm, step 1);
+// swizzle: five 40 KB shared-memory stages of the raw X tile and the R_hi and
+// R_lo tiles).  The split X tile goes to tensor memory and is the MMAs' A
+// operand there, so the tensor cores read only the R tiles from shared
+// memory; TMEM holds one 128 x 256 fp32 accumulator and the five stages' x_hi
+// and x_lo (32 columns each).  Chunks walk the K-blocks alternately forwards
+// and backwards, so a chunk starts on the X tiles the previous one read last
+// (still in L2).  Roles (14 warps):
+//   warps 0-3   converters: thread t owns row t of each X tile, splits it into
+//               x_hi and x_lo and stores both to its TMEM lane (tcgen05.st),
+//               and sums x^2 over the first chunk's K-blocks (the row norm,
+//               step 1);
 //   warp 4      producer: TMA of the X tile and the R_hi / R_lo tiles;
 //   warp 5      MMA issuer: allocates TMEM; one thread issues the three
-//               tcgen05.mma products per K-step (M=128, N=256, K=8);
+//               tcgen05.mma products per K-step (M=128, N=256, K=8; A in
+//               TMEM, B in shared memory);
 //   warps 6-13  epilogue: warp w reads TMEM lanes 32 (w % 4) .. + 31 (one row
 //               per thread), columns 0-127 (warps 6-9) or 128-255 (10-13) of
 //               the chunk: y = acc / ||x|| (step 2), the code by boundary
@@ -55,7 +58,13 @@ constexpr int EK = 16;                      // coordinates per K-block (64 B of 
 constexpr int NSTAGE = 4;                   // K-block stages in flight
 constexpr int X_BYTES = EM * EK * 4;        // 8 KB: an X tile (x_hi after the split)
 constexpr int R_BYTES = EN * EK * 4;        // 16 KB: an R_hi or R_lo tile
-constexpr int STAGE_BYTES = 2 * X_BYTES + 2 * R_BYTES;  // x_hi, x_lo, r_hi, r_lo
+constexpr int STAGE_BYTES = 2 * X_BYTES + 2 * R_BYTES;  // x_hi, x_lo, r_hi, r_lo (the rotation kernel)
+// The encoder keeps the split X tile in tensor memory: a stage in shared
+// memory is the raw X tile and the R_hi, R_lo tiles.
+constexpr int ENC_NSTAGE = 5;
+constexpr int ENC_STAGE_BYTES = X_BYTES + 2 * R_BYTES;  // 40 KB
+constexpr uint32_t TM_A = EN;              // TMEM column of the first stage's x_hi (the accumulator is 0 .. EN-1)
+constexpr uint32_t TM_A_STAGE = 2 * EK;    // columns per stage: x_hi, then x_lo
 constexpr int CONV_WARPS = 4, PROD_WARP = 4, MMA_WARP = 5, EPI_WARP0 = 6, EPI_WARPS = 8;
 constexpr int ENC_THREADS = (EPI_WARP0 + EPI_WARPS) * 32;  // 448
 constexpr int EPI_THREADS = EPI_WARPS * 32;
@@ -66,16 +75,16 @@ constexpr size_t kPlanHeader = 256;
 
 // Offsets in the 1024-byte-aligned dynamic shared memory.
 struct EncSmem {
-  // stage s at s * STAGE_BYTES: x_hi, x_lo, r_hi, r_lo tiles
+  // stage s at s * ENC_STAGE_BYTES: x, r_hi, r_lo tiles
   // boundaries and centroids: with codes of up to 4 bits one copy per bank
   // ([entry][32]), so the epilogue's data-dependent lookups never conflict
-  static constexpr uint32_t bnd = NSTAGE * STAGE_BYTES;  // [512] floats
+  static constexpr uint32_t bnd = ENC_NSTAGE * ENC_STAGE_BYTES;  // [512] floats
   static constexpr uint32_t cen = bnd + 512 * 4;         // [512] floats
   static constexpr uint32_t nrm = cen + 512 * 4;         // [2][128] row norms by panel parity
   static constexpr uint32_t inv = nrm + 2 * EM * 4;      // [2][128] 1 / norm
   static constexpr uint32_t part = inv + 2 * EM * 4;     // [2][2][128] double: sum c^2, sum y c of the column-128..255 warps
   static constexpr uint32_t bars = part + 4 * EM * 8;    // mbarriers
-  static constexpr uint32_t nbars = 24;
+  static constexpr uint32_t nbars = 28;
   static constexpr uint32_t misc = bars + nbars * 8;     // TMEM address, abort flag
   static constexpr uint32_t total = misc + 16;
 };
@@ -92,6 +101,24 @@ __device__ __forceinline__ void mma_tf32(uint32_t d_tmem, uint64_t a, uint64_t b
       "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
       " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}"
       ::"r"(d_tmem), "l"(a), "l"(b), "r"(idesc_tf32()), "r"(accumulate));
+}
+
+// The same with A in tensor memory (M lanes, K columns of 32-bit values).
+__device__ __forceinline__ void mma_tf32_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}"
+      ::"r"(d_tmem), "r"(a_tmem), "l"(b), "r"(idesc_tf32()), "r"(accumulate));
+}
+
+// Stores 16 consecutive TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};"
+      ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
 }
 
 // v rounded to the nearest TF32 value (10 explicit mantissa bits; ties away
@@ -133,15 +160,15 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
   float* sInv = reinterpret_cast<float*>(base + EncSmem::inv);
   double* sPart = reinterpret_cast<double*>(base + EncSmem::part);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + EncSmem::bars);
-  uint64_t* full = bars;             // [NSTAGE] X and R tiles landed
-  uint64_t* conv = bars + 4;         // [NSTAGE] X tile split
-  uint64_t* empty = bars + 8;        // [NSTAGE] MMAs done with the stage
-  uint64_t* acc_full = bars + 12;    // [2] accumulator set complete
-  uint64_t* acc_empty = bars + 14;   // [2] accumulator set read out
-  uint64_t* norm_ready = bars + 16;  // [2] row norms of a panel written (by panel parity)
-  uint64_t* norm_free = bars + 18;   // [2] row norms of a panel read
-  uint64_t* part_ready = bars + 20;  // [2] column-128..255 sums of a panel written
-  uint64_t* fin = bars + 22;         // every MMA of this CTA complete
+  uint64_t* full = bars;             // [ENC_NSTAGE] X and R tiles landed
+  uint64_t* conv = bars + 5;         // [ENC_NSTAGE] X tile split into tensor memory
+  uint64_t* empty = bars + 10;       // [ENC_NSTAGE] MMAs done with the stage
+  uint64_t* acc_full = bars + 15;    // the accumulator complete
+  uint64_t* acc_empty = bars + 16;   // the accumulator read out
+  uint64_t* norm_ready = bars + 18;  // [2] row norms of a panel written (by panel parity)
+  uint64_t* norm_free = bars + 20;   // [2] row norms of a panel read
+  uint64_t* part_ready = bars + 22;  // [2] column-128..255 sums of a panel written
+  uint64_t* fin = bars + 24;         // every MMA of this CTA complete
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(base + EncSmem::misc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(base + EncSmem::misc + 4);
 
@@ -158,14 +185,14 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     sBnd[i] = e < L - 1 ? boundaries[e] : INFINITY;
   }
   if (tid == 0) {
-    for (int s = 0; s < NSTAGE; ++s) {
+    for (int s = 0; s < ENC_NSTAGE; ++s) {
       mbar_init(full + s, 1);
       mbar_init(conv + s, CONV_WARPS);
       mbar_init(empty + s, 1);
     }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, EPI_WARPS);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(acc_full + b, 1);
-      mbar_init(acc_empty + b, EPI_WARPS);
       mbar_init(norm_ready + b, CONV_WARPS * 32);  // every converter thread, after its row
       mbar_init(norm_free + b, EPI_WARPS);
       mbar_init(part_ready + b, EPI_THREADS / 2);  // every column-128..255 thread, after its row
@@ -188,54 +215,50 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     if (lane == 0) {
       long long issued = 0;
       for (long long it = 0; it < total_it; ++it) {
-        const int s = (int)(it % NSTAGE);
-        const long long use = it / NSTAGE;
+        const int s = (int)(it % ENC_NSTAGE);
+        const long long use = it / ENC_NSTAGE;
         if (use > 0 && !mbar_wait(empty + s, (uint32_t)((use - 1) & 1), abort_flag, err, 41)) break;
         const int kb = (int)(it % KB);
         const long long cs = it / KB;
         const int c = (int)(cs % C), i = (int)(cs / C);
         const int panel = (int)blockIdx.x + i * (int)gridDim.x;
         const int kc = (c & 1) ? KB - 1 - kb : kb;  // snake order over the K-blocks
-        unsigned char* st = base + s * STAGE_BYTES;
+        unsigned char* st = base + s * ENC_STAGE_BYTES;
         mbar_arrive_expect_tx(full + s, X_BYTES + 2 * R_BYTES);
         tma_load_2d(st, &xmap, kc * EK, panel * EM, full + s);
         // rows c*256 .. of R_hi, then of R_lo (rows d .. 2d-1 of the plan); in a
         // partial last chunk the rows past d are R_lo rows or zero fill, and the
         // epilogue never reads their columns
-        tma_load_2d(st + 2 * X_BYTES, &rmap, kc * EK, c * EN, full + s);
-        tma_load_2d(st + 2 * X_BYTES + R_BYTES, &rmap, kc * EK, d + c * EN, full + s);
+        tma_load_2d(st + X_BYTES, &rmap, kc * EK, c * EN, full + s);
+        tma_load_2d(st + X_BYTES + R_BYTES, &rmap, kc * EK, d + c * EN, full + s);
         issued = it + 1;
       }
       // never leave with copies in flight: wait (bounded) for the last one of each stage
-      for (int s = 0; s < NSTAGE && s < issued; ++s)
-        mbar_wait_drain(full + s, (uint32_t)(((issued - 1 - s) / NSTAGE) & 1));
+      for (int s = 0; s < ENC_NSTAGE && s < issued; ++s)
+        mbar_wait_drain(full + s, (uint32_t)(((issued - 1 - s) / ENC_NSTAGE) & 1));
     }
   } else if (warp == MMA_WARP) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       for (long long it = 0; it < total_it; ++it) {
-        const int s = (int)(it % NSTAGE);
-        const long long use = it / NSTAGE;
+        const int s = (int)(it % ENC_NSTAGE);
+        const long long use = it / ENC_NSTAGE;
         const int kb = (int)(it % KB);
         const long long cs = it / KB;
-        const int set = (int)(cs & 1);
-        if (kb == 0 && cs >= 2 &&
-            !mbar_wait(acc_empty + set, (uint32_t)(((cs >> 1) - 1) & 1), abort_flag, err, 42))
-          break;
+        if (kb == 0 && cs >= 1 && !mbar_wait(acc_empty, (uint32_t)((cs - 1) & 1), abort_flag, err, 42)) break;
         if (!mbar_wait(conv + s, (uint32_t)(use & 1), abort_flag, err, 43)) break;
         tc_fence_after();
-        const uint32_t xh = smem_u32(base + s * STAGE_BYTES);
-        const uint32_t xl = xh + X_BYTES, rh = xh + 2 * X_BYTES, rl = rh + R_BYTES;
-        const uint32_t dt = tmem + (uint32_t)(set * EN);
+        const uint32_t rh = smem_u32(base + s * ENC_STAGE_BYTES) + X_BYTES, rl = rh + R_BYTES;
+        const uint32_t ah = tmem + TM_A + (uint32_t)s * TM_A_STAGE, al = ah + EK;
 #pragma unroll
-        for (int kk = 0; kk < EK / 8; ++kk) {  // K = 8 TF32 values = 32 bytes of each row
-          const uint32_t o = (uint32_t)kk * 32u;
-          mma_tf32(dt, sw64_desc(xh + o), sw64_desc(rh + o), (kb | kk) != 0);
-          mma_tf32(dt, sw64_desc(xh + o), sw64_desc(rl + o), 1u);
-          mma_tf32(dt, sw64_desc(xl + o), sw64_desc(rh + o), 1u);
+        for (int kk = 0; kk < EK / 8; ++kk) {  // K = 8 TF32 values: 32 bytes of each R row, 8 TMEM columns of x
+          const uint32_t o = (uint32_t)kk * 32u, oa = (uint32_t)kk * 8u;
+          mma_tf32_ta(tmem, ah + oa, sw64_desc(rh + o), (kb | kk) != 0);
+          mma_tf32_ta(tmem, ah + oa, sw64_desc(rl + o), 1u);
+          mma_tf32_ta(tmem, al + oa, sw64_desc(rh + o), 1u);
         }
         mma_commit(empty + s);
-        if (kb == KB - 1) mma_commit(acc_full + set);
+        if (kb == KB - 1) mma_commit(acc_full);
       }
       mma_commit(fin);
       mbar_wait_drain(fin, 0);
@@ -251,15 +274,15 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     const int t = tid;
     double ss = 0.0;
     for (long long it = 0; it < total_it; ++it) {
-      const int s = (int)(it % NSTAGE);
-      const long long use = it / NSTAGE;
+      const int s = (int)(it % ENC_NSTAGE);
+      const long long use = it / ENC_NSTAGE;
       const int kb = (int)(it % KB);
       const long long cs = it / KB;
       const int c = (int)(cs % C), i = (int)(cs / C);
       if (!warp_wait(full + s, (uint32_t)(use & 1), abort_flag, err, 44)) break;
-      unsigned char* xt = base + s * STAGE_BYTES;
-      unsigned char* xlo = xt + X_BYTES;
+      const unsigned char* xt = base + s * ENC_STAGE_BYTES;
       float p0 = 0.f, p1 = 0.f, p2 = 0.f, p3 = 0.f;
+      uint32_t hv[EK], lv[EK];  // row t's x_hi and x_lo, in K order
 #pragma unroll
       for (int q = 0; q < EK / 4; ++q) {
         const uint32_t off = (uint32_t)t * 64u + ((uint32_t)(q ^ ((t >> 1) & 3)) << 4);
@@ -268,13 +291,20 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         p1 = fmaf(v.y, v.y, p1);
         p2 = fmaf(v.z, v.z, p2);
         p3 = fmaf(v.w, v.w, p3);
-        const float4 h = make_float4(tf32_round(v.x), tf32_round(v.y), tf32_round(v.z), tf32_round(v.w));
-        const float4 l = make_float4(tf32_round(v.x - h.x), tf32_round(v.y - h.y), tf32_round(v.z - h.z),
-                                     tf32_round(v.w - h.w));
-        *reinterpret_cast<float4*>(xt + off) = h;
-        *reinterpret_cast<float4*>(xlo + off) = l;
+        const float vv[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const float hi = tf32_round(vv[u]);
+          hv[4 * q + u] = __float_as_uint(hi);
+          lv[4 * q + u] = __float_as_uint(tf32_round(vv[u] - hi));
+        }
       }
-      fence_proxy_async();  // make this thread's writes visible to the tensor core
+      // lane quarter = this warp (warps 0-3), column = K index
+      const uint32_t ta = tmem + ((uint32_t)(warp * 32) << 16) + TM_A + (uint32_t)s * TM_A_STAGE;
+      tmem_st16(ta, hv);
+      tmem_st16(ta + EK, lv);
+      asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(conv + s);
       if (c == 0) ss += (double)((p0 + p1) + (p2 + p3));
@@ -344,7 +374,7 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
     };
     const long long nchunks = (long long)my_panels * C;
     for (long long cs = 0; cs < nchunks; ++cs) {
-      const int c = (int)(cs % C), i = (int)(cs / C), set = (int)(cs & 1);
+      const int c = (int)(cs % C), i = (int)(cs / C);
       const int pp = i & 1;
       if (c == 0) {
         if (!warp_wait(norm_ready + pp, (uint32_t)((i >> 1) & 1), abort_flag, err, 46)) break;
@@ -356,9 +386,9 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         yc = 0.0;
         grow = (int64_t)((int)blockIdx.x + i * (int)gridDim.x) * EM + row;
       }
-      if (!warp_wait(acc_full + set, (uint32_t)((cs >> 1) & 1), abort_flag, err, 47)) break;
+      if (!warp_wait(acc_full, (uint32_t)(cs & 1), abort_flag, err, 47)) break;
       tc_fence_after();
-      const uint32_t ta = tl + (uint32_t)(set * EN);
+      const uint32_t ta = tl;
       const int jb = c * EN + h * (EN / 2);
       uint32_t ra[16], rb[16];
       tmem_ld16_issue(ta, ra);
@@ -406,7 +436,7 @@ k_encode_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CU
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty + set);
+      if (lane == 0) mbar_arrive(acc_empty);
       if (!ok) break;
     }
   }
