@@ -100,6 +100,13 @@ def source_hash(*files):
     return h.hexdigest()[:16]
 
 
+def lookup_kernel(bits: int, n: int, d: int, k: int) -> str:
+    """The lookup scan tq_search's AUTO path runs below the tensor-core batch
+    size: the bulk-copy ring for 3-bit codes, else the register-fed byte-pair
+    (4-bit) or per-code scan."""
+    return "k_scan_ring" if bits == 3 else "k_scan_stream"
+
+
 def recorded_traffic(kernel_file: str, profile_md: str, scale_to: int):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current kernel source (the summary records the source hash).  The
@@ -475,12 +482,15 @@ def run_ours(args, cfg, rank, world):
             # lookup scan (with its last CTA's merge): the corpus, codes + scales,
             # read once per launch
             achieved = alg_bytes / (scan_ms / 1e3) / 1e9
+            kern = lookup_kernel(bits, n, d, k)
+            if kern == "k_scan_stream" and bits == 4:
+                traffic = recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu", "k_scan_stream_250k_batch1.md",
+                                           scale_to=n)
+            else:
+                traffic = None
             roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                    "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"],
-                    "traffic": recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu",
-                                                "k_scan_stream_250k_batch1.md", scale_to=n)
-                    if bits == 4 else None,
-                    "kernel": "k_scan_stream" if bits != 3 else "k_scan_ring", "alg_bytes_per_launch": alg_bytes,
+                    "frac": achieved / pk["hbm_gbs"], "frac_of": pk["source"], "traffic": traffic,
+                    "kernel": kern, "alg_bytes_per_launch": alg_bytes,
                     "kernel_ms": scan_ms, "frac_of_8tbs_nominal": achieved / 8000.0}
         # e2e through the C ABI with host buffers: tq_search_host queues the
         # query upload, the search and the result download on `stream`

@@ -12,7 +12,7 @@ STATUS_NAMES = {0: "TQ_OK", 1: "TQ_EINVAL", 2: "TQ_ENOMEM", 3: "TQ_ECUDA", 4: "T
                 5: "TQ_EUNSUPPORTED"}
 MARGINALS = {"beta": 0, "gauss": 1}
 SCALE_MODES = {"norm": 0, "none": 1, "unbiased": 2}
-PATHS = {"auto": 0, "lut": 1, "mma": 2, "lut_fixed": 3}
+PATHS = {"auto": 0, "lut": 1, "mma": 2, "lut_fixed": 3, "lut_fold": 4}
 
 # name -> (restype, argtypes); every symbol include/tq.h declares
 SIGNATURES = {

@@ -30,7 +30,7 @@ constexpr size_t kAlign = 256;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
 struct SearchPlan {
-  int grid_lut = 1, grid_mma = 0;
+  int grid_lut = 1, grid_mma = 0, grid_fold = 0;
   size_t off_status = 0, off_cnt = 0, off_bias = 0, off_rot = 0, off_part = 0, off_allow = 0, off_mask = 0,
          off_qpack = 0, off_cs = 0, off_ci = 0, total = 0;
   bool rot_tc = false;  // the query rotation runs on the tensor cores
@@ -45,7 +45,8 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
   const bool mma = mma_supported(bits, d, k);
   p.grid_mma = mma ? scan_mma_grid_x(nq, n, k, bits) : 0;
-  const int per_query = std::max(p.grid_lut, p.grid_mma) * k;
+  p.grid_fold = fold_supported(bits, d, k) ? scan_fold_grid_x(nq, n) : 0;
+  const int per_query = std::max(std::max(p.grid_lut, p.grid_mma), p.grid_fold) * k;
   size_t off = 0;
   p.off_status = off;
   off = align_up(off + sizeof(int));
@@ -423,6 +424,13 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
     return fail(TQ_EUNSUPPORTED, "tq_search: the tensor-core scan needs bits 2/4/8, d %% 64 == 0 and k <= %d",
                 tq::kMaxKMma);
   const bool use_mma = can_mma && (path == TQ_PATH_MMA || (path == TQ_PATH_AUTO && nq >= tq::kMmaMinBatch));
+  const bool can_fold = tq::fold_supported(bits, d, k);
+  if (path == TQ_PATH_LUT_FOLD && !can_fold)
+    return fail(TQ_EUNSUPPORTED, "tq_search: the query-folded scan needs bits 4, d >= 256 and k <= %d",
+                tq::kFoldMaxK);
+  // AUTO keeps the byte-pair scan: on GB300 it is the faster of the two (218
+  // against 228 us per query at 999,000 x 1536)
+  const bool use_fold = !use_mma && can_fold && path == TQ_PATH_LUT_FOLD;
   const tq::SearchPlan p = tq::plan_search(nq, n, d, bits, k, filter);
   if (ws_bytes < p.total)
     return fail(TQ_EINVAL, "tq_search: workspace of %zu bytes, %zu needed", ws_bytes, p.total);
@@ -452,7 +460,12 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
   } else {
     if (e == cudaSuccess && filter) e = tq::launch_allow_bits(filter->f, allow_off, allow_tenants, nq, allow, s);
     if (e == cudaSuccess && filter) e = tq::launch_block_mask(filter->f, allow, nq, bmask, s);
-    if (e == cudaSuccess)
+    if (e == cudaSuccess && use_fold)
+      e = tq::launch_scan_fold(qrot, nq, d, centroids, codes, scale, n, deleted, filter ? &filter->f : nullptr,
+                               allow, bmask, k, p.grid_fold, cs, ci, status, counters, ext_ids, out_ids,
+                               out_scores, bias, s, (cudaEvent_t)tq::profile_start(),
+                               (cudaEvent_t)tq::profile_stop());
+    else if (e == cudaSuccess)
       e = tq::launch_scan_lut(qrot, nq, d, centroids, bits, codes, scale, n, deleted,
                               filter ? &filter->f : nullptr, allow, bmask,
                               path == TQ_PATH_LUT_FIXED && d >= tq::kFixMinD,

@@ -252,7 +252,8 @@ extern "C" const char* tq_last_error(void) { return tq::g_error.c_str(); }
 extern "C" int tq_version(void) { return 100; }
 
 extern "C" tq_status tq_set_search_path(int path) {
-  if (path != TQ_PATH_AUTO && path != TQ_PATH_LUT && path != TQ_PATH_MMA && path != TQ_PATH_LUT_FIXED)
+  if (path != TQ_PATH_AUTO && path != TQ_PATH_LUT && path != TQ_PATH_MMA && path != TQ_PATH_LUT_FIXED &&
+      path != TQ_PATH_LUT_FOLD)
     return tq::fail(TQ_EINVAL, "tq_set_search_path: unknown path %d", path);
   tq::g_path = path;
   return tq::ok();

@@ -29,6 +29,8 @@ constexpr int kRotTcMinBatch = 16;  // query batches rotated on the tensor cores
 // sqrt(d)), so below it the exact fp32 table keeps unit-query scores within
 // 1e-5.
 constexpr int kFixMinD = 512;
+// The query-folded 4-bit lookup scan (k_scan_fold, TQ_PATH_LUT_FOLD): largest k.
+constexpr int kFoldMaxK = 32;
 constexpr long long kWaitCyclesMax = 4000000000LL;  // the kernels' wait budget (~2 s at 2 GHz)
 
 // Thread-local count of device allocations still to fail (tq_debug_fail_allocs).

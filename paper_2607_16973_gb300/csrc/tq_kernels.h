@@ -93,6 +93,19 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
                             const uint64_t* ext, int64_t* out_ids, float* out_scores, const float* bias,
                             cudaStream_t s, cudaEvent_t ev0, cudaEvent_t ev1);
 
+// The 4-bit lookup scan with the rotated query folded into per-byte-position
+// tables (k_scan_fold): bits 4, d >= 256 and a multiple of 32, k <= kFoldMaxK,
+// codes 16-byte aligned.  Arguments and results as launch_scan_lut; grid_x
+// from scan_fold_grid_x.
+bool fold_supported(int bits, int d, int k);
+int scan_fold_grid_x(int64_t nq, int64_t n);
+cudaError_t launch_scan_fold(const float* qrot, int64_t nq, int d, const float* centroids, const uint8_t* codes,
+                             const float* scale, int64_t n, const uint32_t* del, const FilterDev* f,
+                             const uint32_t* allow_bits, const uint32_t* bmask, int k, int grid_x, float* cand_s,
+                             int32_t* cand_i, int* err, int* counters, const uint64_t* ext, int64_t* out_ids,
+                             float* out_scores, const float* bias, cudaStream_t s, cudaEvent_t ev0,
+                             cudaEvent_t ev1);
+
 // Per-query bitmap over the filter's blocks: bit b set when block b holds a
 // tenant the query allows.  out [nq * filter_mask_words(f)].
 int filter_mask_words(const FilterDev& f);

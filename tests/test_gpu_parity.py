@@ -105,7 +105,7 @@ def _gpu_search(tq, torch, dev, Q, R, c32, bits, packed, scale, k, **kw):
     return ids.cpu().numpy(), sc.cpu().numpy()
 
 
-@pytest.mark.parametrize("path", ["lut", "lut_fixed", "mma"])
+@pytest.mark.parametrize("path", ["lut", "lut_fixed", "lut_fold", "mma"])
 def test_search_tiny_config(cuda_lib, torch_dev, tiny_config, path):
     torch, dev = torch_dev
     tq = cuda_lib
@@ -255,9 +255,11 @@ def filtered_corpus():
 
 @pytest.mark.parametrize("T", [10, 100, 1000])
 @pytest.mark.parametrize("block", [64, 32])
-def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
+@pytest.mark.parametrize("path", ["lut", "lut_fold"])
+def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block, path):
     """Zipf(1.1) tenants in interleaved order; 1 allowed tenant per query, 10%
-    of queries with 5 (Sec. III-B, the filtered workload)."""
+    of queries with 5 (Sec. III-B, the filtered workload).  The query-folded
+    scan runs one CTA per query here: four passes of 6,656 rows each."""
     torch, dev = torch_dev
     tq = cuda_lib
     c = filtered_corpus
@@ -266,7 +268,7 @@ def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
     off, allow = synth.allowlists(c["src"], tid, values)
     filt = tq.Filter(_t(torch, dev, tid.view(np.int32)), block=block)
     assert filt.info() == {"n": c["n"], "block": block, "n_tenants": T}
-    tq.set_search_path("lut")  # the lookup scan (a batch of 200 would take the tensor-core scan)
+    tq.set_search_path(path)  # a lookup scan (a batch of 200 would take the tensor-core scan)
     try:
         ids, sc = _gpu_search(tq, torch, dev, c["Q"], c["R"], c["c32"], c["bits"], c["enc"].packed,
                               c["enc"].scale, k, filter=filt, allow_off=_t(torch, dev, off),
@@ -282,10 +284,10 @@ def test_filtered_search(cuda_lib, torch_dev, filtered_corpus, T, block):
     filt.close()
 
 
-@pytest.mark.parametrize("path", ["lut", "lut_fixed"])
+@pytest.mark.parametrize("path", ["lut", "lut_fixed", "lut_fold"])
 def test_filter_every_tenant_equals_unfiltered(cuda_lib, torch_dev, filtered_corpus, path):
-    """At d = 1536, with both 4-bit tables: allowing every tenant gives the
-    unfiltered search bit for bit (the same operations on every score)."""
+    """At d = 1536, with each 4-bit lookup scan: allowing every tenant gives
+    the unfiltered search bit for bit (the same operations on every score)."""
     torch, dev = torch_dev
     tq = cuda_lib
     c = filtered_corpus

@@ -96,7 +96,7 @@ def tqp_corpus(tdev):
     return dict(X=X, R=R, c32=c32, cal=cal, enc=enc, src=src, Q=Q, d=d, n=n, bits=bits)
 
 
-@pytest.mark.parametrize("path,nq", [("lut", 5), ("mma", 60)])
+@pytest.mark.parametrize("path,nq", [("lut", 5), ("lut_fold", 5), ("mma", 60)])
 def test_search_tqplus_parity(cuda_lib, tdev, tqp_corpus, path, nq):
     """Calibrated search: the lookup scan and the tensor-core scan add the
     query's term sum_j q'_j mu_j to every raw score before the per-vector
@@ -117,7 +117,7 @@ def test_search_tqplus_parity(cuda_lib, tdev, tqp_corpus, path, nq):
     ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
     ref = O.search(c["Q"][:nq], c["R"], c["c32"], c["bits"], c["enc"].packed, c["enc"].scale, k, c["d"], calib=cal)
     check_topk(ids, sc, ref.ids, ref.scores64, np.ones_like(ref.scores64, bool), k,
-               TOL_LUT if path == "lut" else TOL_MMA)
+               TOL_LUT if path.startswith("lut") else TOL_MMA)
     exact, _ = O.exact_knn(c["X"], c["Q"][:nq], k)
     assert abs(recall(ids, exact) - recall(ref.ids, exact)) <= 0.002
 
