@@ -107,7 +107,7 @@ def lookup_kernel(bits: int, n: int, d: int, k: int) -> str:
     return "k_scan_ring" if bits == 3 else "k_scan_stream"
 
 
-def recorded_traffic(kernel_file: str, profile_md: str, scale_to: int):
+def recorded_traffic(kernel_file, profile_md: str, scale_to: int):
     """DRAM bytes per launch from a committed ncu summary, if it was taken on
     the current kernel source (the summary records the source hash).  The
     summary is captured on a smaller corpus of `captured_n` vectors; traffic
@@ -115,7 +115,7 @@ def recorded_traffic(kernel_file: str, profile_md: str, scale_to: int):
     path = os.path.join(ROOT, "profiles", profile_md)
     if not os.path.exists(path):
         return None
-    want = source_hash(kernel_file)
+    want = source_hash(*((kernel_file,) if isinstance(kernel_file, str) else kernel_file))
     got_hash, traffic, cap_n = None, None, None
     with open(path) as f:
         for line in f:
@@ -412,6 +412,7 @@ def run_ours(args, cfg, rank, world):
     except Exception:
         pci = None
     results = {}
+    tq.set_search_path(args.search_path)  # the timed batches' scans (AUTO unless asked)
     for B in batches:
         nbatches = max(1, len(Qpool) // B)
         ws = torch.empty(tq.search_workspace(B, n, d, bits, k), dtype=torch.uint8, device=dev)
@@ -464,7 +465,8 @@ def run_ours(args, cfg, rank, world):
         scan_ms = statistics.mean(a.elapsed_time(b) for a, b in evs)
         qps = B * args.steps * world / (ms / 1e3)
         alg_bytes = n * (d * bits // 8 + 4)
-        mma = B >= MMA_MIN_BATCH and bits in (2, 3, 4, 8) and k <= 64
+        mma = bits in (2, 4, 8, 3) and k <= 64 and (args.search_path == "mma" or
+                                                    (args.search_path == "auto" and B >= MMA_MIN_BATCH))
         if mma:
             # tensor-core scan: 2*n*d*B flops per launch against the dense fp16/bf16
             # peak (same rate); each launch is a few ms, timed alone: the burst figure
@@ -482,9 +484,14 @@ def run_ours(args, cfg, rank, world):
             # lookup scan (with its last CTA's merge): the corpus, codes + scales,
             # read once per launch
             achieved = alg_bytes / (scan_ms / 1e3) / 1e9
-            kern = lookup_kernel(bits, n, d, k)
-            if kern == "k_scan_stream" and bits == 4:
-                traffic = recorded_traffic("paper_2607_16973_gb300/csrc/tq_scan.cu", "k_scan_stream_250k_batch1.md",
+            kern = "k_scan_fold" if args.search_path == "lut_fold" else lookup_kernel(bits, n, d, k)
+            if kern == "k_scan_fold":
+                traffic = recorded_traffic(("paper_2607_16973_gb300/csrc/tq_fold.cu",
+                                            "paper_2607_16973_gb300/csrc/tq_topk.cuh"), "k_scan_fold_250k_batch1.md",
+                                           scale_to=n)
+            elif kern == "k_scan_stream" and bits == 4 and args.search_path == "auto":
+                traffic = recorded_traffic(("paper_2607_16973_gb300/csrc/tq_scan.cu",
+                                            "paper_2607_16973_gb300/csrc/tq_topk.cuh"), "k_scan_stream_250k_batch1.md",
                                            scale_to=n)
             else:
                 traffic = None
@@ -537,6 +544,7 @@ def run_ours(args, cfg, rank, world):
             f"= {achieved:.0f} GB/s ({100 * achieved / pk['hbm_gbs']:.1f}% of {pk['source']} HBM)")
         del ws
 
+    tq.set_search_path("auto")
     # Recall@k of both scan paths on the same queries
     recall = {"k": k, "queries": nrec,
               "exact": "float32 brute force over the unquantised normalised corpus"}
@@ -583,6 +591,7 @@ def run_ours(args, cfg, rank, world):
         "data": "synthetic (seeded Gaussian-mixture corpus, perturbed-corpus queries)",
         "config": arm_config(args, n, d, bits, k, head, world),
         "roofline": r["roofline"], "clocks": r["clocks"], "e2e": r["e2e"],
+        "search_path": args.search_path,
         "recall": recall,
         "rag_quality": rag,
         "gpu_launches": r["gpu_launches"],
@@ -1137,6 +1146,8 @@ def main():
                     help="code width for the scale/c2/tiny/prof workloads (default: 4)")
     ap.add_argument("--ref-sample", type=int, default=50_000, help="corpus rows the oracle scans per step")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--search-path", default="auto", choices=["auto", "lut", "lut_fixed", "lut_fold", "mma"],
+                    help="scan kernels of the timed batches (tq_set_search_path; default: AUTO)")
     ap.add_argument("--no-extras", action="store_true",
                     help="scale workload only: skip the 100K, filtered and bit-width sweep lines under 'extra'")
     args = ap.parse_args()
