@@ -398,8 +398,9 @@ tq_status tq_idmap_import(tq_idmap* m, const uint64_t* ext_ids, const uint32_t* 
  * a serving loop that must not call cudaMalloc, which can block, synchronise
  * the device or fail under memory pressure mid-request).  The paper has no
  * counterpart: it is an interface convenience of this library.
- * Same arguments and results as tq_search (always the lookup scan), minus
- * workspace/ws_bytes.  Its scratch is one 8 MiB device array per GPU; the
+ * Same arguments and results as tq_search (always the lookup scan: the
+ * byte-pair one, or the fixed-point table under TQ_PATH_LUT_FIXED; never the
+ * query-folded one), minus workspace/ws_bytes.  Its scratch is one 8 MiB device array per GPU; the
  * call allocates nothing.  Sizes whose scratch (about nq*d*4 bytes of rotated
  * queries plus nq*k*8 bytes per scan CTA of candidates) exceeds 8 MiB return
  * TQ_EINVAL with the byte counts.  The first call on each device looks the
