@@ -201,6 +201,10 @@ def test_invalid_arguments_rejected_without_gpu(lib):
     assert lib.tq_debug_bounded_wait(5_000_000_000, p, null) == _lib.TQ_EINVAL
     assert lib.tq_debug_bounded_wait(1000, null, null) == _lib.TQ_EINVAL
     assert lib.tq_set_search_path(7) == _lib.TQ_EINVAL
+    assert lib.tq_set_search_path(-1) == _lib.TQ_EINVAL
+    for name, path in _lib.PATHS.items():  # every named path is accepted (auto last)
+        assert lib.tq_set_search_path(path) == _lib.TQ_OK, name
+    assert lib.tq_set_search_path(_lib.PATHS["auto"]) == _lib.TQ_OK
     assert lib.tq_profile_events(p, null) == _lib.TQ_EINVAL
 
 
