@@ -74,11 +74,11 @@ enum { TQ_SCALE_NORM = 0, TQ_SCALE_NONE = 1, TQ_SCALE_UNBIASED = 2 };
  * weighted by the rotated query, about 2.5e-7 rms for unit queries).  It
  * moves half the shared-memory bytes of the exact fp32 table per code but
  * needs more instructions per code.  LUT_FOLD is the lookup scan for 4-bit
- * codes (d >= 256, k <= 32) with the rotated query folded into one float32
- * table per packed-byte position, T_m[x] = q'_2m c[x & 15] + q'_2m+1 c[x >> 4]
- * (Sec. II-B step 5): one 4-byte lookup and one add per packed byte, built
- * 256 coordinates at a time; TQ_EUNSUPPORTED where it does not apply.  AUTO
- * does not pick it: the byte-pair scan is faster on GB300. */
+ * codes (d >= 256, k <= 32, n < 2^31 - 13312) with the rotated query folded
+ * into one float32 table per packed-byte position, T_m[x] = q'_2m c[x & 15]
+ * + q'_2m+1 c[x >> 4] (Sec. II-B step 5): one 4-byte lookup and one add per
+ * packed byte, built 256 coordinates at a time; TQ_EUNSUPPORTED where it does
+ * not apply.  AUTO does not pick it: the byte-pair scan is faster on GB300. */
 enum { TQ_PATH_AUTO = 0, TQ_PATH_LUT = 1, TQ_PATH_MMA = 2, TQ_PATH_LUT_FIXED = 3, TQ_PATH_LUT_FOLD = 4 };
 
 typedef struct tq_filter tq_filter; /* opaque, library-owned */

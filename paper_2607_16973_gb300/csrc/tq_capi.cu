@@ -45,7 +45,7 @@ SearchPlan plan_search(int64_t nq, int64_t n, int d, int bits, int k, const tq_f
   p.grid_lut = scan_lut_grid_x(nq, n, k, bits, d);
   const bool mma = mma_supported(bits, d, k);
   p.grid_mma = mma ? scan_mma_grid_x(nq, n, k, bits) : 0;
-  p.grid_fold = fold_supported(bits, d, k) ? scan_fold_grid_x(nq, n) : 0;
+  p.grid_fold = fold_supported(bits, d, k, n) ? scan_fold_grid_x(nq, n) : 0;
   const int per_query = std::max(std::max(p.grid_lut, p.grid_mma), p.grid_fold) * k;
   size_t off = 0;
   p.off_status = off;
@@ -424,9 +424,10 @@ extern "C" tq_status tq_search_ex(const float* Q, int64_t nq, int d, const float
     return fail(TQ_EUNSUPPORTED, "tq_search: the tensor-core scan needs bits 2/4/8, d %% 64 == 0 and k <= %d",
                 tq::kMaxKMma);
   const bool use_mma = can_mma && (path == TQ_PATH_MMA || (path == TQ_PATH_AUTO && nq >= tq::kMmaMinBatch));
-  const bool can_fold = tq::fold_supported(bits, d, k);
+  const bool can_fold = tq::fold_supported(bits, d, k, n);
   if (path == TQ_PATH_LUT_FOLD && !can_fold)
-    return fail(TQ_EUNSUPPORTED, "tq_search: the query-folded scan needs bits 4, d >= 256 and k <= %d",
+    return fail(TQ_EUNSUPPORTED,
+                "tq_search: the query-folded scan needs bits 4, d >= 256, k <= %d and n < 2^31 - 13312",
                 tq::kFoldMaxK);
   // AUTO keeps the byte-pair scan: on GB300 it is the faster of the two (218
   // against 228 us per query at 999,000 x 1536)

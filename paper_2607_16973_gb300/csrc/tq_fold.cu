@@ -348,8 +348,10 @@ int fold_list_p(int k) {
 
 }  // namespace
 
-bool fold_supported(int bits, int d, int k) {
-  return bits == 4 && d >= 2 * FOLD_SLICE && d % 32 == 0 && k >= 1 && k <= kFoldMaxK;
+bool fold_supported(int bits, int d, int k, int64_t n) {
+  // rows are int32 in the kernel; a pass start p0 + FOLD_ROWS must not overflow
+  return bits == 4 && d >= 2 * FOLD_SLICE && d % 32 == 0 && k >= 1 && k <= kFoldMaxK &&
+         n <= (int64_t)INT32_MAX - 2 * FOLD_ROWS;
 }
 
 int scan_fold_grid_x(int64_t nq, int64_t n) {
@@ -368,7 +370,7 @@ cudaError_t launch_scan_fold(const float* qrot, int64_t nq, int d, const float* 
                              float* out_scores, const float* bias, cudaStream_t s, cudaEvent_t ev0,
                              cudaEvent_t ev1) {
   if (nq == 0) return cudaSuccess;
-  if (!fold_supported(4, d, k) || n < 1 || grid_x < 1) return cudaErrorInvalidValue;
+  if (!fold_supported(4, d, k, n) || n < 1 || grid_x < 1) return cudaErrorInvalidValue;
   PFN_cuTensorMapEncodeTiled_v12000 enc = get_encode_fn();
   if (!enc) return cudaErrorNotSupported;
   CUtensorMap map;

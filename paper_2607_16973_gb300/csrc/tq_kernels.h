@@ -95,9 +95,9 @@ cudaError_t launch_scan_lut(const float* qrot, int64_t nq, int d, const float* c
 
 // The 4-bit lookup scan with the rotated query folded into per-byte-position
 // tables (k_scan_fold): bits 4, d >= 256 and a multiple of 32, k <= kFoldMaxK,
-// codes 16-byte aligned.  Arguments and results as launch_scan_lut; grid_x
-// from scan_fold_grid_x.
-bool fold_supported(int bits, int d, int k);
+// codes 16-byte aligned, n below 2^31 less two passes.  Arguments and
+// results as launch_scan_lut; grid_x from scan_fold_grid_x.
+bool fold_supported(int bits, int d, int k, int64_t n);
 int scan_fold_grid_x(int64_t nq, int64_t n);
 cudaError_t launch_scan_fold(const float* qrot, int64_t nq, int d, const float* centroids, const uint8_t* codes,
                              const float* scale, int64_t n, const uint32_t* del, const FilterDev* f,
