@@ -163,7 +163,8 @@ k_scan_fold(const __grid_constant__ CUtensorMap tmap, const float* __restrict__ 
   const int row0 = (int)min((int64_t)blockIdx.x * rows_per_cta, (int64_t)n);
   const int row1 = (int)min((int64_t)row0 + rows_per_cta, (int64_t)n);
   const uint32_t* bm = FILT ? bmask + (size_t)q * mask_words : nullptr;
-  // a tile (32 rows from a multiple of 32) lies in one filter block of 32 or 64
+  // a sub-tile (FOLD_SUB rows from a multiple of FOLD_SUB) and a 32-row group
+  // (from a multiple of 32) each lie in one filter block of 32 or 64 rows
   auto tile_on = [&](int r) -> bool {
     if constexpr (FILT) {
       const int fb = r / fblock;
@@ -175,7 +176,7 @@ k_scan_fold(const __grid_constant__ CUtensorMap tmap, const float* __restrict__ 
   };
   auto ntiles_of = [&](int p0) { return (min(FOLD_ROWS, row1 - p0) + FOLD_SUB - 1) / FOLD_SUB; };
   // this warp's sub-tiles in the order it scores them: pass, slice, sub-tile
-  // t = warp + 8i; advances `c` to the next one (false past the last)
+  // t = warp + FOLD_CW i; advances `c` to the next one (false past the last)
   auto next_tile = [&](FoldCursor& c) -> bool {
     for (;;) {
       if (c.p0 >= row1) return false;
@@ -203,7 +204,7 @@ k_scan_fold(const __grid_constant__ CUtensorMap tmap, const float* __restrict__ 
     li[i] = INT_MAX;
   }
   __syncwarp();
-  // lane 0 of each warp streams the warp's own tiles: the next FOLD_NS into
+  // lane 0 of each warp streams the warp's own sub-tiles: the next FOLD_NS into
   // its stages, and FOLD_PF further ones into L2 ahead of them; the codes are
   // the caller's, so (unfiltered) this starts while the rotation may still run
   FoldCursor ic{row0, 0, -1}, pc{row0, 0, -1};
